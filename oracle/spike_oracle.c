@@ -1,0 +1,149 @@
+/*
+ * spike_oracle.c -- plain, slow, single-threaded CPU oracle for the
+ * spike-gated INT8 projection of Section 2.3, Eq. (sparse).
+ *
+ * TEST INFRASTRUCTURE ONLY: used by the test suite, the smoke check and the
+ * CPU-baseline leg of the benchmark.  It is never linked into, loaded by or
+ * called from the CUDA library, and includes none of its headers.
+ *
+ * The method reaches exactly the value of the definition (integer sums are
+ * order-free and the accumulator never leaves the INT32 range for K <= 2^24
+ * / 128), so this file writes the definition out and nothing else:
+ *
+ *   1. A = { k : x_k = 1 }, ascending                       (Section 2.2)
+ *   2. acc_m = sum_{k in A} Q_{m,k},  Q_{m,k} = Q[k*ldq + m] (Eq. sparse,
+ *      column-major storage of Section 2.2), in int64, then checked to fit
+ *      INT32, the paper's accumulator width (Section 2.3)
+ *   3. y_m = s_m * (float)acc_m: one conversion to FP32 and one FP32
+ *      multiply per output channel (Section 2.3).  Built with
+ *      -ffp-contract=off; there is nothing to contract anyway.
+ *
+ * Parity pins for this file live in the test suite: dense integer matmul
+ * (numpy) on tiny and full shapes, exhaustive masks on tiny K, hand-worked
+ * fixtures, invariants (zero, one-hot, additivity, all-ones, permutation,
+ * format equivalence) and closed forms.
+ */
+#include "spike_oracle.h"
+
+#include <stdlib.h>
+
+/* Spike x_k of one row: 1 if column k fires, else 0 (Section 1: x in {0,1}^K;
+ * any nonzero byte counts as a spike in the U8 format). */
+static int spike_at(const void *row, int fmt, int32_t k)
+{
+    if (fmt == SP_ORACLE_BITS32) {
+        const uint32_t *w = (const uint32_t *)row;
+        return (int)((w[k / 32] >> (k % 32)) & 1u);
+    }
+    return ((const uint8_t *)row)[k] != 0;
+}
+
+static const void *spike_row(const void *spikes, int fmt, int64_t ld_spikes,
+                             int32_t t)
+{
+    int64_t elem = (fmt == SP_ORACLE_BITS32) ? 4 : 1;
+    return (const uint8_t *)spikes + (int64_t)t * ld_spikes * elem;
+}
+
+static int check_args(const int8_t *Q, int64_t ldq, int32_t N, int32_t K,
+                      const void *spikes, int fmt, int64_t ld_spikes, int32_t T)
+{
+    if (!Q || !spikes || N < 0 || K < 0 || T < 0 || ldq < N)
+        return -1;
+    if (fmt != SP_ORACLE_BITS32 && fmt != SP_ORACLE_U8)
+        return -1;
+    if (T > 1) {
+        int64_t need = (fmt == SP_ORACLE_BITS32) ? ((int64_t)K + 31) / 32 : K;
+        if (ld_spikes < need)
+            return -1;
+    }
+    return 0;
+}
+
+int sp_oracle_active_set(const void *spikes, int fmt, int32_t K,
+                         int32_t *idx, int32_t *count)
+{
+    if (!spikes || !idx || !count || K < 0)
+        return -1;
+    if (fmt != SP_ORACLE_BITS32 && fmt != SP_ORACLE_U8)
+        return -1;
+    int32_t n = 0;
+    for (int32_t k = 0; k < K; ++k)
+        if (spike_at(spikes, fmt, k))
+            idx[n++] = k;
+    *count = n;
+    return 0;
+}
+
+/* Steps 2 and 3 for one output channel m, given the active set A. */
+static int project_one(const int8_t *Q, int64_t ldq, const float *s,
+                       int32_t m, const int32_t *A, int32_t nA,
+                       int32_t *acc_out, float *y_out)
+{
+    int64_t acc = 0;
+    for (int32_t i = 0; i < nA; ++i)
+        acc += Q[(int64_t)A[i] * ldq + m];
+    if (acc > INT32_MAX || acc < INT32_MIN)
+        return -2;
+    int32_t acc32 = (int32_t)acc;
+    if (acc_out)
+        *acc_out = acc32;
+    if (y_out)
+        *y_out = s[m] * (float)acc32;
+    return 0;
+}
+
+int sp_oracle_project(const int8_t *Q, int64_t ldq, const float *s,
+                      int32_t N, int32_t K,
+                      const void *spikes, int fmt, int64_t ld_spikes, int32_t T,
+                      int32_t *acc, float *y)
+{
+    int rc = check_args(Q, ldq, N, K, spikes, fmt, ld_spikes, T);
+    if (rc)
+        return rc;
+    if (y && !s)
+        return -1;
+    int32_t *A = (int32_t *)malloc(sizeof(int32_t) * (size_t)(K > 0 ? K : 1));
+    if (!A)
+        return -3;
+    for (int32_t t = 0; t < T && rc == 0; ++t) {
+        int32_t nA = 0;
+        sp_oracle_active_set(spike_row(spikes, fmt, ld_spikes, t), fmt, K, A, &nA);
+        for (int32_t m = 0; m < N && rc == 0; ++m)
+            rc = project_one(Q, ldq, s, m, A, nA,
+                             acc ? &acc[(int64_t)t * N + m] : NULL,
+                             y ? &y[(int64_t)t * N + m] : NULL);
+    }
+    free(A);
+    return rc;
+}
+
+int sp_oracle_project_entries(const int8_t *Q, int64_t ldq, const float *s,
+                              int32_t N, int32_t K,
+                              const void *spikes, int fmt, int64_t ld_spikes,
+                              int32_t T, int64_t count,
+                              const int32_t *t_idx, const int32_t *m_idx,
+                              int32_t *acc, float *y)
+{
+    int rc = check_args(Q, ldq, N, K, spikes, fmt, ld_spikes, T);
+    if (rc)
+        return rc;
+    if (count < 0 || (count > 0 && (!t_idx || !m_idx)) || (y && !s))
+        return -1;
+    int32_t *A = (int32_t *)malloc(sizeof(int32_t) * (size_t)(K > 0 ? K : 1));
+    if (!A)
+        return -3;
+    for (int64_t e = 0; e < count && rc == 0; ++e) {
+        int32_t t = t_idx[e], m = m_idx[e];
+        if (t < 0 || t >= T || m < 0 || m >= N) {
+            rc = -1;
+            break;
+        }
+        int32_t nA = 0;
+        sp_oracle_active_set(spike_row(spikes, fmt, ld_spikes, t), fmt, K, A, &nA);
+        rc = project_one(Q, ldq, s, m, A, nA,
+                         acc ? &acc[e] : NULL, y ? &y[e] : NULL);
+    }
+    free(A);
+    return rc;
+}

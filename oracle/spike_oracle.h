@@ -1,0 +1,69 @@
+/*
+ * spike_oracle.h -- CPU oracle for the spike-gated INT8 projection.
+ *
+ * TEST INFRASTRUCTURE ONLY.  Nothing in the product path links, loads or
+ * calls this code: only the test suite, the smoke check and the CPU-baseline
+ * leg of the benchmark do.  It shares no source with the CUDA library.
+ *
+ * What it computes (Section 2.3, Eq. (sparse)):
+ *
+ *     A   = { k : x_k = 1 }                       (Section 2.2, active set)
+ *     y_m = s_m * sum_{k in A} Q_{m,k}             (Eq. sparse)
+ *
+ * with Q an INT8 matrix of M = N output channels by K input columns, stored
+ * column-major (Section 2.2: "each selected column is a contiguous read across
+ * output channels"), so element (m, k) lives at Q[k * ldq + m]; s the FP32
+ * per-output-channel scale (Section 2.3 quantiser); x a binary spike vector.
+ * The sum is held in a 64-bit integer, range-checked and narrowed to INT32
+ * (the paper's general accumulator is INT32, Section 2.3), converted to FP32
+ * and multiplied by s_m once (Section 2.3: "converted to FP32 and scaled once
+ * per output channel").
+ *
+ * Spike formats: SP_ORACLE_U8 -- one byte per column, any nonzero byte is a
+ * spike; SP_ORACLE_BITS32 -- uint32 words, column k is bit (k % 32) of word
+ * (k / 32), bits at or beyond K are ignored.
+ *
+ * All functions are single-threaded, allocate only O(K) scratch, and return
+ * 0 on success, a negative code on a bad argument (-1) or an INT32 overflow of
+ * the accumulator (-2), and -3 if scratch allocation fails.
+ */
+#ifndef SPIKE_ORACLE_H
+#define SPIKE_ORACLE_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+enum { SP_ORACLE_BITS32 = 0, SP_ORACLE_U8 = 1 };
+
+/* Active index set A of one spike row, ascending.  idx must hold K entries;
+ * *count receives |A|.  ld-free: spikes points at the row itself. */
+int sp_oracle_active_set(const void *spikes, int fmt, int32_t K,
+                         int32_t *idx, int32_t *count);
+
+/* Eq. (sparse) for T spike rows.  Row t of the spikes starts at
+ * (const uint8_t*)spikes + t * ld_spikes * (fmt == BITS32 ? 4 : 1), i.e.
+ * ld_spikes counts words for BITS32 and bytes for U8.  Outputs are dense
+ * [T][N]: acc[t*N + m], y[t*N + m].  Either output may be NULL. */
+int sp_oracle_project(const int8_t *Q, int64_t ldq, const float *s,
+                      int32_t N, int32_t K,
+                      const void *spikes, int fmt, int64_t ld_spikes, int32_t T,
+                      int32_t *acc, float *y);
+
+/* Eq. (sparse) at selected outputs only: entry e is token row t_idx[e],
+ * output channel m_idx[e].  For checks at sizes where the full product is
+ * too slow for a single CPU thread. */
+int sp_oracle_project_entries(const int8_t *Q, int64_t ldq, const float *s,
+                              int32_t N, int32_t K,
+                              const void *spikes, int fmt, int64_t ld_spikes,
+                              int32_t T, int64_t count,
+                              const int32_t *t_idx, const int32_t *m_idx,
+                              int32_t *acc, float *y);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* SPIKE_ORACLE_H */

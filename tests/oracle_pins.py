@@ -1,0 +1,205 @@
+"""Pins for the CPU oracle: checks against facts fixed by the paper and by
+arithmetic, not by the oracle itself.
+
+Each ``pin_*`` takes an ``oracle.Oracle`` and raises ``AssertionError`` when
+the oracle disagrees.  ``test_oracle_pins.py`` runs them on the real oracle;
+``test_oracle_mutants.py`` runs them on copies of the oracle with one planted
+mistake each and requires every copy to fail at least one pin.
+
+What pins what (Section 2.3, Eq. sparse: y_m = s_m * sum_{k in A} Q_{m,k}):
+
+* hand-worked fixture (tests/golden/hand_worked.json) -- values worked out by
+  hand from the equation;
+* exhaustive masks and full shapes -- the sum over A equals the dense
+  integer product Q x for binary x (numpy int64 matmul, a library routine);
+* the scale -- one FP32 multiply of an exactly converted integer is the
+  correctly rounded exact product (fp64 holds acc*s exactly: 24 + 24 bits);
+* invariants -- zero spikes, one-hot, additivity over disjoint sets,
+  all-ones row sums, column permutation, format equivalence, tail bits,
+  nonzero bytes;
+* closed forms -- constant Q, INT8 extremes, INT32 overflow reported.
+"""
+from __future__ import annotations
+
+import json
+from pathlib import Path
+
+import numpy as np
+
+from paper_2606_03026_gb300 import synth
+
+GOLDEN = Path(__file__).resolve().parent / "golden"
+
+
+def logical(Qc: np.ndarray, N: int) -> np.ndarray:
+    """Logical [N, K] view of column-major storage [K, ldq]."""
+    return np.asarray(Qc)[:, :N].T.astype(np.int64)
+
+
+def dense_ref(Qc, N, x_u8):
+    """Dense integer product Q x for each binary row of x (numpy int64)."""
+    return (np.asarray(x_u8, dtype=np.int64) != 0).astype(np.int64) @ logical(Qc, N).T
+
+
+def f32_bits(a):
+    return np.asarray(a, dtype=np.float32).view(np.uint32)
+
+
+def exact_scaled(acc, s):
+    """Correctly rounded fp32 of the exact product acc * s (fp64 is exact
+    here: |acc| < 2^24 and s has a 24-bit significand)."""
+    return (np.asarray(acc, np.float64) * np.asarray(s, np.float32).astype(np.float64)).astype(np.float32)
+
+
+# --------------------------------------------------------------------------
+def pin_hand_fixture(orc):
+    g = json.loads((GOLDEN / "hand_worked.json").read_text())
+    N, K, ldq = g["N"], g["K"], g["ldq"]
+    rows = np.array(g["Q_logical_rows_m_by_k"], dtype=np.int64)
+    Qc = np.full((K, ldq), g["pad_byte"], dtype=np.int8)
+    Qc[:, :N] = rows.T.astype(np.int8)
+    s = np.array(g["scale"], dtype=np.float32)
+    for case in g["cases"]:
+        want_acc = np.array(case["acc"], dtype=np.int32)
+        want_y = np.array(case["y"], dtype=np.float32)
+        x = np.array(case["x_u8"], dtype=np.uint8)
+        bits = np.array([case["bits_word_with_tail_garbage"]], dtype=np.uint32)
+        for sp, fmt in ((x, "u8"), (bits, "bits")):
+            acc, y = orc.project(Qc, s, N, K, sp, fmt, ldq=ldq)
+            assert np.array_equal(acc[0], want_acc), (case["name"], fmt, acc)
+            assert np.array_equal(f32_bits(y[0]), f32_bits(want_y)), (case["name"], fmt, y)
+        if "y_sign_bits" in case:
+            assert list((f32_bits(y[0]) >> 31).astype(int)) == case["y_sign_bits"]
+        want_A = np.flatnonzero(x)
+        assert np.array_equal(orc.active_set(x, "u8", K), want_A)
+        assert np.array_equal(orc.active_set(bits, "bits", K), want_A)
+
+
+def pin_exhaustive_small(orc):
+    # N != K and ldq > N so a transposed operand or a dropped ldq shows.
+    N, K, ldq = 5, 10, 7
+    Qc, s, _ = synth.random_case(11, N, K, ldq=ldq)
+    masks = ((np.arange(2 ** K)[:, None] >> np.arange(K)[None, :]) & 1).astype(np.uint8)
+    acc, y = orc.project(Qc, s, N, K, masks, "u8", ldq=ldq)
+    assert np.array_equal(acc.astype(np.int64), dense_ref(Qc, N, masks))
+    acc_b, _ = orc.project(Qc, s, N, K, synth.pack_bits(masks), "bits", ldq=ldq)
+    assert np.array_equal(acc_b, acc)
+
+
+def pin_full_shapes(orc):
+    for (N, K, p, seed) in ((1536, 1536, 0.1, 1), (1536, 6144, 0.2, 2),
+                            (1536, 6144, 0.5, 3)):
+        Qc, s, x = synth.random_case(seed, N, K, T=3, p=p)
+        acc, y = orc.project(Qc, s, N, K, x, "u8")
+        assert np.array_equal(acc.astype(np.int64), dense_ref(Qc, N, x))
+        assert np.array_equal(f32_bits(y), f32_bits(exact_scaled(acc, s[None, :])))
+
+
+def pin_scale_rounding(orc):
+    N, K = 64, 300
+    rng = synth.rng_for(77)
+    Qc = rng.integers(-128, 128, size=(K, N)).astype(np.int8)
+    # scales with full 24-bit significands over a wide exponent range, both signs
+    s = (rng.uniform(1, 2, N) * 2.0 ** rng.integers(-30, 30, N)
+         * rng.choice([-1.0, 1.0], N)).astype(np.float32)
+    x = synth.bernoulli(rng, (4, K), 0.6)
+    x[0] = 0                          # zero sums: signed zeros
+    acc, y = orc.project(Qc, s, N, K, x, "u8")
+    assert np.array_equal(f32_bits(y), f32_bits(exact_scaled(acc, s[None, :])))
+    assert np.all((f32_bits(y[0]) >> 31) == (f32_bits(s) >> 31))
+
+
+def pin_invariants(orc):
+    N, K, ldq = 48, 200, 64
+    Qc, s, x = synth.random_case(5, N, K, T=2, p=0.3, ldq=ldq)
+    L = logical(Qc, N)
+    # zero spikes -> zero accumulators
+    acc0, _ = orc.project(Qc, s, N, K, np.zeros(K, np.uint8), "u8", ldq=ldq)
+    assert not acc0.any()
+    # one-hot e_k -> column k and y = s * float(column)
+    for k in (0, 1, 31, 32, 100, K - 1):
+        e = np.zeros(K, np.uint8)
+        e[k] = 1
+        acc, y = orc.project(Qc, s, N, K, e, "u8", ldq=ldq)
+        assert np.array_equal(acc[0], L[:, k]), k
+        assert np.array_equal(f32_bits(y[0]), f32_bits(s * L[:, k].astype(np.float32)))
+    # additivity over disjoint active sets
+    a = x[0] & (np.arange(K) % 2 == 0)
+    b = x[1] & (np.arange(K) % 2 == 1)
+    acc_ab, _ = orc.project(Qc, s, N, K, (a | b)[None], "u8", ldq=ldq)
+    acc_a, _ = orc.project(Qc, s, N, K, a[None], "u8", ldq=ldq)
+    acc_b, _ = orc.project(Qc, s, N, K, b[None], "u8", ldq=ldq)
+    assert np.array_equal(acc_ab, acc_a + acc_b)
+    # all ones -> row sums
+    acc1, _ = orc.project(Qc, s, N, K, np.ones(K, np.uint8), "u8", ldq=ldq)
+    assert np.array_equal(acc1[0], L.sum(axis=1))
+    # permuting columns of Q together with x changes nothing
+    perm = synth.rng_for(6).permutation(K)
+    accp, _ = orc.project(np.ascontiguousarray(Qc[perm]), s, N, K, x[:, perm], "u8", ldq=ldq)
+    accx, yx = orc.project(Qc, s, N, K, x, "u8", ldq=ldq)
+    assert np.array_equal(accp, accx)
+    # bits == u8; tail bits past K ignored; any nonzero byte is a spike
+    bits = synth.pack_bits(x)
+    bits[:, -1] |= np.uint32(0xFFFFFFFF) << np.uint32(K % 32)
+    accb, yb = orc.project(Qc, s, N, K, bits, "bits", ldq=ldq)
+    assert np.array_equal(accb, accx) and np.array_equal(f32_bits(yb), f32_bits(yx))
+    xv = x * synth.rng_for(8).integers(1, 256, size=x.shape).astype(np.uint8)
+    accv, _ = orc.project(Qc, s, N, K, xv, "u8", ldq=ldq)
+    assert np.array_equal(accv, accx)
+    # rows are independent: a batch equals its rows one at a time
+    for t in range(x.shape[0]):
+        acct, _ = orc.project(Qc, s, N, K, x[t], "u8", ldq=ldq)
+        assert np.array_equal(acct[0], accx[t])
+    # active set is the ascending list of firing columns
+    assert np.array_equal(orc.active_set(x[0], "u8", K), np.flatnonzero(x[0]))
+    assert np.array_equal(orc.active_set(bits[0], "bits", K), np.flatnonzero(x[0]))
+
+
+def pin_closed_forms(orc):
+    N, K = 32, 4096
+    x = synth.bernoulli(synth.rng_for(9), (3, K), 0.25)
+    x[2] = 1
+    nA = x.astype(np.int64).sum(axis=1)
+    s = np.ones(N, np.float32)
+    for c in (1, -1, 127, -127, -128, 0, 5):
+        Qc = np.full((K, N), c, dtype=np.int8)
+        acc, y = orc.project(Qc, s, N, K, x, "u8")
+        assert np.array_equal(acc, np.repeat((c * nA)[:, None], N, 1).astype(np.int32)), c
+        assert np.array_equal(y, acc.astype(np.float32))
+
+
+def pin_overflow_reported(orc):
+    # -128 * (2^24 + 1) = -2^31 - 128 does not fit INT32: must be an error,
+    # never a wrapped value.
+    K = (1 << 24) + 1
+    Qc = np.full((K, 1), -128, dtype=np.int8)
+    x = np.ones(K, np.uint8)
+    try:
+        orc.project(Qc, np.ones(1, np.float32), 1, K, x, "u8")
+    except RuntimeError:
+        pass
+    else:
+        raise AssertionError("INT32 overflow not reported")
+    # the largest sum that fits is exact
+    K2 = (1 << 24)
+    acc, _ = orc.project(Qc[:K2], np.ones(1, np.float32), 1, K2, x[:K2], "u8")
+    assert acc[0, 0] == -(1 << 31)
+
+
+def pin_entries(orc):
+    N, K, T = 96, 333, 5
+    Qc, s, x = synth.random_case(12, N, K, T=T, p=0.2, ldq=112)
+    acc, y = orc.project(Qc, s, N, K, x, "u8", ldq=112)
+    rng = synth.rng_for(13)
+    t = rng.integers(0, T, 200)
+    m = rng.integers(0, N, 200)
+    ae, ye = orc.project_entries(Qc, s, N, K, x, "u8", t, m, ldq=112)
+    assert np.array_equal(ae, acc[t, m])
+    assert np.array_equal(f32_bits(ye), f32_bits(y[t, m]))
+    be, _ = orc.project_entries(Qc, s, N, K, synth.pack_bits(x), "bits", t, m, ldq=112)
+    assert np.array_equal(be, ae)
+
+
+ALL_PINS = [pin_hand_fixture, pin_exhaustive_small, pin_full_shapes,
+            pin_scale_rounding, pin_invariants, pin_closed_forms,
+            pin_overflow_reported, pin_entries]
