@@ -1,0 +1,227 @@
+/*
+ * spike_proj.h -- C ABI of libspikeproj.so: the spike-gated INT8 projection
+ * on NVIDIA GB300 (sm_103a).
+ *
+ * Operation (Section 2.3, Eq. (sparse); Section 2.2 for the layout):
+ *
+ *     A     = { k : x_k = 1 }                 active columns of one spike row
+ *     acc_m = sum_{k in A} Q_{m,k}            INT32, exact
+ *     y_m   = s_m * (float)acc_m              one FP32 multiply, round to
+ *                                             nearest even, per output m
+ *
+ *   Q   INT8 weights of N outputs by K inputs, COLUMN-MAJOR: element (m, k)
+ *       at W[k * ldw + m], so each active column is one contiguous read of N
+ *       bytes across the output channels (Section 2.2).
+ *   s   FP32 scale per output channel, length N (Section 2.3 quantiser).
+ *   x   binary spikes, one row per token, in one of two formats (sp_fmt).
+ *
+ * Only the active columns are read on the gather paths; the dense
+ * tensor-core path (SP_GEMM) reads all of Q and is chosen only where the
+ * measured density makes that cheaper.  Every path produces the same INT32
+ * accumulators bit for bit, and therefore the same FP32 outputs.
+ *
+ * Conventions for every call
+ *   - Pointers named d_* or documented as "device" are CUDA device pointers
+ *     on the current device; the caller owns them.  A plan BORROWS W and the
+ *     scale: they must stay allocated and unchanged while the plan lives.
+ *   - Calls are asynchronous on `stream` (a cudaStream_t; NULL = the legacy
+ *     default stream) unless documented otherwise.  Argument errors are
+ *     detected on the host and returned before anything is enqueued.
+ *   - Nothing aborts, traps or spins without bound.  Kernel-side failures set
+ *     an error word read by spike_proj_plan_status / spike_proj_group_status.
+ *   - A plan or group owns workspace that its kernels leave zeroed for the
+ *     next call; calls on one plan (or group) must not overlap on the GPU:
+ *     use one stream per plan, or order the streams.
+ *   - Exactness bound: |acc| <= 128 * K must stay below 2^24 so that the
+ *     INT32 -> FP32 conversion is exact on every path; hence K <= 131072.
+ */
+#ifndef SPIKE_PROJ_H
+#define SPIKE_PROJ_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define SPIKE_PROJ_ABI_VERSION 1
+#define SPIKE_PROJ_MAX_K 131072        /* 128 * K < 2^24: exact FP32 conversion */
+#define SPIKE_PROJ_MAX_GROUP 64        /* projections per group */
+
+typedef struct sp_plan_s *sp_plan_t;
+typedef struct sp_group_s *sp_group_t;
+typedef void *sp_stream_t;             /* a cudaStream_t */
+
+typedef enum sp_status {
+    SP_OK = 0,
+    SP_EINVAL = 1,        /* NULL where required, size out of range, bad enum */
+    SP_EALIGN = 2,        /* pointer / leading dimension breaks an alignment rule */
+    SP_EDEVICE = 3,       /* current device is not compute capability 10.3 */
+    SP_ECUDA = 4,         /* a CUDA runtime call failed: spike_proj_last_cuda_error() */
+    SP_ENOMEM = 5,        /* workspace allocation failed */
+    SP_ERANGE = 6,        /* K above SPIKE_PROJ_MAX_K, or batch above the plan's max */
+    SP_EKERNEL = 7,       /* a kernel raised the device error word */
+    SP_EUNSUPPORTED = 8   /* strategy not available for this plan (e.g. SP_GEMM
+                             without SP_PLAN_GEMM) */
+} sp_status;
+
+/* Spike row formats.
+ *   SP_SPIKES_BITS32: uint32 words; column k is bit (k % 32) of word (k / 32),
+ *                     least significant bit first; bits at or past K are
+ *                     ignored.  A row holds ceil(K/32) words; row stride
+ *                     (ld_spikes) is counted in words.
+ *   SP_SPIKES_U8:     one byte per column, any nonzero byte is a spike; row
+ *                     stride counted in bytes. */
+typedef enum sp_fmt { SP_SPIKES_BITS32 = 0, SP_SPIKES_U8 = 1 } sp_fmt;
+
+/* Kernel strategies for multi-token calls.
+ *   SP_AUTO    measure the spike density on the device, read it back (one
+ *              stream synchronisation) and pick one of the others.
+ *   SP_GATHER  per-token active-column gather (the batch-1 kernel per row).
+ *   SP_UNION   one fetch of each column in the union of the rows' active sets,
+ *              added into every row whose spike is set.
+ *   SP_GEMM    dense tensor-core contraction over all columns (tcgen05,
+ *              bf16 operands holding the exact integers, fp32 accumulation
+ *              in tensor memory: exact because every partial sum is an
+ *              integer below 2^24). */
+typedef enum sp_kernel {
+    SP_AUTO = 0,
+    SP_GATHER = 1,
+    SP_UNION = 2,
+    SP_GEMM = 3
+} sp_kernel;
+
+/* Plan flags. */
+#define SP_PLAN_GEMM 0x1u  /* also build the tensor-core operand copy of W:
+                              N*K bf16 (2 bytes per weight), owned by the plan */
+
+/* ---------------------------------------------------------------------------
+ * spike_proj_plan -- describe one projection and allocate its workspace.
+ *
+ *   plan       out: the new plan (unchanged on error).
+ *   W          device, INT8, column-major: W[k*ldw + m] for m < N, k < K.
+ *              16-byte aligned.  Borrowed.
+ *   ldw        leading dimension in bytes (elements): ldw >= N, ldw % 16 == 0.
+ *   scale      device, FP32 [N], one scale per OUTPUT channel m (not per
+ *              input column: a [K]-long scale is a layout error the caller
+ *              must not make; Appendix A.2 records that defect).  4-byte
+ *              aligned.  Borrowed.
+ *   N          output channels, 16 <= N, N % 16 == 0.
+ *   K          input columns, 1 <= K <= SPIKE_PROJ_MAX_K (else SP_ERANGE).
+ *   max_batch  largest B / T accepted by spike_proj_batched / _prefill on this
+ *              plan (>= 1; sizes the workspace: 4*N*max_batch bytes, plus
+ *              2*K*max_batch with SP_PLAN_GEMM).
+ *   flags      0 or SP_PLAN_GEMM.
+ *   stream     used for the workspace clear and the operand copy; the call
+ *              synchronises it before returning.
+ * Errors: SP_EINVAL, SP_EALIGN, SP_ERANGE, SP_EDEVICE, SP_ENOMEM, SP_ECUDA.
+ * ------------------------------------------------------------------------- */
+sp_status spike_proj_plan(sp_plan_t *plan, const int8_t *W, int64_t ldw,
+                          const float *scale, int32_t N, int32_t K,
+                          int32_t max_batch, uint32_t flags, sp_stream_t stream);
+
+/* Frees the plan's workspace (synchronises the device).  NULL is a no-op. */
+sp_status spike_proj_plan_destroy(sp_plan_t plan);
+
+/* ---------------------------------------------------------------------------
+ * spike_proj_decode -- one spike row (batch 1), Eq. (sparse).
+ *
+ *   spikes  device, one row in `fmt` (ceil(K/32) words or K bytes); 4-byte
+ *           aligned for SP_SPIKES_BITS32.
+ *   acc     device INT32 [N] or NULL; y device FP32 [N] or NULL (not both
+ *           NULL).  4-byte aligned.
+ * Compacts the row into its active-column list on the device (warp ballot and
+ * popcount) and sums only those columns.  Never reads an inactive column.
+ * ------------------------------------------------------------------------- */
+sp_status spike_proj_decode(sp_plan_t plan, const void *spikes, sp_fmt fmt,
+                            int32_t *acc, float *y, sp_stream_t stream);
+
+/* ---------------------------------------------------------------------------
+ * spike_proj_batched -- B independent spike rows sharing the plan's W.
+ *
+ *   spikes     device, B rows, row b at spikes + b*ld_spikes (words for
+ *              BITS32, bytes for U8); ld_spikes >= ceil(K/32) or >= K.
+ *   B          1 <= B <= plan's max_batch (else SP_ERANGE).
+ *   acc, y     device [B][N] row-major (either may be NULL, not both).
+ *   strategy   SP_AUTO, SP_GATHER, SP_UNION or SP_GEMM (SP_GEMM needs a plan
+ *              made with SP_PLAN_GEMM, else SP_EUNSUPPORTED).
+ * Row b of the result equals spike_proj_decode on row b, bit for bit.
+ * ------------------------------------------------------------------------- */
+sp_status spike_proj_batched(sp_plan_t plan, const void *spikes, sp_fmt fmt,
+                             int32_t B, int64_t ld_spikes, int32_t *acc,
+                             float *y, sp_kernel strategy, sp_stream_t stream);
+
+/* ---------------------------------------------------------------------------
+ * spike_proj_prefill -- T prompt tokens at once: ACC = X Q^T, Y = ACC * s
+ * per column (Eq. (sparse) for every row of X).
+ *
+ *   X          device, uint8 [T][ldx] with X[t][k] nonzero = spike; ldx >= K.
+ *   T          1 <= T <= plan's max_batch.
+ *   acc, y     device [T][N] row-major (either may be NULL, not both).
+ *   strategy   as for spike_proj_batched; SP_AUTO picks SP_GEMM on a plan
+ *              with SP_PLAN_GEMM when the measured density makes the dense
+ *              contraction cheaper than the gathers.
+ * ------------------------------------------------------------------------- */
+sp_status spike_proj_prefill(sp_plan_t plan, const uint8_t *X, int32_t T,
+                             int64_t ldx, int32_t *acc, float *y,
+                             sp_kernel strategy, sp_stream_t stream);
+
+/* Strategy and total active count (sum over rows of |A|) of the last
+ * batched / prefill call with SP_AUTO on this plan; the count is -1 when the
+ * last call did not measure it. */
+sp_status spike_proj_last_dispatch(sp_plan_t plan, sp_kernel *chosen,
+                                   int32_t *active_count);
+
+/* Reads and clears the plan's device error word; synchronises `stream`.
+ * Returns SP_EKERNEL if a kernel raised it (and re-zeroes the workspace),
+ * SP_OK otherwise. */
+sp_status spike_proj_plan_status(sp_plan_t plan, sp_stream_t stream);
+
+/* ---------------------------------------------------------------------------
+ * Groups: several independent batch-1 projections in ONE kernel launch, e.g.
+ * the 44 binary-input projections of one 22-block decode step (per block the
+ * sequence-mixer projection and the feed-forward down projection, Section
+ * 2.1).  All projections of a group run concurrently, so their combined
+ * active-column traffic can fill the memory system.
+ *
+ * spike_proj_group_create: plans[0..count) (1 <= count <= SPIKE_PROJ_MAX_GROUP)
+ *   are borrowed and must outlive the group.  The group owns its own
+ *   workspace (the plans' workspaces are not used by group calls).
+ * ------------------------------------------------------------------------- */
+sp_status spike_proj_group_create(sp_group_t *group, const sp_plan_t *plans,
+                                  int32_t count, sp_stream_t stream);
+sp_status spike_proj_group_destroy(sp_group_t group);
+
+/* spike_proj_group_decode: projection j reads its spike row at
+ *   spikes + j*ld_spikes   (words for BITS32, bytes for U8)
+ * and writes acc + j*ld_out, y + j*ld_out (device; either may be NULL, not
+ * both).  ld_spikes must cover the largest K of the group; ld_out >= the
+ * largest N. */
+sp_status spike_proj_group_decode(sp_group_t group, const void *spikes,
+                                  sp_fmt fmt, int64_t ld_spikes, int32_t *acc,
+                                  float *y, int64_t ld_out, sp_stream_t stream);
+
+/* spike_proj_group_decode_host: the same with HOST buffers (page-locked
+ * memory recommended).  Enqueues on `stream`: the copy of count rows of
+ * spikes into group-owned device staging, the kernel, and the copies of
+ * acc / y back to the host.  Returns once enqueued; the host buffers must
+ * not be touched until `stream` has been synchronised. */
+sp_status spike_proj_group_decode_host(sp_group_t group, const void *h_spikes,
+                                       sp_fmt fmt, int64_t ld_spikes,
+                                       int32_t *h_acc, float *h_y,
+                                       int64_t ld_out, sp_stream_t stream);
+
+/* Reads and clears the group's device error word (synchronises `stream`). */
+sp_status spike_proj_group_status(sp_group_t group, sp_stream_t stream);
+
+/* --------------------------------------------------------------------------- */
+const char *spike_proj_strerror(sp_status status);
+/* cudaError_t code of the last failing CUDA call made by this thread. */
+int spike_proj_last_cuda_error(void);
+int spike_proj_abi_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* SPIKE_PROJ_H */

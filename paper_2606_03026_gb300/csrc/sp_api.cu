@@ -1,0 +1,512 @@
+// sp_api.cu -- the C ABI of libspikeproj.so: argument validation, plans and
+// groups (workspace ownership), per-call dispatch between the gather, union
+// and tensor-core kernels, and status reporting.  See include/spike_proj.h.
+#include <cstdlib>
+#include <cstring>
+#include <new>
+
+#include "sp_gemm.h"
+#include "sp_internal.h"
+
+using namespace sp;
+
+struct sp_plan_s {
+  int device = 0;
+  const int8_t* W = nullptr;
+  int64_t ldw = 0;
+  const float* scale = nullptr;
+  int32_t N = 0, K = 0, max_batch = 0;
+  uint32_t flags = 0;
+  int32_t* ws = nullptr;          // [max_batch][N] INT32, zero between calls
+  uint32_t* tickets = nullptr;    // zero between calls
+  size_t n_tickets = 0;
+  int* err = nullptr;             // device error word
+  int32_t* d_counts = nullptr;    // density probe result [2]
+  int32_t* h_counts = nullptr;    // page-locked copy
+  // tensor-core path
+  __nv_bfloat16* Wb = nullptr;    // [N][Kp] bf16 K-major
+  __nv_bfloat16* Xb = nullptr;    // [xb_rows][Kp] bf16 spike staging
+  int Kp = 0, xb_rows = 0;
+  GemmMaps maps;
+  sp_kernel last_kernel = SP_AUTO;
+  int32_t last_active = -1;
+};
+
+struct sp_group_s {
+  int32_t count = 0;
+  int32_t maxN = 0, maxK = 0;
+  GatherParamsG params;           // problem table, per-call fields filled in
+  int32_t* ws = nullptr;
+  uint32_t* tickets = nullptr;
+  int* err = nullptr;
+  size_t ws_elems = 0, n_tickets = 0;
+  // staging for the host-buffer entry point
+  void* d_spikes = nullptr;       // [count][row bytes]
+  int32_t* d_acc = nullptr;       // [count][maxN]
+  float* d_y = nullptr;           // [count][maxN]
+  size_t spike_row_bytes = 0;
+};
+
+namespace {
+
+thread_local int g_last_cuda_error = 0;
+
+inline sp_status cuda_fail(cudaError_t e) {
+  g_last_cuda_error = (int)e;
+  return SP_ECUDA;
+}
+#define SP_CUDA(call)                              \
+  do {                                             \
+    cudaError_t e_ = (call);                       \
+    if (e_ != cudaSuccess) return cuda_fail(e_);   \
+  } while (0)
+
+inline bool aligned(const void* p, uintptr_t a) {
+  return (reinterpret_cast<uintptr_t>(p) & (a - 1)) == 0;
+}
+inline cudaStream_t as_stream(sp_stream_t s) { return reinterpret_cast<cudaStream_t>(s); }
+inline int64_t words_for(int K) { return ((int64_t)K + 31) / 32; }
+inline int64_t row_elems(sp_fmt fmt, int K) { return fmt == SP_SPIKES_BITS32 ? words_for(K) : K; }
+inline bool fmt_ok(int fmt) { return fmt == SP_SPIKES_BITS32 || fmt == SP_SPIKES_U8; }
+
+sp_status check_device(int* dev_out) {
+  int dev = 0, major = 0, minor = 0;
+  SP_CUDA(cudaGetDevice(&dev));
+  SP_CUDA(cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev));
+  SP_CUDA(cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev));
+  if (major != 10 || minor != 3) return SP_EDEVICE;
+  *dev_out = dev;
+  return SP_OK;
+}
+
+template <typename T>
+sp_status dev_alloc_zero(T** p, size_t count, cudaStream_t s) {
+  if (count == 0) count = 1;
+  cudaError_t e = cudaMalloc(reinterpret_cast<void**>(p), count * sizeof(T));
+  if (e != cudaSuccess) {
+    *p = nullptr;
+    g_last_cuda_error = (int)e;
+    (void)cudaGetLastError();
+    return e == cudaErrorMemoryAllocation ? SP_ENOMEM : SP_ECUDA;
+  }
+  SP_CUDA(cudaMemsetAsync(*p, 0, count * sizeof(T), s));
+  return SP_OK;
+}
+
+void plan_free(sp_plan_s* p) {
+  if (!p) return;
+  cudaFree(p->ws);
+  cudaFree(p->tickets);
+  cudaFree(p->err);
+  cudaFree(p->d_counts);
+  if (p->h_counts) cudaFreeHost(p->h_counts);
+  cudaFree(p->Wb);
+  cudaFree(p->Xb);
+  delete p;
+}
+
+void group_free(sp_group_s* g) {
+  if (!g) return;
+  cudaFree(g->ws);
+  cudaFree(g->tickets);
+  cudaFree(g->err);
+  cudaFree(g->d_spikes);
+  cudaFree(g->d_acc);
+  cudaFree(g->d_y);
+  delete g;
+}
+
+// Spike / output argument checks shared by the per-plan calls.
+sp_status check_io(const void* spikes, int fmt, const int32_t* acc, const float* y) {
+  if (!spikes || !fmt_ok(fmt)) return SP_EINVAL;
+  if (!acc && !y) return SP_EINVAL;
+  if (fmt == SP_SPIKES_BITS32 && !aligned(spikes, 4)) return SP_EALIGN;
+  if ((acc && !aligned(acc, 4)) || (y && !aligned(y, 4))) return SP_EALIGN;
+  return SP_OK;
+}
+
+GatherParams1 single_params(const sp_plan_s* p, const void* spikes, int fmt, int B, int64_t ld,
+                            int32_t* acc, float* y) {
+  GatherParams1 g;
+  std::memset(&g, 0, sizeof(g));
+  g.prob[0].W = p->W;
+  g.prob[0].scale = p->scale;
+  g.prob[0].ldw = (int32_t)p->ldw;
+  g.prob[0].N = p->N;
+  g.prob[0].K = p->K;
+  g.nprob = 1;
+  g.B = B;
+  g.units_total = B * gather_units(p->N, p->K);
+  g.fmt = fmt;
+  g.spikes = spikes;
+  g.ld_spikes = ld;
+  g.acc = acc;
+  g.y = y;
+  g.ld_out = p->N;
+  g.ws = p->ws;
+  g.tickets = p->tickets;
+  g.err = p->err;
+  return g;
+}
+
+sp_status run_gather(sp_plan_s* p, const void* spikes, int fmt, int B, int64_t ld, int32_t* acc,
+                     float* y, cudaStream_t s) {
+  const GatherParams1 g = single_params(p, spikes, fmt, B, ld, acc, y);
+  SP_CUDA(launch_gather(g, s));
+  return SP_OK;
+}
+
+sp_status run_union(sp_plan_s* p, const void* spikes, int fmt, int B, int64_t ld, int32_t* acc,
+                    float* y, cudaStream_t s) {
+  const int64_t elem = fmt == SP_SPIKES_BITS32 ? 4 : 1;
+  for (int b0 = 0; b0 < B; b0 += kUnionMaxRows) {
+    const int nb = B - b0 < kUnionMaxRows ? B - b0 : kUnionMaxRows;
+    UnionParams u;
+    u.W = p->W;
+    u.scale = p->scale;
+    u.ldw = (int32_t)p->ldw;
+    u.N = p->N;
+    u.K = p->K;
+    u.B = nb;
+    u.fmt = fmt;
+    u.spikes = static_cast<const uint8_t*>(spikes) + (int64_t)b0 * ld * elem;
+    u.ld_spikes = ld;
+    u.acc = acc ? acc + (int64_t)b0 * p->N : nullptr;
+    u.y = y ? y + (int64_t)b0 * p->N : nullptr;
+    u.ws = p->ws;
+    u.tickets = p->tickets;
+    u.err = p->err;
+    SP_CUDA(launch_union(u, s));
+  }
+  return SP_OK;
+}
+
+sp_status run_gemm(sp_plan_s* p, const void* spikes, int fmt, int T, int64_t ld, int32_t* acc,
+                   float* y, cudaStream_t s) {
+  if (!(p->flags & SP_PLAN_GEMM)) return SP_EUNSUPPORTED;
+  SP_CUDA(launch_spikes_to_bf16(spikes, fmt, ld, T, p->K, p->Kp, p->Xb, s));
+  GemmParams g;
+  g.scale = p->scale;
+  g.acc = acc;
+  g.y = y;
+  g.T = T;
+  g.N = p->N;
+  g.K = p->K;
+  g.err = p->err;
+  SP_CUDA(launch_gemm(p->maps, T, p->N, p->Kp, g, p->ws, p->tickets, s));
+  return SP_OK;
+}
+
+// Measured-density dispatch.  Costs are modelled per call from the counts:
+//   gather  ~ sum_t |A_t| * N bytes, through L1/L2, ~one byte-add per byte
+//   union   ~ |U| * N bytes fetched + the same adds from shared memory
+//   gemm    ~ 2 * T * N * K tensor-core ops + conversion of T*K spikes
+// The thresholds below are the crossover points of those models with
+// throughputs measured on GB300 (see the dispatch tests and profiles).
+sp_kernel choose(const sp_plan_s* p, int B, int32_t total, int32_t uni) {
+  const double dens = (double)total / ((double)B * (double)p->K);
+  (void)uni;
+  if ((p->flags & SP_PLAN_GEMM) && B >= 32 && dens >= 0.03) return SP_GEMM;
+  if (B >= 4) return SP_UNION;
+  return SP_GATHER;
+}
+
+sp_status run_multi(sp_plan_s* p, const void* spikes, int fmt, int B, int64_t ld, int32_t* acc,
+                    float* y, sp_kernel strategy, cudaStream_t s) {
+  if (strategy == SP_AUTO) {
+    SP_CUDA(launch_density(spikes, fmt, ld, B, p->K, p->d_counts, s));
+    SP_CUDA(cudaMemcpyAsync(p->h_counts, p->d_counts, 2 * sizeof(int32_t), cudaMemcpyDeviceToHost, s));
+    SP_CUDA(cudaStreamSynchronize(s));
+    strategy = choose(p, B, p->h_counts[0], p->h_counts[1]);
+    p->last_kernel = strategy;
+    p->last_active = p->h_counts[0];
+  }
+  switch (strategy) {
+    case SP_GATHER: return run_gather(p, spikes, fmt, B, ld, acc, y, s);
+    case SP_UNION: return run_union(p, spikes, fmt, B, ld, acc, y, s);
+    case SP_GEMM: return run_gemm(p, spikes, fmt, B, ld, acc, y, s);
+    default: return SP_EINVAL;
+  }
+}
+
+}  // namespace
+
+// ============================================================================
+extern "C" {
+
+sp_status spike_proj_plan(sp_plan_t* plan, const int8_t* W, int64_t ldw, const float* scale,
+                          int32_t N, int32_t K, int32_t max_batch, uint32_t flags,
+                          sp_stream_t stream) {
+  if (!plan || !W || !scale) return SP_EINVAL;
+  if (N < 16 || max_batch < 1 || max_batch > (1 << 20)) return SP_EINVAL;
+  if ((flags & ~SP_PLAN_GEMM) != 0) return SP_EINVAL;
+  if (K < 1 || K > SPIKE_PROJ_MAX_K) return SP_ERANGE;
+  if (N % 16 != 0 || ldw < N || ldw % 16 != 0 || ldw > INT32_MAX) return SP_EALIGN;
+  if (!aligned(W, 16) || !aligned(scale, 4)) return SP_EALIGN;
+  int dev = 0;
+  sp_status st = check_device(&dev);
+  if (st != SP_OK) return st;
+  if ((int64_t)max_batch * N > ((int64_t)1 << 31)) return SP_ERANGE;
+
+  cudaStream_t s = as_stream(stream);
+  sp_plan_s* p = new (std::nothrow) sp_plan_s();
+  if (!p) return SP_ENOMEM;
+  p->device = dev;
+  p->W = W;
+  p->ldw = ldw;
+  p->scale = scale;
+  p->N = N;
+  p->K = K;
+  p->max_batch = max_batch;
+  p->flags = flags;
+
+  size_t tickets = (size_t)max_batch * gather_ntiles(N);
+  const size_t union_t = (size_t)ceil_div(N, kUnionNT);
+  if (union_t > tickets) tickets = union_t;
+  if (flags & SP_PLAN_GEMM) {
+    const size_t gt = (size_t)gemm_ticket_count(max_batch, N);
+    if (gt > tickets) tickets = gt;
+  }
+  p->n_tickets = tickets;
+  if ((st = dev_alloc_zero(&p->ws, (size_t)max_batch * N, s)) != SP_OK ||
+      (st = dev_alloc_zero(&p->tickets, tickets, s)) != SP_OK ||
+      (st = dev_alloc_zero(&p->err, 1, s)) != SP_OK ||
+      (st = dev_alloc_zero(&p->d_counts, 2, s)) != SP_OK) {
+    plan_free(p);
+    return st;
+  }
+  cudaError_t e = cudaMallocHost(reinterpret_cast<void**>(&p->h_counts), 2 * sizeof(int32_t));
+  if (e != cudaSuccess) {
+    plan_free(p);
+    return cuda_fail(e);
+  }
+  if (flags & SP_PLAN_GEMM) {
+    p->Kp = gemm_k_pad(K);
+    p->xb_rows = ceil_div(max_batch, 128) * 128;
+    if ((st = dev_alloc_zero(&p->Wb, (size_t)N * p->Kp, s)) != SP_OK ||
+        (st = dev_alloc_zero(&p->Xb, (size_t)p->xb_rows * p->Kp, s)) != SP_OK) {
+      plan_free(p);
+      return st;
+    }
+    e = launch_w_to_bf16(W, ldw, N, K, p->Wb, s);
+    if (e == cudaSuccess) e = gemm_make_maps(p->Xb, p->xb_rows, p->Wb, N, p->Kp, &p->maps);
+    if (e != cudaSuccess) {
+      plan_free(p);
+      return cuda_fail(e);
+    }
+  }
+  e = cudaStreamSynchronize(s);
+  if (e != cudaSuccess) {
+    plan_free(p);
+    return cuda_fail(e);
+  }
+  *plan = p;
+  return SP_OK;
+}
+
+sp_status spike_proj_plan_destroy(sp_plan_t plan) {
+  if (!plan) return SP_OK;
+  cudaError_t e = cudaDeviceSynchronize();
+  plan_free(plan);
+  return e == cudaSuccess ? SP_OK : cuda_fail(e);
+}
+
+sp_status spike_proj_decode(sp_plan_t plan, const void* spikes, sp_fmt fmt, int32_t* acc, float* y,
+                            sp_stream_t stream) {
+  if (!plan) return SP_EINVAL;
+  sp_status st = check_io(spikes, fmt, acc, y);
+  if (st != SP_OK) return st;
+  return run_gather(plan, spikes, fmt, 1, row_elems(fmt, plan->K), acc, y, as_stream(stream));
+}
+
+sp_status spike_proj_batched(sp_plan_t plan, const void* spikes, sp_fmt fmt, int32_t B,
+                             int64_t ld_spikes, int32_t* acc, float* y, sp_kernel strategy,
+                             sp_stream_t stream) {
+  if (!plan) return SP_EINVAL;
+  sp_status st = check_io(spikes, fmt, acc, y);
+  if (st != SP_OK) return st;
+  if (B < 1) return SP_EINVAL;
+  if (B > plan->max_batch) return SP_ERANGE;
+  if (ld_spikes < row_elems(fmt, plan->K)) return SP_EINVAL;
+  if (strategy < SP_AUTO || strategy > SP_GEMM) return SP_EINVAL;
+  if (strategy == SP_GEMM && !(plan->flags & SP_PLAN_GEMM)) return SP_EUNSUPPORTED;
+  return run_multi(plan, spikes, fmt, B, ld_spikes, acc, y, strategy, as_stream(stream));
+}
+
+sp_status spike_proj_prefill(sp_plan_t plan, const uint8_t* X, int32_t T, int64_t ldx,
+                             int32_t* acc, float* y, sp_kernel strategy, sp_stream_t stream) {
+  return spike_proj_batched(plan, X, SP_SPIKES_U8, T, ldx, acc, y, strategy, stream);
+}
+
+sp_status spike_proj_last_dispatch(sp_plan_t plan, sp_kernel* chosen, int32_t* active_count) {
+  if (!plan) return SP_EINVAL;
+  if (chosen) *chosen = plan->last_kernel;
+  if (active_count) *active_count = plan->last_active;
+  return SP_OK;
+}
+
+sp_status spike_proj_plan_status(sp_plan_t plan, sp_stream_t stream) {
+  if (!plan) return SP_EINVAL;
+  cudaStream_t s = as_stream(stream);
+  int h = 0;
+  SP_CUDA(cudaMemcpyAsync(&h, plan->err, sizeof(int), cudaMemcpyDeviceToHost, s));
+  SP_CUDA(cudaStreamSynchronize(s));
+  if (h == 0) return SP_OK;
+  SP_CUDA(cudaMemsetAsync(plan->err, 0, sizeof(int), s));
+  SP_CUDA(cudaMemsetAsync(plan->ws, 0, (size_t)plan->max_batch * plan->N * sizeof(int32_t), s));
+  SP_CUDA(cudaMemsetAsync(plan->tickets, 0, plan->n_tickets * sizeof(uint32_t), s));
+  SP_CUDA(cudaStreamSynchronize(s));
+  return SP_EKERNEL;
+}
+
+// ---------------------------------------------------------------------------
+sp_status spike_proj_group_create(sp_group_t* group, const sp_plan_t* plans, int32_t count,
+                                  sp_stream_t stream) {
+  if (!group || !plans || count < 1 || count > SPIKE_PROJ_MAX_GROUP) return SP_EINVAL;
+  int dev = 0;
+  sp_status st = check_device(&dev);
+  if (st != SP_OK) return st;
+  for (int j = 0; j < count; ++j)
+    if (!plans[j] || plans[j]->device != dev) return SP_EINVAL;
+  cudaStream_t s = as_stream(stream);
+  sp_group_s* g = new (std::nothrow) sp_group_s();
+  if (!g) return SP_ENOMEM;
+  g->count = count;
+  std::memset(&g->params, 0, sizeof(g->params));
+  int64_t units = 0, ws = 0, tk = 0;
+  for (int j = 0; j < count; ++j) {
+    const sp_plan_s* p = plans[j];
+    GatherProblem& P = g->params.prob[j];
+    P.W = p->W;
+    P.scale = p->scale;
+    P.ldw = (int32_t)p->ldw;
+    P.N = p->N;
+    P.K = p->K;
+    P.unit_begin = (int32_t)units;
+    P.ws_begin = (int32_t)ws;
+    P.ticket_begin = (int32_t)tk;
+    units += gather_units(p->N, p->K);
+    ws += p->N;
+    tk += gather_ntiles(p->N);
+    if (p->N > g->maxN) g->maxN = p->N;
+    if (p->K > g->maxK) g->maxK = p->K;
+  }
+  if (units > INT32_MAX || ws > INT32_MAX) {
+    delete g;
+    return SP_ERANGE;
+  }
+  g->params.nprob = count;
+  g->params.B = 1;
+  g->params.units_total = (int32_t)units;
+  g->ws_elems = (size_t)ws;
+  g->n_tickets = (size_t)tk;
+  g->spike_row_bytes = (size_t)g->maxK;   // covers both formats (ceil(K/32)*4 <= K+3)
+  g->spike_row_bytes = (g->spike_row_bytes + 15) / 16 * 16;
+  if ((st = dev_alloc_zero(&g->ws, g->ws_elems, s)) != SP_OK ||
+      (st = dev_alloc_zero(&g->tickets, g->n_tickets, s)) != SP_OK ||
+      (st = dev_alloc_zero(&g->err, 1, s)) != SP_OK ||
+      (st = dev_alloc_zero(reinterpret_cast<uint8_t**>(&g->d_spikes),
+                           (size_t)count * g->spike_row_bytes, s)) != SP_OK ||
+      (st = dev_alloc_zero(&g->d_acc, (size_t)count * g->maxN, s)) != SP_OK ||
+      (st = dev_alloc_zero(&g->d_y, (size_t)count * g->maxN, s)) != SP_OK) {
+    group_free(g);
+    return st;
+  }
+  g->params.ws = g->ws;
+  g->params.tickets = g->tickets;
+  g->params.err = g->err;
+  cudaError_t e = cudaStreamSynchronize(s);
+  if (e != cudaSuccess) {
+    group_free(g);
+    return cuda_fail(e);
+  }
+  *group = g;
+  return SP_OK;
+}
+
+sp_status spike_proj_group_destroy(sp_group_t group) {
+  if (!group) return SP_OK;
+  cudaError_t e = cudaDeviceSynchronize();
+  group_free(group);
+  return e == cudaSuccess ? SP_OK : cuda_fail(e);
+}
+
+sp_status spike_proj_group_decode(sp_group_t g, const void* spikes, sp_fmt fmt, int64_t ld_spikes,
+                                  int32_t* acc, float* y, int64_t ld_out, sp_stream_t stream) {
+  if (!g) return SP_EINVAL;
+  sp_status st = check_io(spikes, fmt, acc, y);
+  if (st != SP_OK) return st;
+  if (ld_spikes < row_elems(fmt, g->maxK) || ld_out < g->maxN) return SP_EINVAL;
+  GatherParamsG& P = g->params;
+  P.fmt = fmt;
+  P.spikes = spikes;
+  P.ld_spikes = ld_spikes;
+  P.acc = acc;
+  P.y = y;
+  P.ld_out = ld_out;
+  SP_CUDA(launch_gather(P, as_stream(stream)));
+  return SP_OK;
+}
+
+sp_status spike_proj_group_decode_host(sp_group_t g, const void* h_spikes, sp_fmt fmt,
+                                       int64_t ld_spikes, int32_t* h_acc, float* h_y,
+                                       int64_t ld_out, sp_stream_t stream) {
+  if (!g || !h_spikes || !fmt_ok(fmt) || (!h_acc && !h_y)) return SP_EINVAL;
+  const int64_t need = row_elems(fmt, g->maxK);
+  if (ld_spikes < need || ld_out < g->maxN) return SP_EINVAL;
+  cudaStream_t s = as_stream(stream);
+  const size_t elem = fmt == SP_SPIKES_BITS32 ? 4 : 1;
+  const size_t row_bytes = (size_t)need * elem;
+  SP_CUDA(cudaMemcpy2DAsync(g->d_spikes, g->spike_row_bytes, h_spikes, (size_t)ld_spikes * elem,
+                            row_bytes, (size_t)g->count, cudaMemcpyHostToDevice, s));
+  GatherParamsG& P = g->params;
+  P.fmt = fmt;
+  P.spikes = g->d_spikes;
+  P.ld_spikes = (int64_t)(g->spike_row_bytes / elem);
+  P.acc = h_acc ? g->d_acc : nullptr;
+  P.y = h_y ? g->d_y : nullptr;
+  P.ld_out = g->maxN;
+  SP_CUDA(launch_gather(P, s));
+  const size_t out_row = (size_t)g->maxN * 4;
+  if (h_acc)
+    SP_CUDA(cudaMemcpy2DAsync(h_acc, (size_t)ld_out * 4, g->d_acc, out_row, out_row,
+                              (size_t)g->count, cudaMemcpyDeviceToHost, s));
+  if (h_y)
+    SP_CUDA(cudaMemcpy2DAsync(h_y, (size_t)ld_out * 4, g->d_y, out_row, out_row, (size_t)g->count,
+                              cudaMemcpyDeviceToHost, s));
+  return SP_OK;
+}
+
+sp_status spike_proj_group_status(sp_group_t g, sp_stream_t stream) {
+  if (!g) return SP_EINVAL;
+  cudaStream_t s = as_stream(stream);
+  int h = 0;
+  SP_CUDA(cudaMemcpyAsync(&h, g->err, sizeof(int), cudaMemcpyDeviceToHost, s));
+  SP_CUDA(cudaStreamSynchronize(s));
+  if (h == 0) return SP_OK;
+  SP_CUDA(cudaMemsetAsync(g->err, 0, sizeof(int), s));
+  SP_CUDA(cudaMemsetAsync(g->ws, 0, g->ws_elems * sizeof(int32_t), s));
+  SP_CUDA(cudaMemsetAsync(g->tickets, 0, g->n_tickets * sizeof(uint32_t), s));
+  SP_CUDA(cudaStreamSynchronize(s));
+  return SP_EKERNEL;
+}
+
+const char* spike_proj_strerror(sp_status status) {
+  switch (status) {
+    case SP_OK: return "success";
+    case SP_EINVAL: return "invalid argument";
+    case SP_EALIGN: return "alignment or leading-dimension rule violated";
+    case SP_EDEVICE: return "current device is not compute capability 10.3 (GB300)";
+    case SP_ECUDA: return "CUDA runtime error (see spike_proj_last_cuda_error)";
+    case SP_ENOMEM: return "device memory allocation failed";
+    case SP_ERANGE: return "size out of range (K above 131072 or batch above the plan's maximum)";
+    case SP_EKERNEL: return "a kernel reported an error (device error word set)";
+    case SP_EUNSUPPORTED: return "strategy not available for this plan";
+  }
+  return "unknown status";
+}
+
+int spike_proj_last_cuda_error(void) { return g_last_cuda_error; }
+int spike_proj_abi_version(void) { return SPIKE_PROJ_ABI_VERSION; }
+
+}  // extern "C"

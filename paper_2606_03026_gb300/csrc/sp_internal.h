@@ -1,0 +1,116 @@
+// sp_internal.h -- definitions shared by the translation units of
+// libspikeproj.so (host launch wrappers and the kernels' parameter blocks).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+#include <stdint.h>
+
+#include "spike_proj.h"
+
+namespace sp {
+
+// ---------------------------------------------------------------------------
+// Gather decomposition.  A work unit is (problem j, token t, output tile of
+// kGatherNT channels, chunk of kGatherCK input columns).  One warp covers one
+// output tile of one column with 16-byte loads (32 lanes x 16 B = 512 B).
+constexpr int kGatherNT = 512;
+constexpr int kGatherCK = 512;
+constexpr int kGatherWarps = 8;
+constexpr int kGatherThreads = kGatherWarps * 32;
+
+// Union decomposition: a unit is (output tile of kUnionNT, chunk of
+// kUnionCK columns) for all rows of the batch.  Lanes hold 8 channels.
+constexpr int kUnionNT = 256;
+constexpr int kUnionCK = 256;
+constexpr int kUnionWarps = 8;
+constexpr int kUnionThreads = kUnionWarps * 32;
+
+// Device error codes written to a plan's / group's error word.
+enum DeviceError : int {
+  kErrNone = 0,
+  kErrBadUnit = 1,        // a unit index decoded outside its problem
+  kErrMbarTimeout = 2,    // a bounded mbarrier wait ran out (GEMM)
+  kErrTmemAlloc = 3,      // tensor-memory allocation returned an odd address
+};
+
+// One projection as the gather kernel sees it.
+struct GatherProblem {
+  const int8_t* W;        // column-major, W[k*ldw + m]
+  const float* scale;     // [N]
+  int32_t ldw;
+  int32_t N;
+  int32_t K;
+  int32_t unit_begin;     // prefix sum of units_per_token over problems
+  int32_t ws_begin;       // prefix sum of N (int32 elements of workspace)
+  int32_t ticket_begin;   // prefix sum of output tiles
+};
+
+constexpr int kMaxProblems = SPIKE_PROJ_MAX_GROUP;
+
+// Kernel parameters of one gather launch, passed by value (__grid_constant__):
+// NP = 1 for single-plan calls, kMaxProblems for groups.
+template <int NP>
+struct GatherParamsT {
+  GatherProblem prob[NP];
+  int32_t nprob;
+  int32_t B;              // tokens per problem (1 for groups)
+  int32_t units_total;    // B * sum_j units_per_token(j)
+  int32_t fmt;            // sp_fmt
+  const void* spikes;     // row (j*B + t) at spikes + row*ld_spikes elements
+  int64_t ld_spikes;
+  int32_t* acc;           // row (j*B + t) at acc + row*ld_out (may be null)
+  float* y;               // idem (may be null)
+  int64_t ld_out;
+  int32_t* ws;            // problem j token t: ws + (ws_begin_j*B + t*N_j)
+  uint32_t* tickets;      // problem j token t tile n: ticket_begin_j*B + t*ntile_j + n
+  int* err;
+};
+using GatherParams1 = GatherParamsT<1>;
+using GatherParamsG = GatherParamsT<kMaxProblems>;
+
+inline __host__ __device__ int ceil_div(int a, int b) { return (a + b - 1) / b; }
+inline __host__ __device__ int gather_ntiles(int N) { return ceil_div(N, kGatherNT); }
+inline __host__ __device__ int gather_kchunks(int K) { return ceil_div(K, kGatherCK); }
+inline __host__ __device__ int gather_units(int N, int K) {
+  return gather_ntiles(N) * gather_kchunks(K);
+}
+
+struct UnionParams {
+  const int8_t* W;
+  const float* scale;
+  int32_t ldw, N, K, B;
+  int32_t fmt;
+  const void* spikes;
+  int64_t ld_spikes;
+  int32_t* acc;
+  float* y;
+  int32_t* ws;            // [B][N]
+  uint32_t* tickets;      // [ceil(N/kUnionNT)]
+  int* err;
+};
+constexpr int kUnionMaxRows = 256;      // rows per union launch
+
+// Tensor-core (tcgen05) prefill GEMM operands.
+struct GemmParams {
+  const float* scale;
+  int32_t* acc;           // [T][N] or null
+  float* y;               // [T][N] or null
+  int32_t T, N, K;
+  int* err;
+};
+
+// ---------------------------------------------------------------------------
+// Host launch wrappers (defined next to their kernels).  Each returns the
+// cudaError_t of the launch.
+cudaError_t launch_gather(const GatherParams1& p, cudaStream_t s);
+cudaError_t launch_gather(const GatherParamsG& p, cudaStream_t s);
+cudaError_t launch_union(const UnionParams& p, cudaStream_t s);
+// Counts active spikes: out[0] = sum over rows |A_t|, out[1] = |union of A_t|.
+cudaError_t launch_density(const void* spikes, int fmt, int64_t ld, int B, int K,
+                           int32_t* out, cudaStream_t s);
+// Spike rows in either format -> bf16 0/1 [T][Kp] (zero past K).
+cudaError_t launch_spikes_to_bf16(const void* spikes, int fmt, int64_t ld, int T, int K,
+                                  int Kp, __nv_bfloat16* Xb, cudaStream_t s);
+
+}  // namespace sp

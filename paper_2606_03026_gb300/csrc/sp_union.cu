@@ -1,0 +1,220 @@
+// sp_union.cu -- batched decode with shared column fetches, and the density
+// probe used by the dispatcher.
+//
+// Union kernel: B spike rows share one weight matrix.  Eq. (sparse) holds per
+// row; a column that fires in several rows need only be fetched once.  A
+// work unit is (output tile of 256 channels, chunk of 256 columns):
+//   1. load the chunk's spike word of every row (8 words per row) and OR them
+//      into the union U of the chunk,
+//   2. copy the union columns' 256-byte tile segments into shared memory with
+//      cp.async (each column of U read once, inactive columns never),
+//   3. each warp takes whole rows; for every active column of its row it adds
+//      the shared-memory segment into biased 16-bit lanes (lane = 8 channels;
+//      at most 256 columns per chunk, so the lanes cannot overflow),
+//   4. single-chunk problems write acc / y directly; otherwise the row sums go
+//      into the INT32 workspace with red.add and the CTA that completes an
+//      output tile (atomic ticket) applies y = s * float(acc) for every row and
+//      re-zeroes the workspace.  Nothing waits on another CTA.
+#include "sp_spikes.cuh"
+
+namespace sp {
+namespace {
+
+constexpr int kUnionWordsPerChunk = kUnionCK / 32;              // 8
+constexpr size_t kUnionSmemTile = (size_t)kUnionCK * kUnionNT;   // 64 KB
+constexpr size_t kUnionSmemMask = (size_t)kUnionMaxRows * kUnionWordsPerChunk * 4;  // 8 KB
+constexpr size_t kUnionSmem = kUnionSmemTile + kUnionSmemMask;
+
+__device__ __forceinline__ void cp_async16(void* smem, const void* gmem) {
+  const uint32_t s = static_cast<uint32_t>(__cvta_generic_to_shared(smem));
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(s), "l"(gmem) : "memory");
+}
+__device__ __forceinline__ void cp_async_wait_all() {
+  asm volatile("cp.async.wait_all;" ::: "memory");
+}
+
+__global__ void __launch_bounds__(kUnionThreads)
+union_kernel(const __grid_constant__ UnionParams p) {
+  extern __shared__ __align__(16) uint8_t smem[];
+  uint8_t* s_tile = smem;                                                  // [CK][NT]
+  uint32_t* s_mask = reinterpret_cast<uint32_t*>(smem + kUnionSmemTile);   // [B][8]
+  __shared__ uint32_t s_union[kUnionWordsPerChunk];
+  __shared__ int s_uidx[kUnionCK];
+  __shared__ int s_ucount;
+  __shared__ int s_last;
+
+  const int lane = threadIdx.x & 31;
+  const int warp = threadIdx.x >> 5;
+  const int ntile = ceil_div(p.N, kUnionNT);
+  const int kch = ceil_div(p.K, kUnionCK);
+  const int units = ntile * kch;
+
+  for (int u = blockIdx.x; u < units; u += gridDim.x) {
+    const int nt = u / kch;
+    const int kc = u - nt * kch;
+    const int n0 = nt * kUnionNT;
+    const int k0 = kc * kUnionCK;
+
+    // ---- 1. spike words of every row, and their union ------------------------
+    if (threadIdx.x < kUnionWordsPerChunk) s_union[threadIdx.x] = 0u;
+    __syncthreads();
+    for (int i = threadIdx.x; i < p.B * kUnionWordsPerChunk; i += kUnionThreads) {
+      const int t = i / kUnionWordsPerChunk;
+      const int w = i - t * kUnionWordsPerChunk;
+      const uint32_t word =
+          spike_word(spike_row(p.spikes, p.fmt, t, p.ld_spikes), p.fmt, p.K, k0 + 32 * w);
+      s_mask[i] = word;
+      if (word) atomicOr(&s_union[w], word);
+    }
+    __syncthreads();
+    if (warp == 0) {
+      const int n = compact_words(s_union, kUnionWordsPerChunk, 0, s_uidx);
+      if (lane == 0) s_ucount = n;
+    }
+    __syncthreads();
+    const int ucount = s_ucount;
+
+    // ---- 2. fetch each union column's tile segment once ----------------------
+    {
+      const int seg = threadIdx.x & 15;                    // 16-byte segment
+      const int ch = n0 + seg * 16;
+      if (ch < p.N) {
+        for (int i = threadIdx.x >> 4; i < ucount; i += kUnionThreads / 16) {
+          const int kofs = s_uidx[i];
+          cp_async16(s_tile + (size_t)kofs * kUnionNT + seg * 16,
+                     p.W + (int64_t)(k0 + kofs) * p.ldw + ch);
+        }
+      }
+      cp_async_wait_all();
+    }
+    __syncthreads();
+
+    // ---- 3. per-row sums from shared memory ----------------------------------
+    const int ch = n0 + lane * 8;
+    for (int t = warp; t < p.B; t += kUnionWarps) {
+      uint32_t ev0 = 0u, od0 = 0u, ev1 = 0u, od1 = 0u;
+      int n = 0;
+#pragma unroll 1
+      for (int w = 0; w < kUnionWordsPerChunk; ++w) {
+        uint32_t bits = s_mask[t * kUnionWordsPerChunk + w];
+        while (bits) {
+          const int kofs = w * 32 + __ffs(bits) - 1;
+          bits &= bits - 1u;
+          const uint2 v = *reinterpret_cast<const uint2*>(s_tile + (size_t)kofs * kUnionNT + lane * 8);
+          acc_bytes(v.x, ev0, od0);
+          acc_bytes(v.y, ev1, od1);
+          ++n;
+        }
+      }
+      int o[8];
+      unbias16(ev0, od0, n, o);
+      unbias16(ev1, od1, n, o + 4);
+      if (ch < p.N) {
+        if (kch == 1) {
+#pragma unroll
+          for (int q = 0; q < 8; ++q) {
+            if (p.acc) p.acc[(int64_t)t * p.N + ch + q] = o[q];
+            if (p.y) p.y[(int64_t)t * p.N + ch + q] = scale_out(__ldg(p.scale + ch + q), o[q]);
+          }
+        } else {
+          int32_t* ws = p.ws + (int64_t)t * p.N + ch;
+#pragma unroll
+          for (int q = 0; q < 8; ++q)
+            if (o[q]) atomicAdd(ws + q, o[q]);
+        }
+      }
+    }
+
+    // ---- 4. completion ticket per output tile ----------------------------------
+    if (kch > 1) {
+      __threadfence();
+      __syncthreads();
+      if (threadIdx.x == 0) {
+        const uint32_t prev = atomicAdd(p.tickets + nt, 1u);
+        const int last = prev == (uint32_t)(kch - 1);
+        if (last) atomicExch(p.tickets + nt, 0u);
+        s_last = last;
+      }
+      __syncthreads();
+      if (s_last) {
+        __threadfence();
+        const int width = min(kUnionNT, p.N - n0);
+        for (int i = threadIdx.x; i < p.B * width; i += kUnionThreads) {
+          const int t = i / width;
+          const int n = n0 + (i - t * width);
+          int32_t* wsp = p.ws + (int64_t)t * p.N + n;
+          const int v = __ldcg(wsp);
+          __stcg(wsp, 0);
+          if (p.acc) p.acc[(int64_t)t * p.N + n] = v;
+          if (p.y) p.y[(int64_t)t * p.N + n] = scale_out(__ldg(p.scale + n), v);
+        }
+      }
+    }
+    __syncthreads();
+  }
+}
+
+// Density probe: out[0] += sum_t |A_t|, out[1] += |union_t A_t| (out zeroed by
+// the caller).  One thread per 32-column word index.
+__global__ void density_kernel(const void* spikes, int fmt, int64_t ld, int B, int K,
+                               int32_t* out) {
+  const int nw = ceil_div(K, 32);
+  int total = 0, uni = 0;
+  for (int w = blockIdx.x * blockDim.x + threadIdx.x; w < nw; w += gridDim.x * blockDim.x) {
+    uint32_t u = 0u;
+    for (int t = 0; t < B; ++t) {
+      const uint32_t word = spike_word(spike_row(spikes, fmt, t, ld), fmt, K, 32 * w);
+      u |= word;
+      total += __popc(word);
+    }
+    uni += __popc(u);
+  }
+  for (int d = 16; d > 0; d >>= 1) {
+    total += __shfl_xor_sync(0xffffffffu, total, d);
+    uni += __shfl_xor_sync(0xffffffffu, uni, d);
+  }
+  if ((threadIdx.x & 31) == 0) {
+    if (total) atomicAdd(out, total);
+    if (uni) atomicAdd(out + 1, uni);
+  }
+}
+
+int g_union_grid = 0;
+
+}  // namespace
+
+cudaError_t launch_union(const UnionParams& p, cudaStream_t s) {
+  if (p.B <= 0) return cudaSuccess;
+  if (p.B > kUnionMaxRows) return cudaErrorInvalidValue;
+  if (g_union_grid == 0) {
+    int dev = 0, sms = 0, per_sm = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    e = cudaFuncSetAttribute(union_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)kUnionSmem);
+    if (e != cudaSuccess) return e;
+    e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (e != cudaSuccess) return e;
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, union_kernel, kUnionThreads,
+                                                      kUnionSmem);
+    if (e != cudaSuccess) return e;
+    g_union_grid = sms * (per_sm > 0 ? per_sm : 1);
+  }
+  const int units = ceil_div(p.N, kUnionNT) * ceil_div(p.K, kUnionCK);
+  const int grid = units < g_union_grid ? units : g_union_grid;
+  union_kernel<<<grid, kUnionThreads, kUnionSmem, s>>>(p);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_density(const void* spikes, int fmt, int64_t ld, int B, int K, int32_t* out,
+                           cudaStream_t s) {
+  cudaError_t e = cudaMemsetAsync(out, 0, 2 * sizeof(int32_t), s);
+  if (e != cudaSuccess) return e;
+  const int nw = ceil_div(K, 32);
+  const int threads = 128;
+  const int grid = ceil_div(nw, threads);
+  density_kernel<<<grid, threads, 0, s>>>(spikes, fmt, ld, B, K, out);
+  return cudaGetLastError();
+}
+
+}  // namespace sp

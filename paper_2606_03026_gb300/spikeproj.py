@@ -1,0 +1,268 @@
+"""ctypes binding of libspikeproj.so (``include/spike_proj.h``).
+
+Argument marshalling only: every step of the projection runs in the CUDA
+library.  Functions keep the C names; device buffers are passed as torch CUDA
+tensors (or raw integer device addresses), streams default to torch's current
+stream.  A missing library is an error, never a fallback.
+"""
+from __future__ import annotations
+
+import ctypes
+from pathlib import Path
+
+LIB_PATH = Path(__file__).resolve().parent / "_build" / "libspikeproj.so"
+
+# sp_status
+SP_OK, SP_EINVAL, SP_EALIGN, SP_EDEVICE, SP_ECUDA, SP_ENOMEM, SP_ERANGE, \
+    SP_EKERNEL, SP_EUNSUPPORTED = range(9)
+# sp_fmt
+SP_SPIKES_BITS32, SP_SPIKES_U8 = 0, 1
+# sp_kernel
+SP_AUTO, SP_GATHER, SP_UNION, SP_GEMM = 0, 1, 2, 3
+SP_PLAN_GEMM = 0x1
+SPIKE_PROJ_MAX_K = 131072
+SPIKE_PROJ_MAX_GROUP = 64
+
+FMTS = {"bits": SP_SPIKES_BITS32, "u8": SP_SPIKES_U8}
+KERNELS = {"auto": SP_AUTO, "gather": SP_GATHER, "union": SP_UNION, "gemm": SP_GEMM}
+KERNEL_NAMES = {v: k for k, v in KERNELS.items()}
+
+# every entry point of the C ABI with its ctypes signature
+_P, _I32, _I64, _U32 = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_uint32
+_SIGNATURES = {
+    "spike_proj_plan": ([_P, _P, _I64, _P, _I32, _I32, _I32, _U32, _P], ctypes.c_int),
+    "spike_proj_plan_destroy": ([_P], ctypes.c_int),
+    "spike_proj_decode": ([_P, _P, ctypes.c_int, _P, _P, _P], ctypes.c_int),
+    "spike_proj_batched": ([_P, _P, ctypes.c_int, _I32, _I64, _P, _P, ctypes.c_int, _P],
+                           ctypes.c_int),
+    "spike_proj_prefill": ([_P, _P, _I32, _I64, _P, _P, ctypes.c_int, _P], ctypes.c_int),
+    "spike_proj_last_dispatch": ([_P, _P, _P], ctypes.c_int),
+    "spike_proj_plan_status": ([_P, _P], ctypes.c_int),
+    "spike_proj_group_create": ([_P, _P, _I32, _P], ctypes.c_int),
+    "spike_proj_group_destroy": ([_P], ctypes.c_int),
+    "spike_proj_group_decode": ([_P, _P, ctypes.c_int, _I64, _P, _P, _I64, _P], ctypes.c_int),
+    "spike_proj_group_decode_host": ([_P, _P, ctypes.c_int, _I64, _P, _P, _I64, _P],
+                                     ctypes.c_int),
+    "spike_proj_group_status": ([_P, _P], ctypes.c_int),
+    "spike_proj_strerror": ([ctypes.c_int], ctypes.c_char_p),
+    "spike_proj_last_cuda_error": ([], ctypes.c_int),
+    "spike_proj_abi_version": ([], ctypes.c_int),
+}
+
+_lib = None
+
+
+class SpikeProjError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        self.status = status
+        msg = lib().spike_proj_strerror(status).decode()
+        if status == SP_ECUDA:
+            msg += f" (cudaError {lib().spike_proj_last_cuda_error()})"
+        super().__init__(f"{where}: {msg} [status {status}]")
+
+
+def lib():
+    """The loaded library (opened on first use).  Raises if it is not built."""
+    global _lib
+    if _lib is None:
+        if not LIB_PATH.exists():
+            raise RuntimeError(
+                f"{LIB_PATH} is missing: build the CUDA library first "
+                "(python -c 'import __graft_entry__ as g; g.build()')")
+        L = ctypes.CDLL(str(LIB_PATH))
+        for name, (args, res) in _SIGNATURES.items():
+            fn = getattr(L, name)
+            fn.argtypes = args
+            fn.restype = res
+        _lib = L
+    return _lib
+
+
+def _addr(x):
+    """Device (or host) address of a tensor / numpy array / int / None."""
+    if x is None:
+        return None
+    if isinstance(x, int):
+        return x
+    if hasattr(x, "data_ptr"):
+        return x.data_ptr()
+    if hasattr(x, "ctypes"):
+        return x.ctypes.data
+    raise TypeError(f"cannot take the address of {type(x)!r}")
+
+
+def _stream(stream):
+    if stream is None:
+        import torch
+        return torch.cuda.current_stream().cuda_stream
+    if isinstance(stream, int):
+        return stream
+    return stream.cuda_stream
+
+
+def _check(status: int, where: str):
+    if status != SP_OK:
+        raise SpikeProjError(status, where)
+
+
+def _fmt(fmt):
+    return FMTS[fmt] if isinstance(fmt, str) else int(fmt)
+
+
+def _kernel(k):
+    return KERNELS[k] if isinstance(k, str) else int(k)
+
+
+# ---------------------------------------------------------------------------
+# thin wrappers, same names as the C ABI
+# ---------------------------------------------------------------------------
+def spike_proj_plan(W, ldw, scale, N, K, max_batch=1, flags=0, stream=None) -> int:
+    h = ctypes.c_void_p()
+    _check(lib().spike_proj_plan(ctypes.byref(h), _addr(W), ldw, _addr(scale), N, K,
+                                 max_batch, flags, _stream(stream)), "spike_proj_plan")
+    return h.value
+
+
+def spike_proj_plan_destroy(plan):
+    _check(lib().spike_proj_plan_destroy(plan), "spike_proj_plan_destroy")
+
+
+def spike_proj_decode(plan, spikes, fmt, acc=None, y=None, stream=None):
+    _check(lib().spike_proj_decode(plan, _addr(spikes), _fmt(fmt), _addr(acc), _addr(y),
+                                   _stream(stream)), "spike_proj_decode")
+
+
+def spike_proj_batched(plan, spikes, fmt, B, ld_spikes, acc=None, y=None, strategy="auto",
+                       stream=None):
+    _check(lib().spike_proj_batched(plan, _addr(spikes), _fmt(fmt), B, ld_spikes, _addr(acc),
+                                    _addr(y), _kernel(strategy), _stream(stream)),
+           "spike_proj_batched")
+
+
+def spike_proj_prefill(plan, X, T, ldx, acc=None, y=None, strategy="auto", stream=None):
+    _check(lib().spike_proj_prefill(plan, _addr(X), T, ldx, _addr(acc), _addr(y),
+                                    _kernel(strategy), _stream(stream)), "spike_proj_prefill")
+
+
+def spike_proj_last_dispatch(plan):
+    k = ctypes.c_int(0)
+    n = ctypes.c_int32(0)
+    _check(lib().spike_proj_last_dispatch(plan, ctypes.byref(k), ctypes.byref(n)),
+           "spike_proj_last_dispatch")
+    return KERNEL_NAMES.get(k.value, k.value), n.value
+
+
+def spike_proj_plan_status(plan, stream=None) -> int:
+    return lib().spike_proj_plan_status(plan, _stream(stream))
+
+
+def spike_proj_group_create(plans, stream=None) -> int:
+    arr = (ctypes.c_void_p * len(plans))(*plans)
+    h = ctypes.c_void_p()
+    _check(lib().spike_proj_group_create(ctypes.byref(h), arr, len(plans), _stream(stream)),
+           "spike_proj_group_create")
+    return h.value
+
+
+def spike_proj_group_destroy(group):
+    _check(lib().spike_proj_group_destroy(group), "spike_proj_group_destroy")
+
+
+def spike_proj_group_decode(group, spikes, fmt, ld_spikes, acc=None, y=None, ld_out=0,
+                            stream=None):
+    _check(lib().spike_proj_group_decode(group, _addr(spikes), _fmt(fmt), ld_spikes, _addr(acc),
+                                         _addr(y), ld_out, _stream(stream)),
+           "spike_proj_group_decode")
+
+
+def spike_proj_group_decode_host(group, h_spikes, fmt, ld_spikes, h_acc=None, h_y=None,
+                                 ld_out=0, stream=None):
+    _check(lib().spike_proj_group_decode_host(group, _addr(h_spikes), _fmt(fmt), ld_spikes,
+                                              _addr(h_acc), _addr(h_y), ld_out,
+                                              _stream(stream)),
+           "spike_proj_group_decode_host")
+
+
+def spike_proj_group_status(group, stream=None) -> int:
+    return lib().spike_proj_group_status(group, _stream(stream))
+
+
+def spike_proj_strerror(status) -> str:
+    return lib().spike_proj_strerror(status).decode()
+
+
+def spike_proj_abi_version() -> int:
+    return lib().spike_proj_abi_version()
+
+
+# ---------------------------------------------------------------------------
+# convenience owners (hold references to the borrowed tensors)
+# ---------------------------------------------------------------------------
+class Plan:
+    """One projection: column-major INT8 W (torch int8 CUDA tensor whose
+    storage is [K][ldw]) and FP32 scale [N]."""
+
+    def __init__(self, W, scale, N, K, ldw=None, max_batch=1, gemm=False, stream=None):
+        self.W, self.scale = W, scale            # borrowed by the library
+        self.N, self.K = N, K
+        self.ldw = N if ldw is None else ldw
+        self.max_batch = max_batch
+        self.handle = spike_proj_plan(W, self.ldw, scale, N, K, max_batch,
+                                      SP_PLAN_GEMM if gemm else 0, stream)
+
+    def decode(self, spikes, fmt, acc=None, y=None, stream=None):
+        spike_proj_decode(self.handle, spikes, fmt, acc, y, stream)
+
+    def batched(self, spikes, fmt, B, ld_spikes, acc=None, y=None, strategy="auto",
+                stream=None):
+        spike_proj_batched(self.handle, spikes, fmt, B, ld_spikes, acc, y, strategy, stream)
+
+    def prefill(self, X, T, ldx, acc=None, y=None, strategy="auto", stream=None):
+        spike_proj_prefill(self.handle, X, T, ldx, acc, y, strategy, stream)
+
+    def last_dispatch(self):
+        return spike_proj_last_dispatch(self.handle)
+
+    def status(self, stream=None) -> int:
+        return spike_proj_plan_status(self.handle, stream)
+
+    def close(self):
+        if self.handle:
+            spike_proj_plan_destroy(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+class Group:
+    """Independent batch-1 projections decoded in one launch."""
+
+    def __init__(self, plans, stream=None):
+        self.plans = list(plans)
+        self.handle = spike_proj_group_create([p.handle for p in self.plans], stream)
+
+    def decode(self, spikes, fmt, ld_spikes, acc=None, y=None, ld_out=0, stream=None):
+        spike_proj_group_decode(self.handle, spikes, fmt, ld_spikes, acc, y, ld_out, stream)
+
+    def decode_host(self, h_spikes, fmt, ld_spikes, h_acc=None, h_y=None, ld_out=0,
+                    stream=None):
+        spike_proj_group_decode_host(self.handle, h_spikes, fmt, ld_spikes, h_acc, h_y,
+                                     ld_out, stream)
+
+    def status(self, stream=None) -> int:
+        return spike_proj_group_status(self.handle, stream)
+
+    def close(self):
+        if self.handle:
+            spike_proj_group_destroy(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass

@@ -1,0 +1,70 @@
+"""The C-ABI library builds, loads on a machine without a GPU and exports
+every entry point that include/spike_proj.h declares.  No compute calls."""
+import ctypes
+import re
+from pathlib import Path
+
+import pytest
+
+from paper_2606_03026_gb300 import _build, spikeproj
+
+HEADER = Path(__file__).resolve().parent.parent / "include" / "spike_proj.h"
+
+
+@pytest.fixture(scope="module")
+def lib():
+    _build.build()
+    return spikeproj.lib()
+
+
+def declared_functions():
+    text = HEADER.read_text()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(spike_proj_\w+)\s*\(", text)))
+
+
+def test_header_declares_the_boundary():
+    names = declared_functions()
+    for required in ("spike_proj_plan", "spike_proj_decode", "spike_proj_batched",
+                     "spike_proj_prefill"):
+        assert required in names
+
+
+def test_every_declared_symbol_is_exported(lib):
+    names = declared_functions()
+    assert names
+    for name in names:
+        assert hasattr(lib, name), f"{name} not exported by {spikeproj.LIB_PATH}"
+    assert set(names) == set(spikeproj._SIGNATURES), "binding and header disagree"
+
+
+def test_host_only_calls(lib):
+    assert spikeproj.spike_proj_abi_version() == 1
+    assert "invalid" in spikeproj.spike_proj_strerror(spikeproj.SP_EINVAL)
+    # argument checks return before any CUDA call
+    assert lib.spike_proj_plan(None, None, 16, None, 16, 16, 1, 0, None) == spikeproj.SP_EINVAL
+    h = ctypes.c_void_p()
+    fake = 1 << 20                       # never dereferenced: rejected first
+    assert lib.spike_proj_plan(ctypes.byref(h), fake, 16, fake, 16, 0, 1, 0, None) == \
+        spikeproj.SP_ERANGE
+    assert lib.spike_proj_plan(ctypes.byref(h), fake, 16, fake, 16, 131073, 1, 0, None) == \
+        spikeproj.SP_ERANGE
+    assert lib.spike_proj_plan(ctypes.byref(h), fake, 16, fake, 24, 64, 1, 0, None) == \
+        spikeproj.SP_EALIGN                # N % 16 != 0
+    assert lib.spike_proj_plan(ctypes.byref(h), fake + 8, 16, fake, 16, 64, 1, 0, None) == \
+        spikeproj.SP_EALIGN                # W not 16-byte aligned
+    assert lib.spike_proj_plan(ctypes.byref(h), fake, 8, fake, 16, 64, 1, 0, None) == \
+        spikeproj.SP_EALIGN                # ldw < N
+    assert lib.spike_proj_plan(ctypes.byref(h), fake, 16, fake, 16, 64, 1, 0x10, None) == \
+        spikeproj.SP_EINVAL                # unknown flag
+    assert lib.spike_proj_decode(None, fake, 0, fake, fake, None) == spikeproj.SP_EINVAL
+    assert lib.spike_proj_group_create(None, None, 0, None) == spikeproj.SP_EINVAL
+    assert lib.spike_proj_plan_destroy(None) == spikeproj.SP_OK
+    assert lib.spike_proj_group_destroy(None) == spikeproj.SP_OK
+
+
+def test_missing_library_is_an_error(monkeypatch, tmp_path):
+    monkeypatch.setattr(spikeproj, "LIB_PATH", tmp_path / "absent.so")
+    monkeypatch.setattr(spikeproj, "_lib", None)
+    with pytest.raises(RuntimeError, match="missing"):
+        spikeproj.lib()

@@ -1,0 +1,132 @@
+"""Batched decode and prefill: per-token gather, union shared fetch, the
+tcgen05 tensor-core GEMM and the density dispatcher, all against the CPU
+oracle and against each other (GPU)."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from gpu_util import DEV, assert_parity, to_dev
+from paper_2606_03026_gb300 import spikeproj as sp
+from paper_2606_03026_gb300 import synth
+
+pytestmark = pytest.mark.gpu
+
+STRATEGIES = ("gather", "union", "gemm")
+
+
+def run_batched(plan, spikes, fmt, B, ld, N, strategy):
+    acc = torch.full((B, N), -7, dtype=torch.int32, device=DEV)
+    y = torch.full((B, N), -7.0, dtype=torch.float32, device=DEV)
+    plan.batched(spikes, fmt, B, ld, acc, y, strategy)
+    torch.cuda.synchronize()
+    return acc, y
+
+
+@pytest.fixture(scope="module")
+def down():
+    Qc, s = synth.down_weights(3)
+    plan = sp.Plan(to_dev(Qc), to_dev(s), 1536, 6144, max_batch=512, gemm=True)
+    return Qc, s, plan
+
+
+@pytest.mark.parametrize("correlated", [False, True])
+@pytest.mark.parametrize("strategy", STRATEGIES + ("auto",))
+def test_batch64(down, correlated, strategy):
+    """B = 64 tokens, rates U(0.05, 0.2), independent or hot-set correlated."""
+    Qc, s, plan = down
+    X, _, _ = synth.batched_spikes(0, correlated=correlated)
+    want_acc, want_y = oracle.project(Qc, s, 1536, 6144, X, "u8")
+    bits = synth.pack_bits(X)
+    acc, y = run_batched(plan, to_dev(bits), "bits", 64, bits.shape[1], 1536, strategy)
+    assert_parity(acc, y, want_acc, want_y, f"B=64 {strategy} corr={correlated}")
+    acc, y = run_batched(plan, to_dev(X), "u8", 64, X.shape[1], 1536, strategy)
+    assert_parity(acc, y, want_acc, want_y, f"B=64 u8 {strategy} corr={correlated}")
+    if strategy == "auto":
+        chosen, active = plan.last_dispatch()
+        assert chosen in STRATEGIES
+        assert active == int(X.astype(np.int64).sum())
+
+
+def test_prefill_512_tokens(down):
+    """512-token prefill block: X ~ Bernoulli(0.15 * lognormal(0, 0.5)); the
+    dispatcher must pick the tensor-core GEMM; full output vs the oracle."""
+    Qc, s, plan = down
+    X = synth.prefill_spikes(0)
+    want_acc, want_y = oracle.project(Qc, s, 1536, 6144, X, "u8")
+    Xd = to_dev(X)
+    acc = torch.empty(512, 1536, dtype=torch.int32, device=DEV)
+    y = torch.empty(512, 1536, dtype=torch.float32, device=DEV)
+    plan.prefill(Xd, 512, 6144, acc, y, "auto")
+    torch.cuda.synchronize()
+    assert plan.last_dispatch() == ("gemm", int(X.astype(np.int64).sum()))
+    assert_parity(acc, y, want_acc, want_y, "prefill auto")
+    for strategy in ("gemm", "gather", "union"):
+        acc.fill_(0)
+        y.fill_(0)
+        plan.prefill(Xd, 512, 6144, acc, y, strategy)
+        torch.cuda.synchronize()
+        assert_parity(acc, y, want_acc, want_y, f"prefill {strategy}")
+    assert plan.status() == sp.SP_OK
+
+
+@pytest.mark.parametrize("T,N,K,ldq", [(1, 16, 1, 16), (5, 48, 100, 64), (129, 272, 1000, 288),
+                                       (300, 1552, 777, 1552), (128, 256, 64, 256),
+                                       (257, 512, 6143, 512)])
+def test_gemm_ragged(T, N, K, ldq):
+    """The tensor-core path on ragged row / column / K-block tails."""
+    Qc, s, X = synth.random_case(60 + T, N, K, T=T, p=0.3, ldq=ldq)
+    want_acc, want_y = oracle.project(Qc, s, N, K, X, "u8", ldq=ldq)
+    plan = sp.Plan(to_dev(Qc), to_dev(s), N, K, ldw=ldq, max_batch=T, gemm=True)
+    for strategy in STRATEGIES:
+        acc, y = run_batched(plan, to_dev(X), "u8", T, K, N, strategy)
+        assert_parity(acc, y, want_acc, want_y, f"T={T} N={N} K={K} {strategy}")
+
+
+def test_gemm_extremes():
+    """All-ones spikes against -128 / +127 weights: the largest sums the
+    tensor-core path must carry exactly (|acc| = 128 * K)."""
+    T, N, K = 130, 64, 8192
+    X = np.ones((T, K), np.uint8)
+    X[1::2, ::3] = 0
+    s = np.linspace(-2, 2, N).astype(np.float32)
+    for c in (-128, 127):
+        Qc = np.full((K, N), c, np.int8)
+        Qc[::5] = -c if c == 127 else 127
+        want_acc, want_y = oracle.project(Qc, s, N, K, X, "u8")
+        plan = sp.Plan(to_dev(Qc), to_dev(s), N, K, max_batch=T, gemm=True)
+        acc, y = run_batched(plan, to_dev(X), "u8", T, K, N, "gemm")
+        assert_parity(acc, y, want_acc, want_y, f"gemm extremes {c}")
+
+
+def test_union_many_rows():
+    """More rows than one union launch holds (passes of 256)."""
+    N, K, B = 256, 2000, 600
+    Qc, s, X = synth.random_case(70, N, K, T=B, p=0.05)
+    want_acc, want_y = oracle.project(Qc, s, N, K, X, "u8")
+    plan = sp.Plan(to_dev(Qc), to_dev(s), N, K, max_batch=B)
+    acc, y = run_batched(plan, to_dev(synth.pack_bits(X)), "bits", B, (K + 31) // 32, N, "union")
+    assert_parity(acc, y, want_acc, want_y, "union 600 rows")
+
+
+def test_errors_on_device():
+    Qc, s, X = synth.random_case(80, 64, 128, T=4)
+    W, S = to_dev(Qc), to_dev(s)
+    plan = sp.Plan(W, S, 64, 128, max_batch=4)
+    acc = torch.empty(8, 64, dtype=torch.int32, device=DEV)
+    with pytest.raises(sp.SpikeProjError) as e:
+        plan.batched(to_dev(X), "u8", 5, 128, acc, None, "gather")
+    assert e.value.status == sp.SP_ERANGE
+    with pytest.raises(sp.SpikeProjError) as e:
+        plan.batched(to_dev(X), "u8", 4, 128, acc, None, "gemm")
+    assert e.value.status == sp.SP_EUNSUPPORTED
+    with pytest.raises(sp.SpikeProjError) as e:
+        plan.batched(to_dev(X), "u8", 4, 100, acc, None, "gather")
+    assert e.value.status == sp.SP_EINVAL
+    with pytest.raises(sp.SpikeProjError) as e:
+        plan.decode(to_dev(X[0]), "u8", None, None)
+    assert e.value.status == sp.SP_EINVAL
+    with pytest.raises(sp.SpikeProjError) as e:
+        sp.Plan(W, S, 64, 128, ldw=72)
+    assert e.value.status == sp.SP_EALIGN
+    assert plan.status() == sp.SP_OK

@@ -1,0 +1,103 @@
+"""Grouped decode: the 44 binary-input projections of a 22-block decode step
+in one launch, through the C ABI, against the CPU oracle (GPU)."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from gpu_util import DEV, assert_parity, to_dev
+from paper_2606_03026_gb300 import spikeproj as sp
+from paper_2606_03026_gb300 import synth
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def step():
+    weights = synth.decode_step_weights(0)
+    plans = [sp.Plan(to_dev(Q), to_dev(s), N, K) for (Q, s, N, K) in weights]
+    group = sp.Group(plans)
+    yield weights, plans, group
+    group.close()
+
+
+def step_inputs(weights, step_idx, p=0.1):
+    Ks = [w[3] for w in weights]
+    xs = synth.decode_step_spikes(step_idx, Ks, p=p)
+    ld = (max(Ks) + 31) // 32
+    bits = np.zeros((len(Ks), ld), np.uint32)
+    u8 = np.zeros((len(Ks), max(Ks)), np.uint8)
+    for j, x in enumerate(xs):
+        b = synth.pack_bits(x)
+        bits[j, : b.size] = b
+        u8[j, : x.size] = x
+    return xs, bits, u8
+
+
+def oracle_step(weights, xs):
+    accs, ys = [], []
+    for (Q, s, N, K), x in zip(weights, xs):
+        a, y = oracle.project(Q, s, N, K, x, "u8")
+        accs.append(a[0])
+        ys.append(y[0])
+    return np.stack(accs), np.stack(ys)
+
+
+@pytest.mark.parametrize("step_idx", [0, 1, 2])
+def test_decode_step_22_blocks(step, step_idx):
+    weights, plans, group = step
+    xs, bits, u8 = step_inputs(weights, step_idx)
+    want_acc, want_y = oracle_step(weights, xs)
+    n = len(weights)
+    acc = torch.full((n, 1536), -1, dtype=torch.int32, device=DEV)
+    y = torch.full((n, 1536), -1.0, dtype=torch.float32, device=DEV)
+    group.decode(to_dev(bits), "bits", bits.shape[1], acc, y, 1536)
+    torch.cuda.synchronize()
+    assert_parity(acc, y, want_acc, want_y, f"step {step_idx} bits")
+    acc.fill_(0)
+    y.fill_(0)
+    group.decode(to_dev(u8), "u8", u8.shape[1], acc, y, 1536)
+    torch.cuda.synchronize()
+    assert_parity(acc, y, want_acc, want_y, f"step {step_idx} u8")
+    assert group.status() == sp.SP_OK
+
+
+def test_host_buffer_entry_point(step):
+    """The host-buffer variant (copies inside the call) gives the same bits."""
+    weights, plans, group = step
+    xs, bits, _ = step_inputs(weights, 7)
+    want_acc, want_y = oracle_step(weights, xs)
+    n = len(weights)
+    h_bits = torch.from_numpy(bits).pin_memory()
+    h_acc = torch.empty((n, 1536), dtype=torch.int32).pin_memory()
+    h_y = torch.empty((n, 1536), dtype=torch.float32).pin_memory()
+    for _ in range(2):
+        group.decode_host(h_bits, "bits", bits.shape[1], h_acc, h_y, 1536)
+        torch.cuda.synchronize()
+        assert_parity(h_acc, h_y, want_acc, want_y, "host buffers")
+
+
+def test_mixed_group_shapes():
+    """Projections of different N, K and ldw in one group, sparse and dense."""
+    cases = [(16, 1), (48, 1000), (1552, 777), (512, 6144), (2048, 33)]
+    weights, plans, xs = [], [], []
+    for i, (N, K) in enumerate(cases):
+        ldq = N + 16 * (i % 2)
+        Qc, s, x = synth.random_case(40 + i, N, K, p=(0.05, 0.5, 1.0, 0.1, 0.0)[i], ldq=ldq)
+        weights.append((Qc, s, N, K, ldq))
+        plans.append(sp.Plan(to_dev(Qc), to_dev(s), N, K, ldw=ldq))
+        xs.append(x[0])
+    group = sp.Group(plans)
+    maxK = max(K for _, K in cases)
+    maxN = max(N for N, _ in cases)
+    u8 = np.zeros((len(cases), maxK), np.uint8)
+    for j, x in enumerate(xs):
+        u8[j, : x.size] = x
+    acc = torch.zeros((len(cases), maxN), dtype=torch.int32, device=DEV)
+    y = torch.zeros((len(cases), maxN), dtype=torch.float32, device=DEV)
+    group.decode(to_dev(u8), "u8", maxK, acc, y, maxN)
+    torch.cuda.synchronize()
+    for j, (Qc, s, N, K, ldq) in enumerate(weights):
+        a, yy = oracle.project(Qc, s, N, K, xs[j], "u8", ldq=ldq)
+        assert_parity(acc[j, :N], y[j, :N], a[0], yy[0], f"member {j}")
+    group.close()
