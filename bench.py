@@ -62,6 +62,12 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
     ap.add_argument("--e2e-steps", type=int, default=6400)
+    ap.add_argument("--weight-copies", type=int, default=WEIGHT_COPIES,
+                    help="rotating copies of the 22-block weights (8 keeps every "
+                         "timed step out of L2; 1 for small profiling runs)")
+    ap.add_argument("--prefill-blocks", type=int, default=22)
+    ap.add_argument("--prefill-only", action="store_true",
+                    help="run only the prefill leg (profiling of the tensor-core path)")
     return ap.parse_args()
 
 
@@ -262,12 +268,20 @@ def run_ours(args):
     sp.lib()
     peaks, peak_kind = load_peaks()
 
+    if args.prefill_only:
+        res = bench_prefill(torch, sp, synth, dev, torch.cuda.Stream(device=dev), peaks,
+                            peak_kind, world, args.prefill_blocks)
+        if rank == 0:
+            print(json.dumps({"prefill": res}))
+        return
+
     weights, sets_np, active = make_step_inputs(rank)
     n_proj = len(weights)
     ld = sets_np.shape[2]
     # weight copies: 8 x 259.5 MB, each projection's copies are distinct buffers
     copies = []
-    for c in range(WEIGHT_COPIES):
+    n_copies = max(1, args.weight_copies)
+    for c in range(n_copies):
         plans = []
         for (Q, s, N, K) in weights:
             Wd = torch.from_numpy(Q).to(dev)
@@ -281,8 +295,8 @@ def run_ours(args):
     stream = torch.cuda.Stream(device=dev)
 
     def step(i, s=None):
-        copies[i % WEIGHT_COPIES].decode(spikes[i % SPIKE_SETS], "bits", ld, acc, y, 1536,
-                                         stream=s)
+        copies[i % n_copies].decode(spikes[i % SPIKE_SETS], "bits", ld, acc, y, 1536,
+                                    stream=s)
 
     # correctness spot check of one step against the oracle before timing
     import oracle
@@ -363,7 +377,7 @@ def run_ours(args):
     e2e_graph = torch.cuda.CUDAGraph()
     with torch.cuda.graph(e2e_graph, stream=stream):
         for i in range(GRAPH_STEPS):
-            copies[i % WEIGHT_COPIES].decode_host(h_sets[i % SPIKE_SETS], "bits", ld, h_acc,
+            copies[i % n_copies].decode_host(h_sets[i % SPIKE_SETS], "bits", ld, h_acc,
                                                   h_y, 1536, stream=torch.cuda.current_stream())
     e2e_runs = max(1, args.e2e_steps // GRAPH_STEPS)
     with torch.cuda.stream(stream):
@@ -391,9 +405,9 @@ def run_ours(args):
         "config": {"workload": WORKLOAD, "global_batch": world,
                    "active_bytes_per_step": bytes_per_step,
                    "weight_bytes_per_copy": weight_bytes,
-                   "l2": f"inputs larger than L2: {WEIGHT_COPIES} rotating weight copies "
-                         f"({WEIGHT_COPIES * weight_bytes / 1e9:.2f} GB) and {SPIKE_SETS} "
-                         "rotating spike sets; no weight reuse within 8 steps",
+                   "l2": f"inputs larger than L2: {n_copies} rotating weight copies "
+                         f"({n_copies * weight_bytes / 1e9:.2f} GB) and {SPIKE_SETS} "
+                         f"rotating spike sets; no weight reuse within {n_copies} steps",
                    "timing": f"CUDA graphs of {GRAPH_STEPS} steps, events on the launching stream",
                    "parallelism": "replicas" if world > 1 else "single GPU"},
         "projected_tokens_per_s": 1e3 / ms_per_step * world,
@@ -411,7 +425,8 @@ def run_ours(args):
     }
 
     if not args.no_prefill:
-        result["prefill"] = bench_prefill(torch, sp, synth, dev, stream, peaks, peak_kind, world)
+        result["prefill"] = bench_prefill(torch, sp, synth, dev, stream, peaks, peak_kind, world,
+                                          args.prefill_blocks)
         result["gpu_launches"] = steps   # prefill is timed outside the headline region
 
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -427,11 +442,10 @@ def run_ours(args):
         print(json.dumps(result))
 
 
-def bench_prefill(torch, sp, synth, dev, stream, peaks, peak_kind, world):
-    """512-token prefill over 22 blocks: one tensor-core launch pair
-    (spike conversion + GEMM) per block, graph-captured."""
+def bench_prefill(torch, sp, synth, dev, stream, peaks, peak_kind, world, blocks=22):
+    """512-token prefill over the decoder's blocks: one tensor-core launch
+    pair (spike conversion + GEMM) per block, graph-captured."""
     import oracle
-    blocks = synth.N_BLOCKS
     T, N, K = 512, 1536, 6144
     plans, Xs, outs = [], [], []
     X0 = None
@@ -479,7 +493,7 @@ def bench_prefill(torch, sp, synth, dev, stream, peaks, peak_kind, world):
     dens = float(np.mean([x.float().mean().item() for x in Xs]))
     for p in plans:
         p.close()
-    return {"value": tops * world, "unit": "TOPS", "ms_per_prefill_22_blocks": ms,
+    return {"value": tops * world, "unit": "TOPS", "blocks": blocks, "ms_per_prefill": ms,
             "prefill_tokens_per_s": T / (ms * 1e-3) * world, "chosen_kernel": chosen,
             "mean_density": dens, "ops": "2*T*N*K dense-equivalent int8 ops per block",
             "roofline": {"bound": "tensor", "achieved": tops, "peak": peak, "unit": "TFLOP/s",

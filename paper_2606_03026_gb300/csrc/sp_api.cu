@@ -35,7 +35,7 @@ struct sp_plan_s {
 struct sp_group_s {
   int32_t count = 0;
   int32_t maxN = 0, maxK = 0;
-  GatherParamsG params;           // problem table, per-call fields filled in
+  GatherParamsG params;           // problem table, per-call fields filled in at each call
   int32_t* ws = nullptr;
   uint32_t* tickets = nullptr;
   int* err = nullptr;
@@ -193,7 +193,7 @@ sp_status run_gemm(sp_plan_s* p, const void* spikes, int fmt, int T, int64_t ld,
   g.N = p->N;
   g.K = p->K;
   g.err = p->err;
-  SP_CUDA(launch_gemm(p->maps, T, p->N, p->Kp, g, p->ws, p->tickets, s));
+  SP_CUDA(launch_gemm(p->maps, T, p->N, p->Kp, g, s));
   return SP_OK;
 }
 
@@ -203,9 +203,8 @@ sp_status run_gemm(sp_plan_s* p, const void* spikes, int fmt, int T, int64_t ld,
 //   gemm    ~ 2 * T * N * K tensor-core ops + conversion of T*K spikes
 // The thresholds below are the crossover points of those models with
 // throughputs measured on GB300 (see the dispatch tests and profiles).
-sp_kernel choose(const sp_plan_s* p, int B, int32_t total, int32_t uni) {
+sp_kernel choose(const sp_plan_s* p, int B, int32_t total) {
   const double dens = (double)total / ((double)B * (double)p->K);
-  (void)uni;
   if ((p->flags & SP_PLAN_GEMM) && B >= 32 && dens >= 0.03) return SP_GEMM;
   if (B >= 4) return SP_UNION;
   return SP_GATHER;
@@ -217,7 +216,7 @@ sp_status run_multi(sp_plan_s* p, const void* spikes, int fmt, int B, int64_t ld
     SP_CUDA(launch_density(spikes, fmt, ld, B, p->K, p->d_counts, s));
     SP_CUDA(cudaMemcpyAsync(p->h_counts, p->d_counts, 2 * sizeof(int32_t), cudaMemcpyDeviceToHost, s));
     SP_CUDA(cudaStreamSynchronize(s));
-    strategy = choose(p, B, p->h_counts[0], p->h_counts[1]);
+    strategy = choose(p, B, p->h_counts[0]);
     p->last_kernel = strategy;
     p->last_active = p->h_counts[0];
   }
@@ -263,10 +262,6 @@ sp_status spike_proj_plan(sp_plan_t* plan, const int8_t* W, int64_t ldw, const f
   size_t tickets = (size_t)max_batch * gather_ntiles(N);
   const size_t union_t = (size_t)ceil_div(N, kUnionNT);
   if (union_t > tickets) tickets = union_t;
-  if (flags & SP_PLAN_GEMM) {
-    const size_t gt = (size_t)gemm_ticket_count(max_batch, N);
-    if (gt > tickets) tickets = gt;
-  }
   p->n_tickets = tickets;
   if ((st = dev_alloc_zero(&p->ws, (size_t)max_batch * N, s)) != SP_OK ||
       (st = dev_alloc_zero(&p->tickets, tickets, s)) != SP_OK ||

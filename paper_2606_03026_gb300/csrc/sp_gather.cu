@@ -2,28 +2,40 @@
 //
 //   acc_m = sum_{k in A} Q[k*ldw + m],   y_m = s_m * float(acc_m)
 //
-// for one or many (projection, token) problems in a single launch.
+// for one or many (projection, token) problems in a single launch: batch-1
+// decode, a group of independent projections (a whole decode step), and the
+// per-token strategy of the batched call.
 //
 // Decomposition: a work unit is (problem j, token t, output tile of 512
-// channels, chunk of 512 input columns).  Per unit the CTA
-//   1. reads the chunk's 16 spike words and compacts them into the ascending
-//      list of active columns (warp popcount + shuffle scan),
-//   2. lets each of its 8 warps stream every 8th listed column: one 16-byte
-//      load per lane covers 512 contiguous bytes of the column, accumulated
-//      as biased 16-bit lanes (at most 64 columns per warp, never overflows),
-//   3. sums the 8 warps through shared memory and
-//      - writes acc / y directly when the problem has a single K chunk, or
-//      - adds into the INT32 workspace with red.add, then takes a ticket:
-//        the CTA that completes the tile (ticket == chunks - 1) reads the
+// channels, chunk of 512 input columns), and one 128-thread CTA does one
+// unit.  Units are small (about 26 KB of active columns at 10% spikes) and
+// many CTAs fit on an SM, so all units of a decode step are resident at once
+// and the memory system sees the whole step's column reads together.  Per
+// unit, with no CTA-wide barrier before the data loads:
+//   1. every warp reads the chunk's 16 spike words and compacts them (warp
+//      popcount and shuffle scan); warp w keeps the active columns whose rank
+//      is w modulo 4,
+//   2. each lane issues all of its warp's column loads at once (16 bytes of
+//      the 512-byte tile row per column, ld.global.nc, not allocated in L1)
+//      and adds them into biased 16-bit lanes (at most 128 columns per warp,
+//      so the lanes cannot overflow),
+//   3. the 4 warps are summed through shared memory and
+//      - acc / y are written directly when the problem has a single chunk, or
+//      - the partial is added into the INT32 workspace with red.add; the CTA
+//        that completes the tile (atomic ticket == chunks - 1) reads the
 //        workspace back, writes acc and y = s * float(acc), and re-zeroes the
-//        workspace and the ticket for the next call.  No CTA ever waits on
-//        another.
+//        workspace and the ticket.  No CTA ever waits on another.
 // Inactive columns are never read.  Integer sums are order-free, so the
 // result is bit-identical to the definition whatever the CTA schedule.
 #include "sp_spikes.cuh"
 
 namespace sp {
 namespace {
+
+constexpr int kWarps = kGatherWarps;               // 4
+constexpr int kWords = kGatherCK / 32;             // spike words per chunk (16)
+constexpr int kPerWarp = kGatherCK / kWarps;       // column-list capacity per warp
+constexpr int kLoadBatch = 12;                     // column loads in flight per lane
 
 template <int NP>
 __device__ __forceinline__ int find_problem(const GatherParamsT<NP>& p, int u) {
@@ -36,12 +48,10 @@ __device__ __forceinline__ int find_problem(const GatherParamsT<NP>& p, int u) {
 }
 
 template <int NP>
-__global__ void __launch_bounds__(kGatherThreads)
+__global__ void __launch_bounds__(kGatherThreads, 7)
 gather_kernel(const __grid_constant__ GatherParamsT<NP> p) {
-  __shared__ uint32_t s_words[kGatherCK / 32];
-  __shared__ int s_idx[kGatherCK];
-  __shared__ __align__(16) int s_red[kGatherWarps][kGatherNT];
-  __shared__ int s_count;
+  __shared__ int s_cols[kWarps][kPerWarp];
+  __shared__ __align__(16) int s_red[kWarps][kGatherNT];
   __shared__ int s_last;
 
   const int lane = threadIdx.x & 31;
@@ -51,15 +61,15 @@ gather_kernel(const __grid_constant__ GatherParamsT<NP> p) {
     // ---- decode the unit ---------------------------------------------------
     const int j = find_problem(p, u);
     const GatherProblem& P = p.prob[j];
-    const int upt = gather_units(P.N, P.K);
+    const int kch = gather_kchunks(P.K);
+    const int ntile = gather_ntiles(P.N);
+    const int upt = ntile * kch;
     const int ul = u - P.unit_begin * p.B;
     const int t = ul / upt;
     const int r = ul - t * upt;
-    const int kch = gather_kchunks(P.K);
-    const int ntile = gather_ntiles(P.N);
     const int nt = r / kch;
     const int kc = r - nt * kch;
-    if (t >= p.B || nt >= ntile) {           // cannot happen for a valid table
+    if (t >= p.B) {                          // cannot happen for a valid table
       if (threadIdx.x == 0) atomicExch(p.err, kErrBadUnit);
       return;
     }
@@ -67,62 +77,62 @@ gather_kernel(const __grid_constant__ GatherParamsT<NP> p) {
     const int k0 = kc * kGatherCK;
     const int64_t row = (int64_t)j * p.B + t;
 
-    // ---- 1. spike words of the chunk -> active list -------------------------
+    // ---- 1. this warp's share of the chunk's active columns -------------------
     const void* srow = spike_row(p.spikes, p.fmt, row, p.ld_spikes);
-    if (threadIdx.x < kGatherCK / 32)
-      s_words[threadIdx.x] = spike_word(srow, p.fmt, P.K, k0 + threadIdx.x * 32);
-    __syncthreads();
-    if (warp == 0) {
-      const int n = compact_words(s_words, kGatherCK / 32, k0, s_idx);
-      if (lane == 0) s_count = n;
+    const uint32_t word = lane < kWords ? spike_word(srow, p.fmt, P.K, k0 + 32 * lane) : 0u;
+    const int c = __popc(word);
+    int incl = c;
+#pragma unroll
+    for (int d = 1; d < 32; d <<= 1) {
+      const int v = __shfl_up_sync(0xffffffffu, incl, d);
+      if (lane >= d) incl += v;
     }
-    __syncthreads();
-    const int cnt = s_count;
+    const int total = __shfl_sync(0xffffffffu, incl, 31);
+    {
+      uint32_t w = word;
+      int rank = incl - c;
+      while (w) {
+        const int b = __ffs(w) - 1;
+        w &= w - 1u;
+        if ((rank & (kWarps - 1)) == warp) s_cols[warp][rank >> 2] = k0 + 32 * lane + b;
+        ++rank;
+      }
+    }
+    __syncwarp();
+    const int mine = (total - warp + kWarps - 1) / kWarps;   // ranks warp, warp+4, ...
 
-    // ---- 2. stream the active columns of this output tile -------------------
+    // ---- 2. stream the columns of this output tile -------------------------------
     const int ch = n0 + lane * 16;          // first channel of this lane
     const bool lane_on = ch < P.N;
     const int8_t* wcol = P.W + ch;
     const int64_t ldw = P.ldw;
     uint32_t ev[4] = {0u, 0u, 0u, 0u}, od[4] = {0u, 0u, 0u, 0u};
-    int mine = 0;
-    int i = warp;
-    for (; i + 3 * kGatherWarps < cnt; i += 4 * kGatherWarps) {
-      const int c0 = s_idx[i], c1 = s_idx[i + kGatherWarps];
-      const int c2 = s_idx[i + 2 * kGatherWarps], c3 = s_idx[i + 3 * kGatherWarps];
-      uint4 v0 = make_uint4(0x80808080u, 0x80808080u, 0x80808080u, 0x80808080u);
-      uint4 v1 = v0, v2 = v0, v3 = v0;
-      if (lane_on) {
-        v0 = ld_weights16(wcol + c0 * ldw);
-        v1 = ld_weights16(wcol + c1 * ldw);
-        v2 = ld_weights16(wcol + c2 * ldw);
-        v3 = ld_weights16(wcol + c3 * ldw);
+    for (int i0 = 0; i0 < mine; i0 += kLoadBatch) {
+      uint4 v[kLoadBatch];
+#pragma unroll
+      for (int b = 0; b < kLoadBatch; ++b) {
+        v[b] = make_uint4(0x80808080u, 0x80808080u, 0x80808080u, 0x80808080u);
+        if (lane_on && i0 + b < mine) v[b] = ld_weights16(wcol + s_cols[warp][i0 + b] * ldw);
       }
-      acc_bytes(v0.x, ev[0], od[0]); acc_bytes(v0.y, ev[1], od[1]);
-      acc_bytes(v0.z, ev[2], od[2]); acc_bytes(v0.w, ev[3], od[3]);
-      acc_bytes(v1.x, ev[0], od[0]); acc_bytes(v1.y, ev[1], od[1]);
-      acc_bytes(v1.z, ev[2], od[2]); acc_bytes(v1.w, ev[3], od[3]);
-      acc_bytes(v2.x, ev[0], od[0]); acc_bytes(v2.y, ev[1], od[1]);
-      acc_bytes(v2.z, ev[2], od[2]); acc_bytes(v2.w, ev[3], od[3]);
-      acc_bytes(v3.x, ev[0], od[0]); acc_bytes(v3.y, ev[1], od[1]);
-      acc_bytes(v3.z, ev[2], od[2]); acc_bytes(v3.w, ev[3], od[3]);
-      mine += 4;
+#pragma unroll
+      for (int b = 0; b < kLoadBatch; ++b) {
+        acc_bytes(v[b].x, ev[0], od[0]);
+        acc_bytes(v[b].y, ev[1], od[1]);
+        acc_bytes(v[b].z, ev[2], od[2]);
+        acc_bytes(v[b].w, ev[3], od[3]);
+      }
     }
-    for (; i < cnt; i += kGatherWarps) {
-      uint4 v = make_uint4(0x80808080u, 0x80808080u, 0x80808080u, 0x80808080u);
-      if (lane_on) v = ld_weights16(wcol + s_idx[i] * ldw);
-      acc_bytes(v.x, ev[0], od[0]); acc_bytes(v.y, ev[1], od[1]);
-      acc_bytes(v.z, ev[2], od[2]); acc_bytes(v.w, ev[3], od[3]);
-      ++mine;
-    }
+    // padding loads (0x80 bytes) add 0 to the biased lanes: only the `mine`
+    // real columns carry the +128 bias
+    const int nacc = mine;
 
     // ---- 3. reduce the warps -------------------------------------------------
     {
       int o[16];
-      unbias16(ev[0], od[0], mine, o + 0);
-      unbias16(ev[1], od[1], mine, o + 4);
-      unbias16(ev[2], od[2], mine, o + 8);
-      unbias16(ev[3], od[3], mine, o + 12);
+      unbias16(ev[0], od[0], nacc, o + 0);
+      unbias16(ev[1], od[1], nacc, o + 4);
+      unbias16(ev[2], od[2], nacc, o + 8);
+      unbias16(ev[3], od[3], nacc, o + 12);
       int4* dst = reinterpret_cast<int4*>(&s_red[warp][lane * 16]);
       dst[0] = make_int4(o[0], o[1], o[2], o[3]);
       dst[1] = make_int4(o[4], o[5], o[6], o[7]);
@@ -137,9 +147,7 @@ gather_kernel(const __grid_constant__ GatherParamsT<NP> p) {
       for (int o = threadIdx.x; o < kGatherNT; o += kGatherThreads) {
         const int n = n0 + o;
         if (n >= P.N) break;
-        int v = 0;
-#pragma unroll
-        for (int w = 0; w < kGatherWarps; ++w) v += s_red[w][o];
+        const int v = s_red[0][o] + s_red[1][o] + s_red[2][o] + s_red[3][o];
         if (acc_row) acc_row[n] = v;
         if (y_row) y_row[n] = scale_out(__ldg(P.scale + n), v);
       }
@@ -148,9 +156,7 @@ gather_kernel(const __grid_constant__ GatherParamsT<NP> p) {
       for (int o = threadIdx.x; o < kGatherNT; o += kGatherThreads) {
         const int n = n0 + o;
         if (n >= P.N) break;
-        int v = 0;
-#pragma unroll
-        for (int w = 0; w < kGatherWarps; ++w) v += s_red[w][o];
+        const int v = s_red[0][o] + s_red[1][o] + s_red[2][o] + s_red[3][o];
         if (v) atomicAdd(ws + n, v);
       }
       __threadfence();
@@ -165,13 +171,20 @@ gather_kernel(const __grid_constant__ GatherParamsT<NP> p) {
       __syncthreads();
       if (s_last) {
         __threadfence();
-        for (int o = threadIdx.x; o < kGatherNT; o += kGatherThreads) {
-          const int n = n0 + o;
-          if (n >= P.N) break;
-          const int v = __ldcg(ws + n);
-          __stcg(ws + n, 0);
-          if (acc_row) acc_row[n] = v;
-          if (y_row) y_row[n] = scale_out(__ldg(P.scale + n), v);
+        int vals[kGatherNT / kGatherThreads];
+#pragma unroll
+        for (int q = 0; q < kGatherNT / kGatherThreads; ++q) {
+          const int n = n0 + threadIdx.x + q * kGatherThreads;
+          vals[q] = n < P.N ? __ldcg(ws + n) : 0;
+        }
+#pragma unroll
+        for (int q = 0; q < kGatherNT / kGatherThreads; ++q) {
+          const int n = n0 + threadIdx.x + q * kGatherThreads;
+          if (n < P.N) {
+            __stcg(ws + n, 0);
+            if (acc_row) acc_row[n] = vals[q];
+            if (y_row) y_row[n] = scale_out(__ldg(P.scale + n), vals[q]);
+          }
         }
       }
     }
@@ -181,20 +194,10 @@ gather_kernel(const __grid_constant__ GatherParamsT<NP> p) {
 
 template <int NP>
 cudaError_t launch_gather_t(const GatherParamsT<NP>& p, cudaStream_t s) {
-  static int grid_cap = 0;                  // SMs x resident CTAs per SM
   if (p.units_total <= 0) return cudaSuccess;
-  if (grid_cap == 0) {
-    int dev = 0, sms = 0, per_sm = 0;
-    cudaError_t e = cudaGetDevice(&dev);
-    if (e != cudaSuccess) return e;
-    e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-    if (e != cudaSuccess) return e;
-    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, gather_kernel<NP>,
-                                                      kGatherThreads, 0);
-    if (e != cudaSuccess) return e;
-    grid_cap = sms * (per_sm > 0 ? per_sm : 1);
-  }
-  const int grid = p.units_total < grid_cap ? p.units_total : grid_cap;
+  // one CTA per unit; the hardware keeps every unit of a decode step resident
+  // (7 CTAs of 128 threads per SM) and schedules the rest in waves
+  const int grid = p.units_total < (1 << 30) ? p.units_total : (1 << 30);
   gather_kernel<NP><<<grid, kGatherThreads, 0, s>>>(p);
   return cudaGetLastError();
 }

@@ -29,13 +29,14 @@
 // that units ~ number of SMs when the output has few tiles (T = 512 gives only
 // 24 tiles of 128x256 for N = 1536).
 //
-// Every mbarrier wait is bounded (about one second of %globaltimer); on
+// Every mbarrier wait is bounded (2^31 SM cycles, about a second); on
 // timeout the kernel sets the error word, stops issuing work, drains what it
 // issued and frees its tensor memory before exiting.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
 #include "sp_gemm.h"
+#include "sp_ptx.cuh"
 #include "sp_spikes.cuh"
 
 namespace sp {
@@ -52,107 +53,6 @@ constexpr size_t SMEM_RING = (size_t)STAGES * STAGE_BYTES;
 constexpr size_t SMEM_TR = (size_t)4 * 32 * TR_STRIDE * 4;
 constexpr size_t SMEM_BARS = 256;
 constexpr size_t kGemmSmem = 1024 + SMEM_RING + SMEM_TR + SMEM_BARS;
-constexpr uint64_t kWaitLimitNs = 1000000000ull;   // 1 s
-
-// ---- PTX wrappers -------------------------------------------------------------
-__device__ __forceinline__ uint32_t smem_u32(const void* p) {
-  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
-}
-__device__ __forceinline__ uint64_t globaltimer() {
-  uint64_t t;
-  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
-  return t;
-}
-__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
-  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count));
-}
-__device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, uint32_t bytes) {
-  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)),
-               "r"(bytes)
-               : "memory");
-}
-__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
-  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
-}
-__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
-  uint32_t ok;
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
-      "selp.u32 %0, 1, 0, p;\n\t}"
-      : "=r"(ok)
-      : "r"(smem_u32(bar)), "r"(parity)
-      : "memory");
-  return ok != 0;
-}
-// Bounded wait for the phase with the given parity; false on timeout.
-__device__ __noinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
-  if (mbar_try_wait(bar, parity)) return true;
-  const uint64_t t0 = globaltimer();
-  for (;;) {
-    for (int i = 0; i < 64; ++i)
-      if (mbar_try_wait(bar, parity)) return true;
-    if (globaltimer() - t0 > kWaitLimitNs) return false;
-  }
-}
-__device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, uint64_t* bar,
-                                            int x, int y) {
-  asm volatile(
-      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
-      " [%0], [%1, {%3, %4}], [%2];" ::"r"(smem_u32(dst)),
-      "l"(reinterpret_cast<uint64_t>(map)), "r"(smem_u32(bar)), "r"(x), "r"(y)
-      : "memory");
-}
-__device__ __forceinline__ void tma_prefetch_desc(const CUtensorMap* map) {
-  asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
-}
-__device__ __forceinline__ void tc_fence_before() {
-  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-}
-__device__ __forceinline__ void tc_fence_after() {
-  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
-}
-__device__ __forceinline__ void tmem_alloc(uint32_t* dst_smem, uint32_t cols) {
-  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
-                   smem_u32(dst_smem)),
-               "r"(cols)
-               : "memory");
-  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
-}
-__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t cols) {
-  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(cols)
-               : "memory");
-}
-__device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc,
-                                         uint32_t idesc, uint32_t accumulate) {
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "setp.ne.b32 p, %4, 0;\n\t"
-      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
-      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
-      : "memory");
-}
-// Arrive on a CTA-local mbarrier once all previously issued MMAs complete.
-__device__ __forceinline__ void mma_commit(uint64_t* bar) {
-  asm volatile(
-      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
-          smem_u32(bar))
-      : "memory");
-}
-// 32 lanes x 32 consecutive 32-bit columns: thread i gets row (lane base + i).
-__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&v)[32]) {
-  asm volatile(
-      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
-      "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, "
-      "%16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
-      : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]),
-        "=r"(v[7]), "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]),
-        "=r"(v[14]), "=r"(v[15]), "=r"(v[16]), "=r"(v[17]), "=r"(v[18]), "=r"(v[19]),
-        "=r"(v[20]), "=r"(v[21]), "=r"(v[22]), "=r"(v[23]), "=r"(v[24]), "=r"(v[25]),
-        "=r"(v[26]), "=r"(v[27]), "=r"(v[28]), "=r"(v[29]), "=r"(v[30]), "=r"(v[31])
-      : "r"(taddr));
-  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-}
 
 // Shared-memory matrix descriptor (tcgen05 format): K-major operand whose rows
 // are 128 bytes (64 bf16) laid out by TMA with the 128-byte swizzle; 8-row
@@ -173,11 +73,31 @@ __device__ __forceinline__ uint64_t smem_desc_k128(const void* p) {
 constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(BN >> 3) << 17) |
                             ((uint32_t)(BM >> 4) << 24);
 
+constexpr int kSlotBytes = 32 * BM * 4;        // one 128-row x 32-column fp32 partial
+
+__device__ __forceinline__ uint32_t cluster_ctarank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+// Arrive + wait on the cluster barrier (release / acquire: shared-memory
+// writes to other CTAs of the cluster before it are visible after it).
+// Every thread of every CTA of the cluster executes it.
+__device__ __forceinline__ void cluster_sync() {
+  asm volatile("barrier.cluster.arrive;\n\tbarrier.cluster.wait;" ::: "memory");
+}
+__device__ __forceinline__ uint32_t map_to_rank(uint32_t smem_addr, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(smem_addr), "r"(rank));
+  return r;
+}
+__device__ __forceinline__ void st_cluster_u32(uint32_t addr, uint32_t v) {
+  asm volatile("st.shared::cluster.u32 [%0], %1;" ::"r"(addr), "r"(v) : "memory");
+}
+
 struct GemmArgs {
   GemmParams p;
   int tiles_m, tiles_n, splits, kb_per_split, nkb, units;
-  int32_t* ws;
-  uint32_t* tickets;
 };
 
 __device__ __forceinline__ void unit_coords(const GemmArgs& a, int u, int& tile, int& mb, int& nb,
@@ -188,6 +108,31 @@ __device__ __forceinline__ void unit_coords(const GemmArgs& a, int u, int& tile,
   nb = tile - mb * a.tiles_n;
   kb0 = sp * a.kb_per_split;
   kb1 = min(a.nkb, kb0 + a.kb_per_split);
+}
+
+// One warp writes a 32-row x 32-column chunk of integer-valued fp32 sums
+// (v[i] = column col0 + i of row row0 + lane): transposed through shared
+// memory so that each store instruction covers 32 consecutive columns of one
+// row; acc = exact int conversion, y = s * float(acc).
+__device__ __forceinline__ void store_chunk(const GemmParams& p, uint32_t* tr,
+                                            const uint32_t (&v)[32], int row0, int col0) {
+  const int lane = threadIdx.x & 31;
+#pragma unroll
+  for (int i = 0; i < 32; ++i) tr[lane * TR_STRIDE + i] = v[i];
+  __syncwarp();
+  const int n = col0 + lane;
+  if (n < p.N) {
+    const float sc = p.y ? __ldg(p.scale + n) : 0.f;
+    for (int rr = 0; rr < 32; ++rr) {
+      const int r = row0 + rr;
+      if (r >= p.T) break;
+      const int val = __float2int_rn(__uint_as_float(tr[rr * TR_STRIDE + lane]));
+      const int64_t o = (int64_t)r * p.N + n;
+      if (p.acc) p.acc[o] = val;
+      if (p.y) p.y[o] = scale_out(sc, val);
+    }
+  }
+  __syncwarp();
 }
 
 __global__ void __launch_bounds__(kGemmThreads, 1)
@@ -306,8 +251,8 @@ gemm_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CU
       mma_commit(done);                      // retire every issued MMA
       mbar_wait(done, 0);
     }
-  } else {
-    // ------------------------------ epilogue ----------------------------------
+  } else if (a.splits == 1) {
+    // ------------------------------ epilogue (whole K) ------------------------
     // Each warp owns one 32-row quarter of the tile (its TMEM lane quarter) and
     // works alone: no barrier joins the epilogue warps, so a warp that gives up
     // on a timed-out wait cannot strand the others.
@@ -315,7 +260,6 @@ gemm_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CU
     uint32_t* tr = s_tr + (size_t)(warp - 2) * 32 * TR_STRIDE;
     int ab = 0;
     uint32_t aph = 0;
-    const int T = a.p.T, N = a.p.N;
     for (int u = blockIdx.x; u < a.units; u += gridDim.x) {
       int tile, mb, nb, kb0, kb1;
       unit_coords(a, u, tile, mb, nb, kb0, kb1);
@@ -325,65 +269,70 @@ gemm_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CU
         break;
       }
       tc_fence_after();
-      const int row0 = mb * BM + q * 32;     // first row of this warp's quarter
+      const int row0 = mb * BM + q * 32;
       for (int c = 0; c < BN; c += 32) {
         uint32_t v[32];
         tmem_ld32(tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(ab * BN + c), v);
-        // transpose: lane = row on the way in, lane = column on the way out
-#pragma unroll
-        for (int i = 0; i < 32; ++i) tr[lane * TR_STRIDE + i] = v[i];
-        __syncwarp();
-        const int n = nb * BN + c + lane;
-        const bool col_ok = n < N;
-        const float sc = (col_ok && a.p.y && a.splits == 1) ? __ldg(a.p.scale + n) : 0.f;
-        for (int rr = 0; rr < 32; ++rr) {
-          const int r = row0 + rr;
-          if (r >= T) break;
-          const int val = __float2int_rn(__uint_as_float(tr[rr * TR_STRIDE + lane]));
-          if (!col_ok) continue;
-          const int64_t o = (int64_t)r * N + n;
-          if (a.splits == 1) {
-            if (a.p.acc) a.p.acc[o] = val;
-            if (a.p.y) a.p.y[o] = scale_out(sc, val);
-          } else if (val) {
-            atomicAdd(a.ws + o, val);
-          }
-        }
-        __syncwarp();
+        store_chunk(a.p, tr, v, row0, nb * BN + c);
       }
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&tempty[ab]);
       if (++ab == 2) { ab = 0; aph ^= 1u; }
+    }
+  } else {
+    // ---------------- epilogue (split K): cluster reduce-scatter ---------------
+    // The CTAs of one cluster hold the same output tile for different K ranges.
+    // Output chunk c (32 columns) belongs to cluster rank c % S.  After every
+    // CTA's MMAs have retired (cluster barrier 1: each ring is free), each CTA
+    // writes its partial of every chunk it does not own into the owner's ring
+    // through distributed shared memory; after cluster barrier 2 each owner
+    // adds the S partials of its chunks and writes acc and y.
+    if (mbar_wait(&tfull[0], 0)) {
+      tc_fence_after();
+    } else {
+      *s_abort = 1;
+      if (lane == 0) atomicExch(a.p.err, kErrMbarTimeout);
+    }
+  }
 
-      if (a.splits > 1) {
-        // the warp that completes this quarter's last K split finishes it
-        __threadfence();
-        __syncwarp();
-        int last = 0;
-        if (lane == 0) {
-          uint32_t* tk = a.tickets + (size_t)tile * 4 + q;
-          const uint32_t prev = atomicAdd(tk, 1u);
-          last = prev == (uint32_t)(a.splits - 1);
-          if (last) atomicExch(tk, 0u);
+  if (a.splits > 1) {
+    const int S = a.splits;
+    const int rank = (int)cluster_ctarank();
+    const int maxlc = (BN / 32 + S - 1) / S;            // chunks owned per rank
+    const bool epi = warp >= 2;
+    const int q = warp & 3;
+    const int row = q * 32 + lane;                      // row within the tile
+    cluster_sync();                                     // 1: every ring is free
+    if (epi && !*s_abort) {
+      for (int c = 0; c < BN / 32; ++c) {
+        const int owner = c % S;
+        if (owner == rank) continue;
+        uint32_t v[32];
+        tmem_ld32(tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)c * 32u, v);
+        const int si = rank < owner ? rank : rank - 1;  // source slot at the owner
+        const uint32_t slot = smem_u32(smem) + (uint32_t)((si * maxlc + c / S) * kSlotBytes);
+        const uint32_t dst = map_to_rank(slot, (uint32_t)owner);
+#pragma unroll
+        for (int i = 0; i < 32; ++i) st_cluster_u32(dst + (uint32_t)(i * BM + row) * 4u, v[i]);
+      }
+    }
+    cluster_sync();                                     // 2: partials delivered
+    if (epi && !*s_abort) {
+      uint32_t* tr = s_tr + (size_t)(warp - 2) * 32 * TR_STRIDE;
+      int tile, mb, nb, kb0, kb1;
+      unit_coords(a, blockIdx.x, tile, mb, nb, kb0, kb1);
+      for (int c = rank; c < BN / 32; c += S) {
+        uint32_t v[32];
+        tmem_ld32(tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)c * 32u, v);
+        for (int si = 0; si < S - 1; ++si) {
+          const float* slot =
+              reinterpret_cast<const float*>(smem + (size_t)(si * maxlc + c / S) * kSlotBytes);
+#pragma unroll
+          for (int i = 0; i < 32; ++i)
+            v[i] = __float_as_uint(__uint_as_float(v[i]) + slot[i * BM + row]);
         }
-        last = __shfl_sync(0xffffffffu, last, 0);
-        if (last) {
-          __threadfence();
-          const int cols = min(BN, N - nb * BN);
-          for (int rr = 0; rr < 32; ++rr) {
-            const int r = row0 + rr;
-            if (r >= T) break;
-            for (int cc = lane; cc < cols; cc += 32) {
-              const int n = nb * BN + cc;
-              const int64_t o = (int64_t)r * N + n;
-              const int val = __ldcg(a.ws + o);
-              __stcg(a.ws + o, 0);
-              if (a.p.acc) a.p.acc[o] = val;
-              if (a.p.y) a.p.y[o] = scale_out(__ldg(a.p.scale + n), val);
-            }
-          }
-        }
+        store_chunk(a.p, tr, v, mb * BM + q * 32, nb * BN + c * 32);
       }
     }
   }
@@ -480,7 +429,6 @@ bool encode_2d(CUtensorMap* map, const void* base, uint64_t inner, uint64_t oute
 }  // namespace
 
 int gemm_k_pad(int K) { return ceil_div(K, BK) * BK; }
-int gemm_ticket_count(int T, int N) { return ceil_div(T, BM) * ceil_div(N, BN) * 4; }
 
 cudaError_t gemm_make_maps(const __nv_bfloat16* Xb, int rows_alloc, const __nv_bfloat16* Wb, int N,
                            int Kp, GemmMaps* out) {
@@ -508,8 +456,33 @@ cudaError_t launch_spikes_to_bf16(const void* spikes, int fmt, int64_t ld, int T
   return cudaGetLastError();
 }
 
+// Largest number of clusters of `size` CTAs that can be resident at once.
+int max_active_clusters(int size) {
+  static int cache[9] = {0};
+  if (cache[size] == 0) {
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute attr;
+    attr.id = cudaLaunchAttributeClusterDimension;
+    attr.val.clusterDim.x = size;
+    attr.val.clusterDim.y = 1;
+    attr.val.clusterDim.z = 1;
+    cfg.gridDim = dim3(size, 1, 1);
+    cfg.blockDim = dim3(kGemmThreads, 1, 1);
+    cfg.dynamicSmemBytes = kGemmSmem;
+    cfg.attrs = &attr;
+    cfg.numAttrs = 1;
+    int n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, gemm_kernel, &cfg) != cudaSuccess || n < 1) {
+      (void)cudaGetLastError();
+      n = -1;
+    }
+    cache[size] = n;
+  }
+  return cache[size];
+}
+
 cudaError_t launch_gemm(const GemmMaps& maps, int T, int N, int Kp, const GemmParams& p,
-                        int32_t* ws, uint32_t* tickets, cudaStream_t s) {
+                        cudaStream_t s) {
   if (!g_attr_set) {
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
@@ -519,6 +492,8 @@ cudaError_t launch_gemm(const GemmMaps& maps, int T, int N, int Kp, const GemmPa
     e = cudaFuncSetAttribute(gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              (int)kGemmSmem);
     if (e != cudaSuccess) return e;
+    e = cudaFuncSetAttribute(gemm_kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 0);
+    if (e != cudaSuccess) return e;
     g_attr_set = true;
   }
   GemmArgs a;
@@ -527,17 +502,42 @@ cudaError_t launch_gemm(const GemmMaps& maps, int T, int N, int Kp, const GemmPa
   a.tiles_n = ceil_div(N, BN);
   a.nkb = Kp / BK;
   const int tiles = a.tiles_m * a.tiles_n;
-  int splits = g_num_sms / tiles;
-  if (splits > a.nkb / 4) splits = a.nkb / 4;
-  if (splits < 1) splits = 1;
-  a.kb_per_split = ceil_div(a.nkb, splits);
-  a.splits = ceil_div(a.nkb, a.kb_per_split);
-  a.units = tiles * a.splits;
-  a.ws = ws;
-  a.tickets = tickets;
-  const int grid = a.units < g_num_sms ? a.units : g_num_sms;
-  gemm_kernel<<<grid, kGemmThreads, kGemmSmem, s>>>(maps.a, maps.b, a);
-  return cudaGetLastError();
+  // Split K over a cluster only when the tiles alone leave SMs idle, and only
+  // as far as every cluster stays resident in a single wave.
+  int S = 1;
+  if (tiles < g_num_sms) {
+    S = g_num_sms / tiles;
+    if (S > 8) S = 8;
+    if (S > a.nkb / 4) S = a.nkb / 4;
+    if (S < 1) S = 1;
+    while (S > 1) {
+      const int kbps = ceil_div(a.nkb, S);
+      const int exact = ceil_div(a.nkb, kbps);          // splits with work
+      if (exact == S && max_active_clusters(S) >= tiles) break;
+      --S;
+    }
+  }
+  a.kb_per_split = ceil_div(a.nkb, S);
+  a.splits = S;
+  a.units = tiles * S;
+  if (S == 1) {
+    const int grid = a.units < g_num_sms ? a.units : g_num_sms;
+    gemm_kernel<<<grid, kGemmThreads, kGemmSmem, s>>>(maps.a, maps.b, a);
+    return cudaGetLastError();
+  }
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr;
+  attr.id = cudaLaunchAttributeClusterDimension;
+  attr.val.clusterDim.x = S;
+  attr.val.clusterDim.y = 1;
+  attr.val.clusterDim.z = 1;
+  cfg.gridDim = dim3(a.units, 1, 1);
+  cfg.blockDim = dim3(kGemmThreads, 1, 1);
+  cfg.dynamicSmemBytes = kGemmSmem;
+  cfg.stream = s;
+  cfg.attrs = &attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, gemm_kernel, maps.a, maps.b, a);
 }
 
 }  // namespace sp

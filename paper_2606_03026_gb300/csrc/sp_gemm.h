@@ -15,14 +15,14 @@ struct GemmMaps {
 };
 
 int gemm_k_pad(int K);                  // K rounded up to the 64-column K block
-int gemm_ticket_count(int T, int N);    // tickets one launch may use
 cudaError_t gemm_make_maps(const __nv_bfloat16* Xb, int rows_alloc, const __nv_bfloat16* Wb,
                            int N, int Kp, GemmMaps* out);
 cudaError_t launch_w_to_bf16(const int8_t* W, int64_t ldw, int N, int K, __nv_bfloat16* Wb,
                              cudaStream_t s);
-// ACC = X W^T on the tensor cores, epilogue acc / y; ws [T][N] INT32 and
-// tickets must be zero on entry and are left zero.
+// ACC = X W^T on the tensor cores with the acc / y epilogue.  Splits K over
+// a thread-block cluster (partials reduced through distributed shared memory)
+// when the output has fewer tiles than SMs.
 cudaError_t launch_gemm(const GemmMaps& maps, int T, int N, int Kp, const GemmParams& p,
-                        int32_t* ws, uint32_t* tickets, cudaStream_t s);
+                        cudaStream_t s);
 
 }  // namespace sp

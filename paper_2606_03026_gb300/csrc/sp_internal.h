@@ -12,11 +12,12 @@ namespace sp {
 
 // ---------------------------------------------------------------------------
 // Gather decomposition.  A work unit is (problem j, token t, output tile of
-// kGatherNT channels, chunk of kGatherCK input columns).  One warp covers one
-// output tile of one column with 16-byte loads (32 lanes x 16 B = 512 B).
+// kGatherNT channels, chunk of kGatherCK input columns), one 128-thread CTA
+// each.  One warp covers one output tile of one column with 16-byte loads
+// (32 lanes x 16 B = 512 B).
 constexpr int kGatherNT = 512;
 constexpr int kGatherCK = 512;
-constexpr int kGatherWarps = 8;
+constexpr int kGatherWarps = 4;
 constexpr int kGatherThreads = kGatherWarps * 32;
 
 // Union decomposition: a unit is (output tile of kUnionNT, chunk of
@@ -106,7 +107,7 @@ struct GemmParams {
 cudaError_t launch_gather(const GatherParams1& p, cudaStream_t s);
 cudaError_t launch_gather(const GatherParamsG& p, cudaStream_t s);
 cudaError_t launch_union(const UnionParams& p, cudaStream_t s);
-// Counts active spikes: out[0] = sum over rows |A_t|, out[1] = |union of A_t|.
+// Counts active spikes: out[0] = sum over the B rows of |A_t| (out[1] unused).
 cudaError_t launch_density(const void* spikes, int fmt, int64_t ld, int B, int K,
                            int32_t* out, cudaStream_t s);
 // Spike rows in either format -> bf16 0/1 [T][Kp] (zero past K).

@@ -154,29 +154,23 @@ union_kernel(const __grid_constant__ UnionParams p) {
   }
 }
 
-// Density probe: out[0] += sum_t |A_t|, out[1] += |union_t A_t| (out zeroed by
-// the caller).  One thread per 32-column word index.
+// Density probe: out[0] += sum over rows of |A_t| (out zeroed by the caller).
+// One thread per (row, 32-column word), grid-stride; warp sums, one atomic
+// per warp.
 __global__ void density_kernel(const void* spikes, int fmt, int64_t ld, int B, int K,
                                int32_t* out) {
   const int nw = ceil_div(K, 32);
-  int total = 0, uni = 0;
-  for (int w = blockIdx.x * blockDim.x + threadIdx.x; w < nw; w += gridDim.x * blockDim.x) {
-    uint32_t u = 0u;
-    for (int t = 0; t < B; ++t) {
-      const uint32_t word = spike_word(spike_row(spikes, fmt, t, ld), fmt, K, 32 * w);
-      u |= word;
-      total += __popc(word);
-    }
-    uni += __popc(u);
+  const int64_t total_words = (int64_t)nw * B;
+  int total = 0;
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < total_words;
+       i += (int64_t)gridDim.x * blockDim.x) {
+    const int t = (int)(i / nw);
+    const int w = (int)(i - (int64_t)t * nw);
+    total += __popc(spike_word(spike_row(spikes, fmt, t, ld), fmt, K, 32 * w));
   }
-  for (int d = 16; d > 0; d >>= 1) {
-    total += __shfl_xor_sync(0xffffffffu, total, d);
-    uni += __shfl_xor_sync(0xffffffffu, uni, d);
-  }
-  if ((threadIdx.x & 31) == 0) {
-    if (total) atomicAdd(out, total);
-    if (uni) atomicAdd(out + 1, uni);
-  }
+#pragma unroll
+  for (int d = 16; d > 0; d >>= 1) total += __shfl_xor_sync(0xffffffffu, total, d);
+  if ((threadIdx.x & 31) == 0 && total) atomicAdd(out, total);
 }
 
 int g_union_grid = 0;
@@ -210,10 +204,12 @@ cudaError_t launch_density(const void* spikes, int fmt, int64_t ld, int B, int K
                            cudaStream_t s) {
   cudaError_t e = cudaMemsetAsync(out, 0, 2 * sizeof(int32_t), s);
   if (e != cudaSuccess) return e;
-  const int nw = ceil_div(K, 32);
-  const int threads = 128;
-  const int grid = ceil_div(nw, threads);
-  density_kernel<<<grid, threads, 0, s>>>(spikes, fmt, ld, B, K, out);
+  const int64_t words = (int64_t)ceil_div(K, 32) * B;
+  const int threads = 256;
+  int64_t grid = (words + threads - 1) / threads;
+  if (grid > 2048) grid = 2048;
+  if (grid < 1) grid = 1;
+  density_kernel<<<(int)grid, threads, 0, s>>>(spikes, fmt, ld, B, K, out);
   return cudaGetLastError();
 }
 

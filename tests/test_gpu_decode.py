@@ -56,7 +56,8 @@ def test_down_projection_all_vectors(p):
 
 @pytest.mark.parametrize("N,K,ldq", [(16, 1, 16), (16, 33, 32), (48, 1000, 64),
                                      (1552, 777, 1568), (528, 1025, 528), (512, 512, 512),
-                                     (2048, 4096, 2048)])
+                                     (2048, 4096, 2048), (2064, 300, 2064), (4096, 2000, 4112),
+                                     (6160, 129, 6160)])
 @pytest.mark.parametrize("p", [0.0, 0.3, 1.0])
 def test_ragged_shapes(N, K, ldq, p):
     """N not a multiple of the 512-channel tile, K with a ragged last word
@@ -136,3 +137,15 @@ def test_acc_or_y_only():
     plan.decode(to_dev(c["bits"]), "bits", None, y)
     torch.cuda.synchronize()
     assert_parity(acc, y, want_acc[0], want_y[0], "split outputs")
+
+
+def test_dense_long_rows_multi_round():
+    """p = 0.95 over K = 100000 with N = 4096 (two output tiles, ~190k
+    items): each CTA's share spans several rounds of the streaming kernel and
+    tiles cross CTAs and rounds."""
+    N, K = 4096, 100000
+    Qc, s, x = synth.random_case(21, N, K, T=1, p=0.95)
+    want_acc, want_y = oracle.project(Qc, s, N, K, x, "u8")
+    plan = sp.Plan(to_dev(Qc), to_dev(s), N, K)
+    acc, y = run_decode(plan, to_dev(synth.pack_bits(x)[0]), "bits", N)
+    assert_parity(acc, y, want_acc[0], want_y[0], "multi-round")

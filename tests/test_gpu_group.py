@@ -101,3 +101,30 @@ def test_mixed_group_shapes():
         a, yy = oracle.project(Qc, s, N, K, xs[j], "u8", ldq=ldq)
         assert_parity(acc[j, :N], y[j, :N], a[0], yy[0], f"member {j}")
     group.close()
+
+
+def test_group_of_64_uncached_masks():
+    """The largest group (64 projections): 64 x 6144 columns of spike words
+    exceed the shared-memory mask cache, so the kernel reads them from global
+    memory; rates vary per member, some members have no spike at all."""
+    N, K = 64, 6144
+    weights, plans = [], []
+    rng = synth.rng_for(99)
+    rates = rng.uniform(0.0, 0.3, 64)
+    rates[[3, 17, 40]] = 0.0
+    X = (rng.random((64, K)) < rates[:, None]).astype(np.uint8)
+    for j in range(64):
+        Qc, s, _ = synth.random_case(200 + j, N, K, T=1)
+        weights.append((Qc, s))
+        plans.append(sp.Plan(to_dev(Qc), to_dev(s), N, K))
+    group = sp.Group(plans)
+    acc = torch.full((64, N), 3, dtype=torch.int32, device=DEV)
+    y = torch.full((64, N), 3.0, dtype=torch.float32, device=DEV)
+    bits = synth.pack_bits(X)
+    group.decode(to_dev(bits), "bits", bits.shape[1], acc, y, N)
+    torch.cuda.synchronize()
+    for j, (Qc, s) in enumerate(weights):
+        a, yy = oracle.project(Qc, s, N, K, X[j], "u8")
+        assert_parity(acc[j], y[j], a[0], yy[0], f"member {j}")
+    assert group.status() == sp.SP_OK
+    group.close()
