@@ -137,6 +137,7 @@ GatherParams1 single_params(const sp_plan_s* p, const void* spikes, int fmt, int
   g.nprob = 1;
   g.B = B;
   g.units_total = B * gather_units(p->N, p->K);
+  g.max_units = gather_units(p->N, p->K);
   g.fmt = fmt;
   g.spikes = spikes;
   g.ld_spikes = ld;
@@ -381,6 +382,7 @@ sp_status spike_proj_group_create(sp_group_t* group, const sp_plan_t* plans, int
     P.ws_begin = (int32_t)ws;
     P.ticket_begin = (int32_t)tk;
     units += gather_units(p->N, p->K);
+    if (gather_units(p->N, p->K) > g->params.max_units) g->params.max_units = gather_units(p->N, p->K);
     ws += p->N;
     tk += gather_ntiles(p->N);
     if (p->N > g->maxN) g->maxN = p->N;

@@ -35,17 +35,7 @@ namespace {
 constexpr int kWarps = kGatherWarps;               // 4
 constexpr int kWords = kGatherCK / 32;             // spike words per chunk (16)
 constexpr int kPerWarp = kGatherCK / kWarps;       // column-list capacity per warp
-constexpr int kLoadBatch = 12;                     // column loads in flight per lane
-
-template <int NP>
-__device__ __forceinline__ int find_problem(const GatherParamsT<NP>& p, int u) {
-  int lo = 0, hi = p.nprob - 1;            // largest j with unit_begin_j * B <= u
-  while (lo < hi) {
-    const int mid = (lo + hi + 1) >> 1;
-    if (p.prob[mid].unit_begin * p.B <= u) lo = mid; else hi = mid - 1;
-  }
-  return lo;
-}
+constexpr int kLoadBatch = 11;                     // column loads in flight per lane (72 registers)
 
 template <int NP>
 __global__ void __launch_bounds__(kGatherThreads, 7)
@@ -57,22 +47,19 @@ gather_kernel(const __grid_constant__ GatherParamsT<NP> p) {
   const int lane = threadIdx.x & 31;
   const int warp = threadIdx.x >> 5;
 
-  for (int u = blockIdx.x; u < p.units_total; u += gridDim.x) {
-    // ---- decode the unit ---------------------------------------------------
-    const int j = find_problem(p, u);
+  // grid = (tokens x units of the largest problem, problems): token t, unit x
+  // of problem blockIdx.y; the output tile is the fastest index so that the
+  // tiles of one column chunk run side by side
+  {
+    const int j = blockIdx.y;
+    const int t = (int)(blockIdx.x / (unsigned)p.max_units);
+    const int x = (int)blockIdx.x - t * p.max_units;
     const GatherProblem& P = p.prob[j];
     const int kch = gather_kchunks(P.K);
     const int ntile = gather_ntiles(P.N);
-    const int upt = ntile * kch;
-    const int ul = u - P.unit_begin * p.B;
-    const int t = ul / upt;
-    const int r = ul - t * upt;
-    const int nt = r / kch;
-    const int kc = r - nt * kch;
-    if (t >= p.B) {                          // cannot happen for a valid table
-      if (threadIdx.x == 0) atomicExch(p.err, kErrBadUnit);
-      return;
-    }
+    if (x >= ntile * kch) return;           // this problem has fewer units
+    const int kc = x / ntile;
+    const int nt = x - kc * ntile;
     const int n0 = nt * kGatherNT;
     const int k0 = kc * kGatherCK;
     const int64_t row = (int64_t)j * p.B + t;
@@ -159,18 +146,24 @@ gather_kernel(const __grid_constant__ GatherParamsT<NP> p) {
         const int v = s_red[0][o] + s_red[1][o] + s_red[2][o] + s_red[3][o];
         if (v) atomicAdd(ws + n, v);
       }
-      __threadfence();
+      // Release: the barrier orders the CTA's red.adds before thread 0, whose
+      // GPU-scope fence makes them visible before its ticket increment.  The
+      // thread that completes the tile fences again (acquire) before the CTA
+      // reads the workspace back.
       __syncthreads();
       if (threadIdx.x == 0) {
         uint32_t* tk = p.tickets + (int64_t)P.ticket_begin * p.B + (int64_t)t * ntile + nt;
+        __threadfence();
         const uint32_t prev = atomicAdd(tk, 1u);
         const int last = prev == (uint32_t)(kch - 1);
-        if (last) atomicExch(tk, 0u);       // every chunk has arrived: reset
+        if (last) {
+          atomicExch(tk, 0u);               // every chunk has arrived: reset
+          __threadfence();
+        }
         s_last = last;
       }
       __syncthreads();
       if (s_last) {
-        __threadfence();
         int vals[kGatherNT / kGatherThreads];
 #pragma unroll
         for (int q = 0; q < kGatherNT / kGatherThreads; ++q) {
@@ -188,16 +181,16 @@ gather_kernel(const __grid_constant__ GatherParamsT<NP> p) {
         }
       }
     }
-    __syncthreads();   // shared buffers are reused by the next unit
   }
 }
 
 template <int NP>
 cudaError_t launch_gather_t(const GatherParamsT<NP>& p, cudaStream_t s) {
-  if (p.units_total <= 0) return cudaSuccess;
+  if (p.units_total <= 0 || p.B <= 0 || p.max_units <= 0) return cudaSuccess;
+  if ((int64_t)p.max_units * p.B > 0x7fffffffll) return cudaErrorInvalidConfiguration;
   // one CTA per unit; the hardware keeps every unit of a decode step resident
   // (7 CTAs of 128 threads per SM) and schedules the rest in waves
-  const int grid = p.units_total < (1 << 30) ? p.units_total : (1 << 30);
+  const dim3 grid((unsigned)(p.max_units * p.B), (unsigned)p.nprob, 1);
   gather_kernel<NP><<<grid, kGatherThreads, 0, s>>>(p);
   return cudaGetLastError();
 }

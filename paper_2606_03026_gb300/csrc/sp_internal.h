@@ -57,6 +57,7 @@ struct GatherParamsT {
   int32_t nprob;
   int32_t B;              // tokens per problem (1 for groups)
   int32_t units_total;    // B * sum_j units_per_token(j)
+  int32_t max_units;      // largest units_per_token(j): grid.x = B * max_units
   int32_t fmt;            // sp_fmt
   const void* spikes;     // row (j*B + t) at spikes + row*ld_spikes elements
   int64_t ld_spikes;
