@@ -47,6 +47,7 @@ extern "C" {
 #define SPIKE_PROJ_ABI_VERSION 1
 #define SPIKE_PROJ_MAX_K 131072        /* 128 * K < 2^24: exact FP32 conversion */
 #define SPIKE_PROJ_MAX_GROUP 64        /* projections per group */
+#define SPIKE_PROJ_NOALLOC_MAX_N 32768 /* largest N of spike_proj_decode_noalloc */
 
 typedef struct sp_plan_s *sp_plan_t;
 typedef struct sp_group_s *sp_group_t;
@@ -61,8 +62,10 @@ typedef enum sp_status {
     SP_ENOMEM = 5,        /* workspace allocation failed */
     SP_ERANGE = 6,        /* K above SPIKE_PROJ_MAX_K, or batch above the plan's max */
     SP_EKERNEL = 7,       /* a kernel raised the device error word */
-    SP_EUNSUPPORTED = 8   /* strategy not available for this plan (e.g. SP_GEMM
+    SP_EUNSUPPORTED = 8,  /* strategy not available for this plan (e.g. SP_GEMM
                              without SP_PLAN_GEMM) */
+    SP_ESCRATCH = 9       /* N above SPIKE_PROJ_NOALLOC_MAX_N: the fixed scratch
+                             of spike_proj_decode_noalloc is too small */
 } sp_status;
 
 /* Spike row formats.
@@ -213,6 +216,47 @@ sp_status spike_proj_group_decode_host(sp_group_t group, const void *h_spikes,
 
 /* Reads and clears the group's device error word (synchronises `stream`). */
 sp_status spike_proj_group_status(sp_group_t group, sp_stream_t stream);
+
+/* ---------------------------------------------------------------------------
+ * spike_proj_decode_noalloc -- batch-1 decode (Eq. (sparse)) that allocates
+ * no memory at all.  The paper has no counterpart: this is a library
+ * convenience, not part of the method.
+ *
+ * Who needs it: callers that may not allocate device memory on their decode
+ * path -- a serving loop where cudaMalloc / cudaFree would synchronise the
+ * device and stall every other stream, a process whose device memory is
+ * already handed out in full by another allocator, or code that has no place
+ * to keep a plan handle and free it later.  It takes the projection's
+ * arguments directly (no plan) and gives the same bits as
+ * spike_proj_decode on a plan of the same W, scale, N and K.
+ *
+ * Scratch: the split-K workspace, tile tickets and error word live in one
+ * fixed array of static device memory inside the library (about 128.5 KiB
+ * per device: SPIKE_PROJ_NOALLOC_MAX_N INT32 words plus 128 words), so N is
+ * limited to SPIKE_PROJ_NOALLOC_MAX_N; a larger N returns SP_ESCRATCH before
+ * anything is enqueued.  No cudaMalloc, cudaFree or other allocating call is
+ * made, on the first call or later.
+ *
+ * First call per device: it checks the device, looks up the scratch address
+ * on the current device, clears the scratch on `stream` and synchronises
+ * that stream.  Make the first call on each device before any stream
+ * capture begins; later calls on that device only enqueue the kernel.
+ *
+ * Concurrency: every call on one device shares the one scratch, whatever its
+ * W.  Calls whose kernels can overlap on the GPU race on it and give wrong
+ * results: issue them on one stream, or order the streams.  The kernel
+ * leaves the scratch zeroed for the next call.
+ *
+ *   W, ldw, scale, N, K   as for spike_proj_plan (W, scale borrowed for the
+ *                         duration of the call); N <= SPIKE_PROJ_NOALLOC_MAX_N.
+ *   spikes, fmt, acc, y   as for spike_proj_decode.
+ * Errors: SP_EINVAL, SP_EALIGN, SP_ERANGE, SP_ESCRATCH, SP_EDEVICE, SP_ECUDA.
+ * ------------------------------------------------------------------------- */
+sp_status spike_proj_decode_noalloc(const int8_t *W, int64_t ldw,
+                                    const float *scale, int32_t N, int32_t K,
+                                    const void *spikes, sp_fmt fmt,
+                                    int32_t *acc, float *y,
+                                    sp_stream_t stream);
 
 /* --------------------------------------------------------------------------- */
 const char *spike_proj_strerror(sp_status status);

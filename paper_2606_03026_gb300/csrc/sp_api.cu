@@ -1,14 +1,26 @@
 // sp_api.cu -- the C ABI of libspikeproj.so: argument validation, plans and
 // groups (workspace ownership), per-call dispatch between the gather, union
 // and tensor-core kernels, and status reporting.  See include/spike_proj.h.
+#include <atomic>
 #include <cstdlib>
 #include <cstring>
+#include <mutex>
 #include <new>
 
 #include "sp_gemm.h"
 #include "sp_internal.h"
 
 using namespace sp;
+
+// Scratch of spike_proj_decode_noalloc, one copy per device in static device
+// memory: the INT32 split-K workspace of one spike row at the largest N, one
+// ticket per 512-channel output tile, and the kernel's error word (the tail is
+// padding).  Zero when the module loads; the gather kernel leaves it zero.
+constexpr int kNoallocMaxN = SPIKE_PROJ_NOALLOC_MAX_N;
+constexpr int kNoallocTickets = kNoallocMaxN / kGatherNT;
+constexpr int kNoallocWords = kNoallocMaxN + 2 * kNoallocTickets;
+static_assert(kNoallocMaxN % kGatherNT == 0, "whole output tiles");
+static __device__ __align__(256) int32_t g_noalloc_scratch[kNoallocWords];
 
 struct sp_plan_s {
   int device = 0;
@@ -227,6 +239,36 @@ sp_status run_multi(sp_plan_s* p, const void* spikes, int fmt, int B, int64_t ld
     case SP_GEMM: return run_gemm(p, spikes, fmt, B, ld, acc, y, s);
     default: return SP_EINVAL;
   }
+}
+
+// Per-device address of g_noalloc_scratch, set once by the first call on the
+// device (with that device current).  Later calls read it without a lock.
+constexpr int kNoallocDevices = 64;
+std::mutex g_noalloc_mu;
+std::atomic<int32_t*> g_noalloc_ptr[kNoallocDevices];
+
+sp_status noalloc_scratch(cudaStream_t s, int32_t** out) {
+  int dev = 0;
+  SP_CUDA(cudaGetDevice(&dev));
+  if (dev < 0 || dev >= kNoallocDevices) return SP_EDEVICE;
+  int32_t* ptr = g_noalloc_ptr[dev].load(std::memory_order_acquire);
+  if (!ptr) {
+    std::lock_guard<std::mutex> lock(g_noalloc_mu);
+    ptr = g_noalloc_ptr[dev].load(std::memory_order_relaxed);
+    if (!ptr) {
+      int checked = 0;
+      const sp_status st = check_device(&checked);
+      if (st != SP_OK) return st;
+      void* sym = nullptr;
+      SP_CUDA(cudaGetSymbolAddress(&sym, g_noalloc_scratch));
+      SP_CUDA(cudaMemsetAsync(sym, 0, sizeof(g_noalloc_scratch), s));
+      SP_CUDA(cudaStreamSynchronize(s));
+      ptr = static_cast<int32_t*>(sym);
+      g_noalloc_ptr[dev].store(ptr, std::memory_order_release);
+    }
+  }
+  *out = ptr;
+  return SP_OK;
 }
 
 }  // namespace
@@ -488,6 +530,44 @@ sp_status spike_proj_group_status(sp_group_t g, sp_stream_t stream) {
   return SP_EKERNEL;
 }
 
+sp_status spike_proj_decode_noalloc(const int8_t* W, int64_t ldw, const float* scale, int32_t N,
+                                    int32_t K, const void* spikes, sp_fmt fmt, int32_t* acc,
+                                    float* y, sp_stream_t stream) {
+  if (!W || !scale) return SP_EINVAL;
+  sp_status st = check_io(spikes, fmt, acc, y);
+  if (st != SP_OK) return st;
+  if (N < 16) return SP_EINVAL;
+  if (N > kNoallocMaxN) return SP_ESCRATCH;
+  if (K < 1 || K > SPIKE_PROJ_MAX_K) return SP_ERANGE;
+  if (N % 16 != 0 || ldw < N || ldw % 16 != 0 || ldw > INT32_MAX) return SP_EALIGN;
+  if (!aligned(W, 16) || !aligned(scale, 4)) return SP_EALIGN;
+  cudaStream_t s = as_stream(stream);
+  int32_t* scratch = nullptr;
+  if ((st = noalloc_scratch(s, &scratch)) != SP_OK) return st;
+  GatherParams1 g;
+  std::memset(&g, 0, sizeof(g));
+  g.prob[0].W = W;
+  g.prob[0].scale = scale;
+  g.prob[0].ldw = (int32_t)ldw;
+  g.prob[0].N = N;
+  g.prob[0].K = K;
+  g.nprob = 1;
+  g.B = 1;
+  g.units_total = gather_units(N, K);
+  g.max_units = gather_units(N, K);
+  g.fmt = fmt;
+  g.spikes = spikes;
+  g.ld_spikes = row_elems(fmt, K);
+  g.acc = acc;
+  g.y = y;
+  g.ld_out = N;
+  g.ws = scratch;
+  g.tickets = reinterpret_cast<uint32_t*>(scratch + kNoallocMaxN);
+  g.err = scratch + kNoallocMaxN + kNoallocTickets;
+  SP_CUDA(launch_gather(g, s));
+  return SP_OK;
+}
+
 const char* spike_proj_strerror(sp_status status) {
   switch (status) {
     case SP_OK: return "success";
@@ -499,6 +579,9 @@ const char* spike_proj_strerror(sp_status status) {
     case SP_ERANGE: return "size out of range (K above 131072 or batch above the plan's maximum)";
     case SP_EKERNEL: return "a kernel reported an error (device error word set)";
     case SP_EUNSUPPORTED: return "strategy not available for this plan";
+    case SP_ESCRATCH:
+      return "N above SPIKE_PROJ_NOALLOC_MAX_N (32768): too large for the fixed scratch of "
+             "spike_proj_decode_noalloc";
   }
   return "unknown status";
 }

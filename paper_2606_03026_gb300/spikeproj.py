@@ -14,7 +14,7 @@ LIB_PATH = Path(__file__).resolve().parent / "_build" / "libspikeproj.so"
 
 # sp_status
 SP_OK, SP_EINVAL, SP_EALIGN, SP_EDEVICE, SP_ECUDA, SP_ENOMEM, SP_ERANGE, \
-    SP_EKERNEL, SP_EUNSUPPORTED = range(9)
+    SP_EKERNEL, SP_EUNSUPPORTED, SP_ESCRATCH = range(10)
 # sp_fmt
 SP_SPIKES_BITS32, SP_SPIKES_U8 = 0, 1
 # sp_kernel
@@ -22,6 +22,7 @@ SP_AUTO, SP_GATHER, SP_UNION, SP_GEMM = 0, 1, 2, 3
 SP_PLAN_GEMM = 0x1
 SPIKE_PROJ_MAX_K = 131072
 SPIKE_PROJ_MAX_GROUP = 64
+SPIKE_PROJ_NOALLOC_MAX_N = 32768
 
 FMTS = {"bits": SP_SPIKES_BITS32, "u8": SP_SPIKES_U8}
 KERNELS = {"auto": SP_AUTO, "gather": SP_GATHER, "union": SP_UNION, "gemm": SP_GEMM}
@@ -44,6 +45,8 @@ _SIGNATURES = {
     "spike_proj_group_decode_host": ([_P, _P, ctypes.c_int, _I64, _P, _P, _I64, _P],
                                      ctypes.c_int),
     "spike_proj_group_status": ([_P, _P], ctypes.c_int),
+    "spike_proj_decode_noalloc": ([_P, _I64, _P, _I32, _I32, _P, ctypes.c_int, _P, _P, _P],
+                                  ctypes.c_int),
     "spike_proj_strerror": ([ctypes.c_int], ctypes.c_char_p),
     "spike_proj_last_cuda_error": ([], ctypes.c_int),
     "spike_proj_abi_version": ([], ctypes.c_int),
@@ -185,6 +188,15 @@ def spike_proj_group_decode_host(group, h_spikes, fmt, ld_spikes, h_acc=None, h_
 
 def spike_proj_group_status(group, stream=None) -> int:
     return lib().spike_proj_group_status(group, _stream(stream))
+
+
+def spike_proj_decode_noalloc(W, ldw, scale, N, K, spikes, fmt, acc=None, y=None,
+                              stream=None):
+    """Batch-1 decode without a plan and without any allocation (the
+    library's fixed per-device scratch; N <= SPIKE_PROJ_NOALLOC_MAX_N)."""
+    _check(lib().spike_proj_decode_noalloc(_addr(W), ldw, _addr(scale), N, K, _addr(spikes),
+                                           _fmt(fmt), _addr(acc), _addr(y), _stream(stream)),
+           "spike_proj_decode_noalloc")
 
 
 def spike_proj_strerror(status) -> str:
