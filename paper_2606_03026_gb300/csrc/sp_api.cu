@@ -38,7 +38,8 @@ struct sp_plan_s {
   // tensor-core path
   __nv_bfloat16* Wb = nullptr;    // [N][Kp] bf16 K-major
   __nv_bfloat16* Xb = nullptr;    // [xb_rows][Kp] bf16 spike staging
-  int Kp = 0, xb_rows = 0;
+  float* part = nullptr;          // split-K partials, part_units x 128 x 256 fp32
+  int Kp = 0, xb_rows = 0, part_units = 0;
   GemmMaps maps;
   sp_kernel last_kernel = SP_AUTO;
   int32_t last_active = -1;
@@ -114,6 +115,7 @@ void plan_free(sp_plan_s* p) {
   if (p->h_counts) cudaFreeHost(p->h_counts);
   cudaFree(p->Wb);
   cudaFree(p->Xb);
+  cudaFree(p->part);
   delete p;
 }
 
@@ -206,6 +208,8 @@ sp_status run_gemm(sp_plan_s* p, const void* spikes, int fmt, int T, int64_t ld,
   g.N = p->N;
   g.K = p->K;
   g.err = p->err;
+  g.part = p->part;
+  g.part_units = p->part_units;
   SP_CUDA(launch_gemm(p->maps, T, p->N, p->Kp, g, s));
   return SP_OK;
 }
@@ -321,8 +325,17 @@ sp_status spike_proj_plan(sp_plan_t* plan, const int8_t* W, int64_t ldw, const f
   if (flags & SP_PLAN_GEMM) {
     p->Kp = gemm_k_pad(K);
     p->xb_rows = ceil_div(max_batch, 128) * 128;
+    // a split-K launch has at most one unit per SM
+    int sms = 0;
+    e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (e != cudaSuccess) {
+      plan_free(p);
+      return cuda_fail(e);
+    }
+    p->part_units = sms;
     if ((st = dev_alloc_zero(&p->Wb, (size_t)N * p->Kp, s)) != SP_OK ||
-        (st = dev_alloc_zero(&p->Xb, (size_t)p->xb_rows * p->Kp, s)) != SP_OK) {
+        (st = dev_alloc_zero(&p->Xb, (size_t)p->xb_rows * p->Kp, s)) != SP_OK ||
+        (st = dev_alloc_zero(&p->part, (size_t)p->part_units * kGemmPartialElems, s)) != SP_OK) {
       plan_free(p);
       return st;
     }

@@ -12,22 +12,24 @@
 // of magnitude <= 128 * K < 2^24, so no fp32 addition ever rounds.  The
 // epilogue converts the accumulator to INT32 without loss.
 //
-// Kernel structure (one CTA per SM, persistent over work units):
+// Kernel structure:
 //   warp 0      TMA producer: 128x64 (X) and 256x64 (W) bf16 boxes, 128-byte
 //               swizzle, into a 4-stage shared-memory ring (mbarriers)
 //   warp 1      allocates 512 TMEM columns (two 128x256 fp32 accumulators) and
 //               issues tcgen05.mma (M=128, N=256, K=16) from one thread;
 //               tcgen05.commit frees ring slots and publishes accumulators
-//   warps 2-5   epilogue: tcgen05.ld 32 columns at a time, transpose through
-//               shared memory so each warp store covers 128 contiguous bytes
-//               of one output row, then either write acc / y, or (split K)
-//               add the INT32 partial into the workspace; the warp that
-//               completes the last split of its 32-row quarter of a tile
-//               (atomic ticket per quarter) writes acc / y and re-zeroes the
-//               workspace.
-// A work unit is (128-row block, 256-column block, K split).  K is split so
-// that units ~ number of SMs when the output has few tiles (T = 512 gives only
-// 24 tiles of 128x256 for N = 1536).
+//   warps 2-5   epilogue: warp w reads TMEM lane quarter w % 4 (32 rows),
+//               32 columns per tcgen05.ld
+// Whole K (enough output tiles for every SM): one CTA per SM, persistent over
+// 128x256 tiles; the epilogue of one tile overlaps the next tile's MMAs
+// (double-buffered accumulator) and writes acc / y through a shared-memory
+// transpose so that every store covers 128 contiguous bytes of a row.
+// Split K (few output tiles, e.g. T = 512 rows give 4 x 6 tiles for N =
+// 1536): the S CTAs of a thread-block cluster hold one tile for S K ranges.
+// Each CTA stores the 32-column chunks it does not own (chunk c belongs to
+// cluster rank c % S) into an fp32 workspace that stays in L2, one cluster
+// barrier (release / acquire) publishes them, and each owner adds the S - 1
+// partials of its chunks to its own accumulator and writes acc / y.
 //
 // Every mbarrier wait is bounded (2^31 SM cycles, about a second); on
 // timeout the kernel sets the error word, stops issuing work, drains what it
@@ -73,27 +75,26 @@ __device__ __forceinline__ uint64_t smem_desc_k128(const void* p) {
 constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(BN >> 3) << 17) |
                             ((uint32_t)(BM >> 4) << 24);
 
-constexpr int kSlotBytes = 32 * BM * 4;        // one 128-row x 32-column fp32 partial
-
 __device__ __forceinline__ uint32_t cluster_ctarank() {
   uint32_t r;
   asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
   return r;
 }
-// Arrive + wait on the cluster barrier (release / acquire: shared-memory
-// writes to other CTAs of the cluster before it are visible after it).
-// Every thread of every CTA of the cluster executes it.
+// Arrive + wait on the cluster barrier (release / acquire at cluster scope:
+// memory writes of every thread of the cluster before it are visible to
+// every thread of the cluster after it).  Every thread of every CTA of the
+// cluster executes it.
 __device__ __forceinline__ void cluster_sync() {
-  asm volatile("barrier.cluster.arrive;\n\tbarrier.cluster.wait;" ::: "memory");
+  asm volatile("barrier.cluster.arrive.release;\n\tbarrier.cluster.wait.acquire;" ::: "memory");
 }
-__device__ __forceinline__ uint32_t map_to_rank(uint32_t smem_addr, uint32_t rank) {
-  uint32_t r;
-  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(smem_addr), "r"(rank));
-  return r;
-}
-__device__ __forceinline__ void st_cluster_u32(uint32_t addr, uint32_t v) {
-  asm volatile("st.shared::cluster.u32 [%0], %1;" ::"r"(addr), "r"(v) : "memory");
-}
+
+// Split-K exchange: one partial chunk (32 columns x 128 rows fp32) is 16 KB;
+// a rank owns at most kMaxOwned of the 8 chunks (S >= 2), and the S - 1
+// incoming partials of its chunks fit the idle ring: (S - 1) * ceil(8 / S)
+// chunks <= 12 for S <= 8.
+constexpr int kPartChunkBytes = 32 * BM * 4;
+constexpr int kMaxOwned = 4;
+static_assert(12 * kPartChunkBytes <= (int)SMEM_RING, "split-K partials fit the ring");
 
 struct GemmArgs {
   GemmParams p;
@@ -110,26 +111,42 @@ __device__ __forceinline__ void unit_coords(const GemmArgs& a, int u, int& tile,
   kb1 = min(a.nkb, kb0 + a.kb_per_split);
 }
 
+// Scale of output column n for the calling lane (0 when y is not written).
+__device__ __forceinline__ float column_scale(const GemmParams& p, int n) {
+  return (p.y && n < p.N) ? __ldg(p.scale + n) : 0.f;
+}
+
 // One warp writes a 32-row x 32-column chunk of integer-valued fp32 sums
 // (v[i] = column col0 + i of row row0 + lane): transposed through shared
 // memory so that each store instruction covers 32 consecutive columns of one
-// row; acc = exact int conversion, y = s * float(acc).
+// row; acc = exact int conversion, y = s * float(acc) with sc = the scale of
+// column col0 + lane.
 __device__ __forceinline__ void store_chunk(const GemmParams& p, uint32_t* tr,
-                                            const uint32_t (&v)[32], int row0, int col0) {
+                                            const uint32_t (&v)[32], int row0, int col0,
+                                            float sc) {
   const int lane = threadIdx.x & 31;
 #pragma unroll
   for (int i = 0; i < 32; ++i) tr[lane * TR_STRIDE + i] = v[i];
   __syncwarp();
   const int n = col0 + lane;
+  const int nrows = p.T - row0 < 32 ? p.T - row0 : 32;
   if (n < p.N) {
-    const float sc = p.y ? __ldg(p.scale + n) : 0.f;
-    for (int rr = 0; rr < 32; ++rr) {
-      const int r = row0 + rr;
-      if (r >= p.T) break;
-      const int val = __float2int_rn(__uint_as_float(tr[rr * TR_STRIDE + lane]));
-      const int64_t o = (int64_t)r * p.N + n;
-      if (p.acc) p.acc[o] = val;
-      if (p.y) p.y[o] = scale_out(sc, val);
+    int32_t* acc = p.acc ? p.acc + (int64_t)row0 * p.N + n : nullptr;
+    float* y = p.y ? p.y + (int64_t)row0 * p.N + n : nullptr;
+    if (nrows == 32) {
+      // full chunk: unrolled, so the 32 shared-memory reads are in flight together
+#pragma unroll
+      for (int rr = 0; rr < 32; ++rr) {
+        const int val = __float2int_rn(__uint_as_float(tr[rr * TR_STRIDE + lane]));
+        if (acc) acc[(int64_t)rr * p.N] = val;
+        if (y) y[(int64_t)rr * p.N] = scale_out(sc, val);
+      }
+    } else {
+      for (int rr = 0; rr < nrows; ++rr) {
+        const int val = __float2int_rn(__uint_as_float(tr[rr * TR_STRIDE + lane]));
+        if (acc) acc[(int64_t)rr * p.N] = val;
+        if (y) y[(int64_t)rr * p.N] = scale_out(sc, val);
+      }
     }
   }
   __syncwarp();
@@ -150,7 +167,8 @@ gemm_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CU
   uint64_t* tfull = bars + 2 * STAGES;   // [2] MMA -> epilogue
   uint64_t* tempty = tfull + 2;          // [2] epilogue -> MMA
   uint64_t* done = tempty + 2;           // all MMAs retired
-  uint32_t* s_tmem = reinterpret_cast<uint32_t*>(done + 1);
+  uint64_t* pfull = done + 1;            // split K: peers' partials landed
+  uint32_t* s_tmem = reinterpret_cast<uint32_t*>(pfull + 1);
   volatile int* s_abort = reinterpret_cast<volatile int*>(s_tmem + 1);
 
   const int warp = threadIdx.x >> 5;
@@ -166,6 +184,7 @@ gemm_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CU
       mbar_init(&tempty[b], 4);          // one arrive per epilogue warp
     }
     mbar_init(done, 1);
+    mbar_init(pfull, 1);
     *s_abort = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     tma_prefetch_desc(&mapA);
@@ -273,7 +292,7 @@ gemm_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CU
       for (int c = 0; c < BN; c += 32) {
         uint32_t v[32];
         tmem_ld32(tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(ab * BN + c), v);
-        store_chunk(a.p, tr, v, row0, nb * BN + c);
+        store_chunk(a.p, tr, v, row0, nb * BN + c, column_scale(a.p, nb * BN + c + lane));
       }
       tc_fence_before();
       __syncwarp();
@@ -281,13 +300,8 @@ gemm_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CU
       if (++ab == 2) { ab = 0; aph ^= 1u; }
     }
   } else {
-    // ---------------- epilogue (split K): cluster reduce-scatter ---------------
-    // The CTAs of one cluster hold the same output tile for different K ranges.
-    // Output chunk c (32 columns) belongs to cluster rank c % S.  After every
-    // CTA's MMAs have retired (cluster barrier 1: each ring is free), each CTA
-    // writes its partial of every chunk it does not own into the owner's ring
-    // through distributed shared memory; after cluster barrier 2 each owner
-    // adds the S partials of its chunks and writes acc and y.
+    // ---------------- epilogue (split K): reduce-scatter through L2 -----------
+    // One unit per CTA.  Wait for this CTA's accumulator.
     if (mbar_wait(&tfull[0], 0)) {
       tc_fence_after();
     } else {
@@ -297,42 +311,76 @@ gemm_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CU
   }
 
   if (a.splits > 1) {
+    // Partial of cluster rank r for chunk c, quarter q: 32 columns x 32 rows
+    // at part + ((tile * S + r) * 8 + c) * 4096 + q * 1024, column-major with
+    // the row fastest, so that a warp writes 128 contiguous bytes (one column
+    // of its quarter) per store, and each (r, c) partial is 16 KB contiguous.
     const int S = a.splits;
     const int rank = (int)cluster_ctarank();
-    const int maxlc = (BN / 32 + S - 1) / S;            // chunks owned per rank
     const bool epi = warp >= 2;
     const int q = warp & 3;
-    const int row = q * 32 + lane;                      // row within the tile
-    cluster_sync();                                     // 1: every ring is free
-    if (epi && !*s_abort) {
-      for (int c = 0; c < BN / 32; ++c) {
-        const int owner = c % S;
-        if (owner == rank) continue;
-        uint32_t v[32];
-        tmem_ld32(tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)c * 32u, v);
-        const int si = rank < owner ? rank : rank - 1;  // source slot at the owner
-        const uint32_t slot = smem_u32(smem) + (uint32_t)((si * maxlc + c / S) * kSlotBytes);
-        const uint32_t dst = map_to_rank(slot, (uint32_t)owner);
+    int tile, mb, nb, kb0, kb1;
+    unit_coords(a, blockIdx.x, tile, mb, nb, kb0, kb1);
+    const float* tile_part = a.p.part + (size_t)tile * S * (BM * BN);
+    // scales of the owned chunks' columns, in flight while the partials go out
+    float sc[kMaxOwned];
 #pragma unroll
-        for (int i = 0; i < 32; ++i) st_cluster_u32(dst + (uint32_t)(i * BM + row) * 4u, v[i]);
+    for (int j = 0; j < kMaxOwned; ++j)
+      sc[j] = (epi && rank + j * S < BN / 32) ? column_scale(a.p, nb * BN + (rank + j * S) * 32 + lane)
+                                              : 0.f;
+    if (epi && !*s_abort) {
+      // chunks two at a time: two TMEM loads behind one wait
+      float* mine = a.p.part + ((size_t)tile * S + rank) * (BM * BN) + q * 1024 + lane;
+      for (int c = 0; c < BN / 32; c += 2) {
+        uint32_t v0[32], v1[32];
+        tmem_ld32x2(tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)c * 32u, v0, v1);
+        if (c % S != rank) {
+          float* dst = mine + (size_t)c * 4096;
+#pragma unroll
+          for (int i = 0; i < 32; ++i) __stcg(dst + i * 32, __uint_as_float(v0[i]));
+        }
+        if ((c + 1) % S != rank) {
+          float* dst = mine + (size_t)(c + 1) * 4096;
+#pragma unroll
+          for (int i = 0; i < 32; ++i) __stcg(dst + i * 32, __uint_as_float(v1[i]));
+        }
       }
     }
-    cluster_sync();                                     // 2: partials delivered
+    cluster_sync();                                     // partials published
+    // The ring is idle (every MMA of this CTA has completed): one thread pulls
+    // the S - 1 peer partials of every owned chunk into it with bulk copies.
+    const int owned = (BN / 32 - rank + S - 1) / S;
+    if (warp == 2 && lane == 0 && !*s_abort) {
+      asm volatile("fence.proxy.async.global;" ::: "memory");
+      mbar_arrive_expect_tx(pfull, (uint32_t)((S - 1) * owned * kPartChunkBytes));
+      int slot = 0;
+      for (int c = rank; c < BN / 32; c += S)
+        for (int r = 0; r < S; ++r)
+          if (r != rank)
+            bulk_load(smem + (size_t)(slot++) * kPartChunkBytes,
+                      tile_part + ((size_t)r * 8 + c) * 4096, kPartChunkBytes, pfull);
+    }
     if (epi && !*s_abort) {
-      uint32_t* tr = s_tr + (size_t)(warp - 2) * 32 * TR_STRIDE;
-      int tile, mb, nb, kb0, kb1;
-      unit_coords(a, blockIdx.x, tile, mb, nb, kb0, kb1);
-      for (int c = rank; c < BN / 32; c += S) {
-        uint32_t v[32];
-        tmem_ld32(tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)c * 32u, v);
-        for (int si = 0; si < S - 1; ++si) {
-          const float* slot =
-              reinterpret_cast<const float*>(smem + (size_t)(si * maxlc + c / S) * kSlotBytes);
+      if (!mbar_wait(pfull, 0)) {
+        *s_abort = 1;
+        if (lane == 0) atomicExch(a.p.err, kErrMbarTimeout);
+      } else {
+        uint32_t* tr = s_tr + (size_t)(warp - 2) * 32 * TR_STRIDE;
 #pragma unroll
-          for (int i = 0; i < 32; ++i)
-            v[i] = __float_as_uint(__uint_as_float(v[i]) + slot[i * BM + row]);
+        for (int j = 0; j < kMaxOwned; ++j) {
+          const int c = rank + j * S;
+          if (c >= BN / 32) break;
+          uint32_t v[32];
+          tmem_ld32(tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)c * 32u, v);
+          for (int r = 0; r < S - 1; ++r) {
+            const float* src = reinterpret_cast<const float*>(
+                                   smem + (size_t)(j * (S - 1) + r) * kPartChunkBytes) +
+                               q * 1024 + lane;
+#pragma unroll
+            for (int i = 0; i < 32; ++i) v[i] = __float_as_uint(__uint_as_float(v[i]) + src[i * 32]);
+          }
+          store_chunk(a.p, tr, v, mb * BM + q * 32, nb * BN + c * 32, sc[j]);
         }
-        store_chunk(a.p, tr, v, mb * BM + q * 32, nb * BN + c * 32);
       }
     }
   }
@@ -366,34 +414,44 @@ __global__ void w_to_bf16_kernel(const int8_t* __restrict__ W, int64_t ldw, int 
 }
 
 // Spike rows (either format) -> bf16 0/1 [T][Kp], zero past K.  One thread
-// per 8 consecutive columns of a row.
+// per 16 consecutive columns of a row: one 16-byte load of u8 spikes (or a
+// half word of bits), two 16-byte stores.  kVec: u8 rows are 16-byte aligned
+// (base and leading dimension), so whole 16-column groups load as one vector.
+template <bool kVec>
 __global__ void spikes_to_bf16_kernel(const void* __restrict__ spikes, int fmt, int64_t ld, int T,
                                       int K, int Kp, __nv_bfloat16* __restrict__ Xb) {
-  const int per_row = Kp / 8;
+  const int per_row = Kp / 16;
   const int64_t total = (int64_t)T * per_row;
   for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < total;
        i += (int64_t)gridDim.x * blockDim.x) {
     const int t = (int)(i / per_row);
-    const int k = (int)(i - (int64_t)t * per_row) * 8;
-    uint32_t bits = 0u;                      // spikes of columns k .. k+7
+    const int k = (int)(i - (int64_t)t * per_row) * 16;
+    uint32_t bits = 0u;                      // spikes of columns k .. k+15
     if (k < K) {
       const void* row = spike_row(spikes, fmt, t, ld);
       if (fmt == SP_SPIKES_BITS32) {
-        bits = (__ldg(reinterpret_cast<const uint32_t*>(row) + (k >> 5)) >> (k & 31)) & 0xffu;
+        bits = (__ldg(reinterpret_cast<const uint32_t*>(row) + (k >> 5)) >> (k & 31)) & 0xffffu;
       } else {
         const uint8_t* x = reinterpret_cast<const uint8_t*>(row) + k;
-        const int n = K - k < 8 ? K - k : 8;
-        for (int j = 0; j < n; ++j) bits |= (uint32_t)(__ldg(x + j) != 0) << j;
+        if (kVec && K - k >= 16) {
+          const uint4 w = __ldg(reinterpret_cast<const uint4*>(x));
+          bits = nonzero_bytes_to_bits(w.x) | (nonzero_bytes_to_bits(w.y) << 4) |
+                 (nonzero_bytes_to_bits(w.z) << 8) | (nonzero_bytes_to_bits(w.w) << 12);
+        } else {
+          const int n = K - k < 16 ? K - k : 16;
+          for (int j = 0; j < n; ++j) bits |= (uint32_t)(__ldg(x + j) != 0) << j;
+        }
       }
-      if (K - k < 8) bits &= (1u << (K - k)) - 1u;
+      if (K - k < 16) bits &= (1u << (K - k)) - 1u;
     }
     // bf16 1.0 = 0x3F80; two columns per 32-bit word
-    uint4 o;
-    o.x = ((bits >> 0) & 1u ? 0x3F80u : 0u) | ((bits >> 1) & 1u ? 0x3F800000u : 0u);
-    o.y = ((bits >> 2) & 1u ? 0x3F80u : 0u) | ((bits >> 3) & 1u ? 0x3F800000u : 0u);
-    o.z = ((bits >> 4) & 1u ? 0x3F80u : 0u) | ((bits >> 5) & 1u ? 0x3F800000u : 0u);
-    o.w = ((bits >> 6) & 1u ? 0x3F80u : 0u) | ((bits >> 7) & 1u ? 0x3F800000u : 0u);
-    *reinterpret_cast<uint4*>(Xb + (int64_t)t * Kp + k) = o;
+    uint32_t o[8];
+#pragma unroll
+    for (int j = 0; j < 8; ++j)
+      o[j] = ((bits >> (2 * j)) & 1u ? 0x3F80u : 0u) | ((bits >> (2 * j + 1)) & 1u ? 0x3F800000u : 0u);
+    uint4* dst = reinterpret_cast<uint4*>(Xb + (int64_t)t * Kp + k);
+    dst[0] = make_uint4(o[0], o[1], o[2], o[3]);
+    dst[1] = make_uint4(o[4], o[5], o[6], o[7]);
   }
 }
 
@@ -447,12 +505,17 @@ cudaError_t launch_w_to_bf16(const int8_t* W, int64_t ldw, int N, int K, __nv_bf
 
 cudaError_t launch_spikes_to_bf16(const void* spikes, int fmt, int64_t ld, int T, int K, int Kp,
                                   __nv_bfloat16* Xb, cudaStream_t s) {
-  const int64_t total = (int64_t)T * (Kp / 8);
+  const int64_t total = (int64_t)T * (Kp / 16);
   const int threads = 256;
   int64_t blocks = (total + threads - 1) / threads;
-  if (blocks > 4096) blocks = 4096;
+  if (blocks > 8192) blocks = 8192;
   if (blocks < 1) blocks = 1;
-  spikes_to_bf16_kernel<<<(int)blocks, threads, 0, s>>>(spikes, fmt, ld, T, K, Kp, Xb);
+  const bool vec = fmt == SP_SPIKES_U8 && (reinterpret_cast<uintptr_t>(spikes) & 15u) == 0 &&
+                   ld % 16 == 0;
+  if (vec)
+    spikes_to_bf16_kernel<true><<<(int)blocks, threads, 0, s>>>(spikes, fmt, ld, T, K, Kp, Xb);
+  else
+    spikes_to_bf16_kernel<false><<<(int)blocks, threads, 0, s>>>(spikes, fmt, ld, T, K, Kp, Xb);
   return cudaGetLastError();
 }
 
@@ -513,7 +576,7 @@ cudaError_t launch_gemm(const GemmMaps& maps, int T, int N, int Kp, const GemmPa
     while (S > 1) {
       const int kbps = ceil_div(a.nkb, S);
       const int exact = ceil_div(a.nkb, kbps);          // splits with work
-      if (exact == S && max_active_clusters(S) >= tiles) break;
+      if (exact == S && max_active_clusters(S) >= tiles && tiles * S <= p.part_units) break;
       --S;
     }
   }

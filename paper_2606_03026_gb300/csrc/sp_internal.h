@@ -100,6 +100,8 @@ struct GemmParams {
   float* y;               // [T][N] or null
   int32_t T, N, K;
   int* err;
+  float* part;            // split-K partials, part_units x (128 x 256) fp32
+  int32_t part_units;
 };
 
 // ---------------------------------------------------------------------------
