@@ -21,12 +21,14 @@
 //      so the lanes cannot overflow),
 //   3. the 4 warps are summed through shared memory and
 //      - acc / y are written directly when the problem has a single chunk, or
-//      - the partial is added into the INT32 workspace with red.add; the CTA
-//        that completes the tile (atomic ticket == chunks - 1) reads the
-//        workspace back, writes acc and y = s * float(acc), and re-zeroes the
-//        workspace and the ticket.  No CTA ever waits on another.
+//      - the partial is added into the workspace with 16-byte fp32 vector
+//        reductions (exact: integer values below 2^24); the CTA that
+//        completes the tile (atomic ticket == chunks - 1) reads the workspace
+//        back, writes acc and y = s * float(acc), and re-zeroes the workspace
+//        and the ticket.  No CTA ever waits on another.
 // Inactive columns are never read.  Integer sums are order-free, so the
 // result is bit-identical to the definition whatever the CTA schedule.
+#include "sp_ptx.cuh"
 #include "sp_spikes.cuh"
 
 namespace sp {
@@ -36,6 +38,13 @@ constexpr int kWarps = kGatherWarps;               // 4
 constexpr int kWords = kGatherCK / 32;             // spike words per chunk (16)
 constexpr int kPerWarp = kGatherCK / kWarps;       // column-list capacity per warp
 constexpr int kLoadBatch = 11;                     // column loads in flight per lane (72 registers)
+static_assert(kGatherNT == 4 * kGatherThreads, "one 4-channel vector per thread in the flush");
+
+__device__ __forceinline__ void red_add_v4(float* addr, float a, float b, float c, float d) {
+  asm volatile("red.relaxed.gpu.global.add.v4.f32 [%0], {%1, %2, %3, %4};" ::"l"(addr), "f"(a),
+               "f"(b), "f"(c), "f"(d)
+               : "memory");
+}
 
 template <int NP>
 __global__ void __launch_bounds__(kGatherThreads, 7)
@@ -46,6 +55,10 @@ gather_kernel(const __grid_constant__ GatherParamsT<NP> p) {
 
   const int lane = threadIdx.x & 31;
   const int warp = threadIdx.x >> 5;
+  // the next launch may take free SM slots now; this grid's own memory work
+  // starts once the previous kernel has finished
+  pdl_launch_dependents();
+  pdl_wait();
 
   // grid = (tokens x units of the largest problem, problems): token t, unit x
   // of problem blockIdx.y; the output tile is the fastest index so that the
@@ -139,14 +152,23 @@ gather_kernel(const __grid_constant__ GatherParamsT<NP> p) {
         if (y_row) y_row[n] = scale_out(__ldg(P.scale + n), v);
       }
     } else {
-      int32_t* ws = p.ws + (int64_t)P.ws_begin * p.B + (int64_t)t * P.N;
-      for (int o = threadIdx.x; o < kGatherNT; o += kGatherThreads) {
-        const int n = n0 + o;
-        if (n >= P.N) break;
-        const int v = s_red[0][o] + s_red[1][o] + s_red[2][o] + s_red[3][o];
-        if (v) atomicAdd(ws + n, v);
+      // Partials go into the workspace as fp32 16-byte vector reductions (one
+      // per thread: channels n0 + 4i .. n0 + 4i + 3).  fp32 is exact here:
+      // every partial and every sum is an integer of magnitude <= 128 * K <
+      // 2^24, so the result does not depend on the order of the additions.
+      float* ws = reinterpret_cast<float*>(p.ws) + (int64_t)P.ws_begin * p.B + (int64_t)t * P.N;
+      const int o = threadIdx.x * 4;
+      const int n = n0 + o;                 // N % 16 == 0: the 4 channels are all valid or none
+      if (n < P.N) {
+        const int4 r0 = *reinterpret_cast<const int4*>(&s_red[0][o]);
+        const int4 r1 = *reinterpret_cast<const int4*>(&s_red[1][o]);
+        const int4 r2 = *reinterpret_cast<const int4*>(&s_red[2][o]);
+        const int4 r3 = *reinterpret_cast<const int4*>(&s_red[3][o]);
+        const int v0 = r0.x + r1.x + r2.x + r3.x, v1 = r0.y + r1.y + r2.y + r3.y;
+        const int v2 = r0.z + r1.z + r2.z + r3.z, v3 = r0.w + r1.w + r2.w + r3.w;
+        if (v0 | v1 | v2 | v3) red_add_v4(ws + n, (float)v0, (float)v1, (float)v2, (float)v3);
       }
-      // Release: the barrier orders the CTA's red.adds before thread 0, whose
+      // Release: the barrier orders the CTA's reductions before thread 0, whose
       // GPU-scope fence makes them visible before its ticket increment.  The
       // thread that completes the tile fences again (acquire) before the CTA
       // reads the workspace back.
@@ -163,21 +185,15 @@ gather_kernel(const __grid_constant__ GatherParamsT<NP> p) {
         s_last = last;
       }
       __syncthreads();
-      if (s_last) {
-        int vals[kGatherNT / kGatherThreads];
+      if (s_last && n < P.N) {
+        const float4 f = __ldcg(reinterpret_cast<const float4*>(ws + n));
+        __stcg(reinterpret_cast<float4*>(ws + n), make_float4(0.f, 0.f, 0.f, 0.f));
+        const int v[4] = {__float2int_rn(f.x), __float2int_rn(f.y), __float2int_rn(f.z),
+                          __float2int_rn(f.w)};
 #pragma unroll
-        for (int q = 0; q < kGatherNT / kGatherThreads; ++q) {
-          const int n = n0 + threadIdx.x + q * kGatherThreads;
-          vals[q] = n < P.N ? __ldcg(ws + n) : 0;
-        }
-#pragma unroll
-        for (int q = 0; q < kGatherNT / kGatherThreads; ++q) {
-          const int n = n0 + threadIdx.x + q * kGatherThreads;
-          if (n < P.N) {
-            __stcg(ws + n, 0);
-            if (acc_row) acc_row[n] = vals[q];
-            if (y_row) y_row[n] = scale_out(__ldg(P.scale + n), vals[q]);
-          }
+        for (int k = 0; k < 4; ++k) {
+          if (acc_row) acc_row[n + k] = v[k];
+          if (y_row) y_row[n + k] = scale_out(__ldg(P.scale + n + k), v[k]);
         }
       }
     }
@@ -191,8 +207,7 @@ cudaError_t launch_gather_t(const GatherParamsT<NP>& p, cudaStream_t s) {
   // one CTA per unit; the hardware keeps every unit of a decode step resident
   // (7 CTAs of 128 threads per SM) and schedules the rest in waves
   const dim3 grid((unsigned)(p.max_units * p.B), (unsigned)p.nprob, 1);
-  gather_kernel<NP><<<grid, kGatherThreads, 0, s>>>(p);
-  return cudaGetLastError();
+  return launch_pdl(gather_kernel<NP>, grid, dim3(kGatherThreads), 0, s, p);
 }
 
 }  // namespace

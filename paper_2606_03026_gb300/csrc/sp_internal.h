@@ -64,7 +64,7 @@ struct GatherParamsT {
   int32_t* acc;           // row (j*B + t) at acc + row*ld_out (may be null)
   float* y;               // idem (may be null)
   int64_t ld_out;
-  int32_t* ws;            // problem j token t: ws + (ws_begin_j*B + t*N_j)
+  int32_t* ws;            // problem j token t: ws + (ws_begin_j*B + t*N_j); the gather kernel adds fp32 into it
   uint32_t* tickets;      // problem j token t tile n: ticket_begin_j*B + t*ntile_j + n
   int* err;
 };
@@ -103,6 +103,25 @@ struct GemmParams {
   float* part;            // split-K partials, part_units x (128 x 256) fp32
   int32_t part_units;
 };
+
+// Launches `kernel` with programmatic stream serialization: its blocks may
+// become resident while the previous kernel of the stream is still running
+// and wait for it in pdl_wait (see sp_ptx.cuh) before touching memory.
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                       cudaStream_t s, Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr;
+  attr.id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr.val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = &attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, static_cast<Args&&>(args)...);
+}
 
 // ---------------------------------------------------------------------------
 // Host launch wrappers (defined next to their kernels).  Each returns the

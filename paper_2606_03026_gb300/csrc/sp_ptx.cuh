@@ -154,4 +154,15 @@ __device__ __forceinline__ void bulk_load(void* dst, const void* src, uint32_t b
       : "memory");
 }
 
+// Programmatic dependent launch.  pdl_launch_dependents lets the next kernel
+// of the stream (when launched with programmatic stream serialization) start
+// its blocks now; pdl_wait blocks until every kernel this one depends on has
+// completed and its memory writes are visible.  A kernel reads or writes no
+// global memory that another kernel may touch before pdl_wait.  Both are
+// no-ops for a kernel launched without a programmatic dependency.
+__device__ __forceinline__ void pdl_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
 }  // namespace sp
