@@ -15,10 +15,11 @@
 //   1. every warp reads the chunk's 16 spike words and compacts them (warp
 //      popcount and shuffle scan); warp w keeps the active columns whose rank
 //      is w modulo 4,
-//   2. each lane issues all of its warp's column loads at once (16 bytes of
-//      the 512-byte tile row per column, ld.global.nc, not allocated in L1)
-//      and adds them into biased 16-bit lanes (at most 128 columns per warp,
-//      so the lanes cannot overflow),
+//   2. each lane issues its warp's column loads, up to 19 at once (16 bytes
+//      of the 512-byte tile row per column: 11 into registers with
+//      ld.global.nc, not allocated in L1, and 8 into shared memory with
+//      cp.async) and adds them into biased 16-bit lanes (at most 128 columns
+//      per warp, so the lanes cannot overflow),
 //   3. the 4 warps are summed through shared memory and
 //      - acc / y are written directly when the problem has a single chunk, or
 //      - the partial is added into the workspace with 16-byte fp32 vector
@@ -28,6 +29,8 @@
 //        and the ticket.  No CTA ever waits on another.
 // Inactive columns are never read.  Integer sums are order-free, so the
 // result is bit-identical to the definition whatever the CTA schedule.
+#include <atomic>
+
 #include "sp_ptx.cuh"
 #include "sp_spikes.cuh"
 
@@ -37,8 +40,20 @@ namespace {
 constexpr int kWarps = kGatherWarps;               // 4
 constexpr int kWords = kGatherCK / 32;             // spike words per chunk (16)
 constexpr int kPerWarp = kGatherCK / kWarps;       // column-list capacity per warp
-constexpr int kLoadBatch = 11;                     // column loads in flight per lane (72 registers)
+constexpr int kLoadBatch = 11;                     // column loads per lane into registers (72 registers)
+constexpr int kSmemSlots = 8;                      // further column loads per lane into shared memory
 static_assert(kGatherNT == 4 * kGatherThreads, "one 4-channel vector per thread in the flush");
+
+__device__ __forceinline__ void cp_async16(void* smem, const void* gmem) {
+  const uint32_t s = (uint32_t)__cvta_generic_to_shared(smem);
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(s), "l"(gmem) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() {
+  asm volatile("cp.async.commit_group;" ::: "memory");
+}
+__device__ __forceinline__ void cp_async_wait_all() {
+  asm volatile("cp.async.wait_all;" ::: "memory");
+}
 
 __device__ __forceinline__ void red_add_v4(float* addr, float a, float b, float c, float d) {
   asm volatile("red.relaxed.gpu.global.add.v4.f32 [%0], {%1, %2, %3, %4};" ::"l"(addr), "f"(a),
@@ -46,11 +61,33 @@ __device__ __forceinline__ void red_add_v4(float* addr, float a, float b, float 
                : "memory");
 }
 
+// CTA x of the first grid row prefetches rows x, x + gridDim.x, ... of the
+// (problem, token) spike rows into L2, one 128-byte line per thread.
+template <int NP>
+__device__ __forceinline__ void prefetch_spike_rows(const GatherParamsT<NP>& p) {
+  const int rows = p.nprob * p.B;
+  for (int r = blockIdx.x; r < rows; r += gridDim.x) {
+    const int j = r / p.B;
+    const int K = p.prob[j].K;
+    const int64_t bytes = p.fmt == SP_SPIKES_BITS32 ? ((int64_t)K + 31) / 32 * 4 : (int64_t)K;
+    const char* row = static_cast<const char*>(spike_row(p.spikes, p.fmt, r, p.ld_spikes));
+    for (int64_t off = (int64_t)threadIdx.x * 128; off < bytes; off += (int64_t)kGatherThreads * 128)
+      asm volatile("prefetch.global.L2 [%0];" ::"l"(row + off));
+  }
+}
+
 template <int NP>
 __global__ void __launch_bounds__(kGatherThreads, 7)
 gather_kernel(const __grid_constant__ GatherParamsT<NP> p) {
   __shared__ int s_cols[kWarps][kPerWarp];
-  __shared__ __align__(16) int s_red[kWarps][kGatherNT];
+  // Per warp: the landing slots of its shared-memory column loads, reused for
+  // its 512 partial sums once its loads are consumed (each warp touches only
+  // its own region until the barrier before the cross-warp sum).
+  union WarpArea {
+    uint4 stage[kSmemSlots][32];
+    int red[kGatherNT];
+  };
+  __shared__ __align__(16) WarpArea s_area[kWarps];
   __shared__ int s_last;
 
   const int lane = threadIdx.x & 31;
@@ -59,6 +96,10 @@ gather_kernel(const __grid_constant__ GatherParamsT<NP> p) {
   // starts once the previous kernel has finished
   pdl_launch_dependents();
   pdl_wait();
+  // The first grid row starts first: it pulls every spike row of the launch
+  // into L2 before the column-load burst fills the DRAM queues, so that units
+  // that start late do not wait behind that burst for their spike words.
+  if (blockIdx.y == 0) prefetch_spike_rows(p);
 
   // grid = (tokens x units of the largest problem, problems): token t, unit x
   // of problem blockIdx.y; the output tile is the fastest index so that the
@@ -107,7 +148,17 @@ gather_kernel(const __grid_constant__ GatherParamsT<NP> p) {
     const int8_t* wcol = P.W + ch;
     const int64_t ldw = P.ldw;
     uint32_t ev[4] = {0u, 0u, 0u, 0u}, od[4] = {0u, 0u, 0u, 0u};
-    for (int i0 = 0; i0 < mine; i0 += kLoadBatch) {
+    uint4* stage = &s_area[warp].stage[0][lane];     // slot b at stage[32 * b]
+    // Rounds of up to kLoadBatch + kSmemSlots columns per warp, all in flight
+    // together (one round covers a unit at 10% spikes): the columns past the
+    // register batch are copied into shared memory with cp.async first, then
+    // the register batch is loaded and added, then the shared-memory columns.
+    for (int i0 = 0; i0 < mine; i0 += kLoadBatch + kSmemSlots) {
+      const int ns = min(kSmemSlots, mine - i0 - kLoadBatch);   // warp-uniform, may be <= 0
+      if (lane_on)
+        for (int b = 0; b < ns; ++b)
+          cp_async16(stage + 32 * b, wcol + s_cols[warp][i0 + kLoadBatch + b] * ldw);
+      cp_async_commit();
       uint4 v[kLoadBatch];
 #pragma unroll
       for (int b = 0; b < kLoadBatch; ++b) {
@@ -121,6 +172,14 @@ gather_kernel(const __grid_constant__ GatherParamsT<NP> p) {
         acc_bytes(v[b].z, ev[2], od[2]);
         acc_bytes(v[b].w, ev[3], od[3]);
       }
+      cp_async_wait_all();                  // this lane's copies have landed
+      for (int b = 0; b < ns; ++b) {
+        const uint4 w = stage[32 * b];
+        acc_bytes(w.x, ev[0], od[0]);
+        acc_bytes(w.y, ev[1], od[1]);
+        acc_bytes(w.z, ev[2], od[2]);
+        acc_bytes(w.w, ev[3], od[3]);
+      }
     }
     // padding loads (0x80 bytes) add 0 to the biased lanes: only the `mine`
     // real columns carry the +128 bias
@@ -133,7 +192,8 @@ gather_kernel(const __grid_constant__ GatherParamsT<NP> p) {
       unbias16(ev[1], od[1], nacc, o + 4);
       unbias16(ev[2], od[2], nacc, o + 8);
       unbias16(ev[3], od[3], nacc, o + 12);
-      int4* dst = reinterpret_cast<int4*>(&s_red[warp][lane * 16]);
+      __syncwarp();                         // every lane is done with the warp's slots
+      int4* dst = reinterpret_cast<int4*>(&s_area[warp].red[lane * 16]);
       dst[0] = make_int4(o[0], o[1], o[2], o[3]);
       dst[1] = make_int4(o[4], o[5], o[6], o[7]);
       dst[2] = make_int4(o[8], o[9], o[10], o[11]);
@@ -147,7 +207,7 @@ gather_kernel(const __grid_constant__ GatherParamsT<NP> p) {
       for (int o = threadIdx.x; o < kGatherNT; o += kGatherThreads) {
         const int n = n0 + o;
         if (n >= P.N) break;
-        const int v = s_red[0][o] + s_red[1][o] + s_red[2][o] + s_red[3][o];
+        const int v = s_area[0].red[o] + s_area[1].red[o] + s_area[2].red[o] + s_area[3].red[o];
         if (acc_row) acc_row[n] = v;
         if (y_row) y_row[n] = scale_out(__ldg(P.scale + n), v);
       }
@@ -160,10 +220,10 @@ gather_kernel(const __grid_constant__ GatherParamsT<NP> p) {
       const int o = threadIdx.x * 4;
       const int n = n0 + o;                 // N % 16 == 0: the 4 channels are all valid or none
       if (n < P.N) {
-        const int4 r0 = *reinterpret_cast<const int4*>(&s_red[0][o]);
-        const int4 r1 = *reinterpret_cast<const int4*>(&s_red[1][o]);
-        const int4 r2 = *reinterpret_cast<const int4*>(&s_red[2][o]);
-        const int4 r3 = *reinterpret_cast<const int4*>(&s_red[3][o]);
+        const int4 r0 = *reinterpret_cast<const int4*>(&s_area[0].red[o]);
+        const int4 r1 = *reinterpret_cast<const int4*>(&s_area[1].red[o]);
+        const int4 r2 = *reinterpret_cast<const int4*>(&s_area[2].red[o]);
+        const int4 r3 = *reinterpret_cast<const int4*>(&s_area[3].red[o]);
         const int v0 = r0.x + r1.x + r2.x + r3.x, v1 = r0.y + r1.y + r2.y + r3.y;
         const int v2 = r0.z + r1.z + r2.z + r3.z, v3 = r0.w + r1.w + r2.w + r3.w;
         if (v0 | v1 | v2 | v3) red_add_v4(ws + n, (float)v0, (float)v1, (float)v2, (float)v3);
@@ -200,9 +260,27 @@ gather_kernel(const __grid_constant__ GatherParamsT<NP> p) {
   }
 }
 
+// Asks for the largest shared-memory carveout once per device, so that 7
+// CTAs (7 x 18 KB of shared memory) fit on an SM beside their L1.
+template <int NP>
+cudaError_t set_carveout() {
+  static std::atomic<uint64_t> done{0};
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  const uint64_t bit = dev < 64 ? (uint64_t)1 << dev : 0;
+  if (bit && (done.load(std::memory_order_relaxed) & bit)) return cudaSuccess;
+  e = cudaFuncSetAttribute(gather_kernel<NP>, cudaFuncAttributePreferredSharedMemoryCarveout,
+                           (int)cudaSharedmemCarveoutMaxShared);
+  if (e == cudaSuccess && bit) done.fetch_or(bit, std::memory_order_relaxed);
+  return e;
+}
+
 template <int NP>
 cudaError_t launch_gather_t(const GatherParamsT<NP>& p, cudaStream_t s) {
   if (p.units_total <= 0 || p.B <= 0 || p.max_units <= 0) return cudaSuccess;
+  const cudaError_t e = set_carveout<NP>();
+  if (e != cudaSuccess) return e;
   if ((int64_t)p.max_units * p.B > 0x7fffffffll) return cudaErrorInvalidConfiguration;
   // one CTA per unit; the hardware keeps every unit of a decode step resident
   // (7 CTAs of 128 threads per SM) and schedules the rest in waves
