@@ -6,27 +6,29 @@
 // decode, a group of independent projections (a whole decode step), and the
 // per-token strategy of the batched call.
 //
-// Decomposition: a work unit is (problem j, token t, output tile of 512
-// channels, chunk of 512 input columns), and one 128-thread CTA does one
-// unit.  Units are small (about 26 KB of active columns at 10% spikes) and
-// many CTAs fit on an SM, so all units of a decode step are resident at once
-// and the memory system sees the whole step's column reads together.  Per
-// unit, with no CTA-wide barrier before the data loads:
-//   1. every warp reads the chunk's 16 spike words and compacts them (warp
-//      popcount and shuffle scan); warp w keeps the active columns whose rank
-//      is w modulo 4,
-//   2. each lane issues its warp's column loads, up to 19 at once (16 bytes
-//      of the 512-byte tile row per column: 11 into registers with
-//      ld.global.nc, not allocated in L1, and 8 into shared memory with
-//      cp.async) and adds them into biased 16-bit lanes (at most 128 columns
-//      per warp, so the lanes cannot overflow),
-//   3. the 4 warps are summed through shared memory and
-//      - acc / y are written directly when the problem has a single chunk, or
-//      - the partial is added into the workspace with 16-byte fp32 vector
-//        reductions (exact: integer values below 2^24); the CTA that
-//        completes the tile (atomic ticket == chunks - 1) reads the workspace
-//        back, writes acc and y = s * float(acc), and re-zeroes the workspace
-//        and the ticket.  No CTA ever waits on another.
+// Two forms share the per-unit work.  A unit is (problem j, token t, output
+// tile of 512 channels, chunk of input columns); per unit, with no CTA-wide
+// barrier before the data loads:
+//   1. every warp reads the chunk's spike words (one per lane) and compacts
+//      them (warp popcount and shuffle scan); warp w of W keeps the active
+//      columns whose rank is w modulo W,
+//   2. each lane issues its warp's column loads in rounds that keep them all
+//      in flight (16 bytes of the 512-byte tile row per column: a batch into
+//      registers with ld.global.nc, not allocated in L1, and a batch into
+//      shared memory with cp.async) and adds them into biased 16-bit lanes
+//      (at most 256 columns per warp, so the lanes cannot overflow),
+//   3. the warps' partials meet in shared memory.
+// Cluster form (one token per problem, K <= 6 x 1024: batch-1 decode and
+// grouped decode steps): 256-thread CTAs, chunks of up to 1024 columns, and
+// the chunk CTAs of a tile in one thread-block cluster that reduces its
+// partials through distributed shared memory (no workspace, no atomics).
+// Ticket form (any batch and K): 128-thread CTAs, 512-column chunks; acc / y
+// are written directly when a tile has a single chunk, else the partial is
+// added into the workspace with 16-byte fp32 vector reductions (exact:
+// integer values below 2^24) and the CTA that completes the tile (atomic
+// ticket == chunks - 1) reads the workspace back, writes acc and
+// y = s * float(acc), and re-zeroes the workspace and the ticket.  No CTA
+// ever waits on another.
 // Inactive columns are never read.  Integer sums are order-free, so the
 // result is bit-identical to the definition whatever the CTA schedule.
 #include <atomic>
@@ -37,12 +39,8 @@
 namespace sp {
 namespace {
 
-constexpr int kWarps = kGatherWarps;               // 4
-constexpr int kWords = kGatherCK / 32;             // spike words per chunk (16)
-constexpr int kPerWarp = kGatherCK / kWarps;       // column-list capacity per warp
-constexpr int kLoadBatch = 11;                     // column loads per lane into registers (72 registers)
-constexpr int kSmemSlots = 8;                      // further column loads per lane into shared memory
 static_assert(kGatherNT == 4 * kGatherThreads, "one 4-channel vector per thread in the flush");
+static_assert(kGatherNT / 4 <= kGatherClusterThreads, "one 4-channel group per thread");
 
 __device__ __forceinline__ void cp_async16(void* smem, const void* gmem) {
   const uint32_t s = (uint32_t)__cvta_generic_to_shared(smem);
@@ -61,6 +59,19 @@ __device__ __forceinline__ void red_add_v4(float* addr, float a, float b, float 
                : "memory");
 }
 
+__device__ __forceinline__ void cluster_sync_all() {
+  asm volatile("barrier.cluster.arrive.release;\n\tbarrier.cluster.wait.acquire;" ::: "memory");
+}
+// Stores 16 bytes into CTA `rank`'s shared memory at the address that
+// `local` has in this CTA (distributed shared memory of the cluster).
+__device__ __forceinline__ void st_peer_v4(uint32_t local, uint32_t rank, int4 v) {
+  uint32_t a;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(a) : "r"(local), "r"(rank));
+  asm volatile("st.shared::cluster.v4.s32 [%0], {%1, %2, %3, %4};" ::"r"(a), "r"(v.x), "r"(v.y),
+               "r"(v.z), "r"(v.w)
+               : "memory");
+}
+
 // CTA x of the first grid row prefetches rows x, x + gridDim.x, ... of the
 // (problem, token) spike rows into L2, one 128-byte line per thread.
 template <int NP>
@@ -71,27 +82,163 @@ __device__ __forceinline__ void prefetch_spike_rows(const GatherParamsT<NP>& p) 
     const int K = p.prob[j].K;
     const int64_t bytes = p.fmt == SP_SPIKES_BITS32 ? ((int64_t)K + 31) / 32 * 4 : (int64_t)K;
     const char* row = static_cast<const char*>(spike_row(p.spikes, p.fmt, r, p.ld_spikes));
-    for (int64_t off = (int64_t)threadIdx.x * 128; off < bytes; off += (int64_t)kGatherThreads * 128)
+    for (int64_t off = (int64_t)threadIdx.x * 128; off < bytes; off += (int64_t)blockDim.x * 128)
       asm volatile("prefetch.global.L2 [%0];" ::"l"(row + off));
   }
 }
 
+// Shared memory of one unit with W warps, chunks of at most MAXCK columns and
+// S shared-memory column slots per lane.  Per warp: its column list, and the
+// landing slots of its shared-memory column loads, reused for its 512 partial
+// sums once its loads are consumed (each warp touches only its own area
+// until the barrier before the cross-warp sum).
+template <int W, int MAXCK, int S>
+struct UnitSmem {
+  int cols[W][MAXCK / W];
+  union WarpArea {
+    uint4 stage[S][32];
+    int red[kGatherNT];
+  } area[W];
+};
+
+// One unit: the active columns of spike-row chunk [k0, k0 + ck) (ck a
+// multiple of 32, at most MAXCK <= 1024) summed over output channels
+// [n0, n0 + 512) of problem P by W warps.  Each lane keeps up to L column
+// loads in registers and S more landing in shared memory in flight.  Leaves
+// warp w's partial sums in sm.area[w].red and ends with a CTA barrier.
+template <int W, int MAXCK, int L, int S>
+__device__ __forceinline__ void unit_partial(UnitSmem<W, MAXCK, S>& sm, const GatherProblem& P,
+                                             const void* srow, int fmt, int n0, int k0, int ck) {
+  static_assert(MAXCK % 32 == 0 && MAXCK / 32 <= 32, "one spike word per lane");
+  static_assert(MAXCK / W <= 256, "biased 16-bit lanes hold at most 257 columns");
+  const int lane = threadIdx.x & 31;
+  const int warp = threadIdx.x >> 5;
+
+  // ---- 1. this warp's share of the chunk's active columns ---------------------
+  const uint32_t word = lane < ck / 32 ? spike_word(srow, fmt, P.K, k0 + 32 * lane) : 0u;
+  const int c = __popc(word);
+  int incl = c;
+#pragma unroll
+  for (int d = 1; d < 32; d <<= 1) {
+    const int v = __shfl_up_sync(0xffffffffu, incl, d);
+    if (lane >= d) incl += v;
+  }
+  const int total = __shfl_sync(0xffffffffu, incl, 31);
+  {
+    uint32_t w = word;
+    int rank = incl - c;
+    while (w) {
+      const int b = __ffs(w) - 1;
+      w &= w - 1u;
+      if (rank % W == warp) sm.cols[warp][rank / W] = k0 + 32 * lane + b;
+      ++rank;
+    }
+  }
+  __syncwarp();
+  const int mine = (total - warp + W - 1) / W;       // ranks warp, warp + W, ...
+
+  // ---- 2. stream the columns of this output tile -------------------------------
+  const int ch = n0 + lane * 16;            // first channel of this lane
+  const bool lane_on = ch < P.N;
+  const int8_t* wcol = P.W + ch;
+  const int64_t ldw = P.ldw;
+  uint32_t ev[4] = {0u, 0u, 0u, 0u}, od[4] = {0u, 0u, 0u, 0u};
+  uint4* stage = &sm.area[warp].stage[0][lane];     // slot b at stage[32 * b]
+  // Rounds of up to L + S columns per warp, all in flight together: the
+  // columns past the register batch are copied into shared memory with
+  // cp.async first, then the register batch is loaded and added, then the
+  // shared-memory columns.
+  for (int i0 = 0; i0 < mine; i0 += L + S) {
+    const int ns = min(S, mine - i0 - L);   // warp-uniform, may be <= 0
+    if (lane_on)
+      for (int b = 0; b < ns; ++b) cp_async16(stage + 32 * b, wcol + sm.cols[warp][i0 + L + b] * ldw);
+    cp_async_commit();
+    uint4 v[L];
+#pragma unroll
+    for (int b = 0; b < L; ++b) {
+      v[b] = make_uint4(0x80808080u, 0x80808080u, 0x80808080u, 0x80808080u);
+      if (lane_on && i0 + b < mine) v[b] = ld_weights16(wcol + sm.cols[warp][i0 + b] * ldw);
+    }
+#pragma unroll
+    for (int b = 0; b < L; ++b) {
+      acc_bytes(v[b].x, ev[0], od[0]);
+      acc_bytes(v[b].y, ev[1], od[1]);
+      acc_bytes(v[b].z, ev[2], od[2]);
+      acc_bytes(v[b].w, ev[3], od[3]);
+    }
+    cp_async_wait_all();                    // this lane's copies have landed
+    for (int b = 0; b < ns; ++b) {
+      const uint4 w = stage[32 * b];
+      acc_bytes(w.x, ev[0], od[0]);
+      acc_bytes(w.y, ev[1], od[1]);
+      acc_bytes(w.z, ev[2], od[2]);
+      acc_bytes(w.w, ev[3], od[3]);
+    }
+  }
+
+  // ---- 3. per-warp partials ------------------------------------------------------
+  // padding loads (0x80 bytes) add 0 to the biased lanes: only the `mine`
+  // real columns carry the +128 bias
+  int o[16];
+  unbias16(ev[0], od[0], mine, o + 0);
+  unbias16(ev[1], od[1], mine, o + 4);
+  unbias16(ev[2], od[2], mine, o + 8);
+  unbias16(ev[3], od[3], mine, o + 12);
+  __syncwarp();                             // every lane is done with the warp's slots
+  int4* dst = reinterpret_cast<int4*>(&sm.area[warp].red[lane * 16]);
+  dst[0] = make_int4(o[0], o[1], o[2], o[3]);
+  dst[1] = make_int4(o[4], o[5], o[6], o[7]);
+  dst[2] = make_int4(o[8], o[9], o[10], o[11]);
+  dst[3] = make_int4(o[12], o[13], o[14], o[15]);
+  __syncthreads();
+}
+
+// Sum of the W warps' partials for tile channels o .. o + 3.
+template <int W, int MAXCK, int S>
+__device__ __forceinline__ int4 unit_sum4(const UnitSmem<W, MAXCK, S>& sm, int o) {
+  int4 s = make_int4(0, 0, 0, 0);
+#pragma unroll
+  for (int w = 0; w < W; ++w) {
+    const int4 r = *reinterpret_cast<const int4*>(&sm.area[w].red[o]);
+    s.x += r.x;
+    s.y += r.y;
+    s.z += r.z;
+    s.w += r.w;
+  }
+  return s;
+}
+
+__device__ __forceinline__ void write4(const GatherProblem& P, int32_t* acc_row, float* y_row,
+                                       int n, int4 v) {
+  if (acc_row) {
+    acc_row[n] = v.x;
+    acc_row[n + 1] = v.y;
+    acc_row[n + 2] = v.z;
+    acc_row[n + 3] = v.w;
+  }
+  if (y_row) {
+    y_row[n] = scale_out(__ldg(P.scale + n), v.x);
+    y_row[n + 1] = scale_out(__ldg(P.scale + n + 1), v.y);
+    y_row[n + 2] = scale_out(__ldg(P.scale + n + 2), v.z);
+    y_row[n + 3] = scale_out(__ldg(P.scale + n + 3), v.w);
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Ticket form: any number of tokens and chunks.  128-thread CTAs, one per
+// (problem, token, 512-channel tile, 512-column chunk) unit.  Grid = (tokens
+// x units of the largest problem, problems); the output tile is the fastest
+// index so that the tiles of one column chunk run side by side.
+constexpr int kTicketWarps = kGatherWarps;         // 4
+constexpr int kTicketLoads = 11;                   // column loads per lane in registers (72 registers)
+constexpr int kTicketSlots = 8;                    // and in shared memory
+using TicketSmem = UnitSmem<kTicketWarps, kGatherCK, kTicketSlots>;
+
 template <int NP>
 __global__ void __launch_bounds__(kGatherThreads, 7)
 gather_kernel(const __grid_constant__ GatherParamsT<NP> p) {
-  __shared__ int s_cols[kWarps][kPerWarp];
-  // Per warp: the landing slots of its shared-memory column loads, reused for
-  // its 512 partial sums once its loads are consumed (each warp touches only
-  // its own region until the barrier before the cross-warp sum).
-  union WarpArea {
-    uint4 stage[kSmemSlots][32];
-    int red[kGatherNT];
-  };
-  __shared__ __align__(16) WarpArea s_area[kWarps];
+  __shared__ TicketSmem sm;
   __shared__ int s_last;
-
-  const int lane = threadIdx.x & 31;
-  const int warp = threadIdx.x >> 5;
   // the next launch may take free SM slots now; this grid's own memory work
   // starts once the previous kernel has finished
   pdl_launch_dependents();
@@ -101,185 +248,223 @@ gather_kernel(const __grid_constant__ GatherParamsT<NP> p) {
   // that start late do not wait behind that burst for their spike words.
   if (blockIdx.y == 0) prefetch_spike_rows(p);
 
-  // grid = (tokens x units of the largest problem, problems): token t, unit x
-  // of problem blockIdx.y; the output tile is the fastest index so that the
-  // tiles of one column chunk run side by side
-  {
-    const int j = blockIdx.y;
-    const int t = (int)(blockIdx.x / (unsigned)p.max_units);
-    const int x = (int)blockIdx.x - t * p.max_units;
-    const GatherProblem& P = p.prob[j];
-    const int kch = gather_kchunks(P.K);
-    const int ntile = gather_ntiles(P.N);
-    if (x >= ntile * kch) return;           // this problem has fewer units
-    const int kc = x / ntile;
-    const int nt = x - kc * ntile;
-    const int n0 = nt * kGatherNT;
-    const int k0 = kc * kGatherCK;
-    const int64_t row = (int64_t)j * p.B + t;
+  const int j = blockIdx.y;
+  const int t = (int)(blockIdx.x / (unsigned)p.max_units);
+  const int x = (int)blockIdx.x - t * p.max_units;
+  const GatherProblem& P = p.prob[j];
+  const int kch = gather_kchunks(P.K);
+  const int ntile = gather_ntiles(P.N);
+  if (x >= ntile * kch) return;             // this problem has fewer units
+  const int kc = x / ntile;
+  const int nt = x - kc * ntile;
+  const int n0 = nt * kGatherNT;
+  const int64_t row = (int64_t)j * p.B + t;
+  unit_partial<kTicketWarps, kGatherCK, kTicketLoads, kTicketSlots>(
+      sm, P, spike_row(p.spikes, p.fmt, row, p.ld_spikes), p.fmt, n0, kc * kGatherCK, kGatherCK);
 
-    // ---- 1. this warp's share of the chunk's active columns -------------------
-    const void* srow = spike_row(p.spikes, p.fmt, row, p.ld_spikes);
-    const uint32_t word = lane < kWords ? spike_word(srow, p.fmt, P.K, k0 + 32 * lane) : 0u;
-    const int c = __popc(word);
-    int incl = c;
-#pragma unroll
-    for (int d = 1; d < 32; d <<= 1) {
-      const int v = __shfl_up_sync(0xffffffffu, incl, d);
-      if (lane >= d) incl += v;
+  int32_t* acc_row = p.acc ? p.acc + row * p.ld_out : nullptr;
+  float* y_row = p.y ? p.y + row * p.ld_out : nullptr;
+  const int o = threadIdx.x * 4;
+  const int n = n0 + o;                     // N % 16 == 0: the 4 channels are all valid or none
+  if (kch == 1) {
+    if (n < P.N) write4(P, acc_row, y_row, n, unit_sum4(sm, o));
+    return;
+  }
+  // Partials go into the workspace as fp32 16-byte vector reductions (one per
+  // thread).  fp32 is exact here: every partial and every sum is an integer
+  // of magnitude <= 128 * K < 2^24, so the result does not depend on the
+  // order of the additions.
+  float* ws = reinterpret_cast<float*>(p.ws) + (int64_t)P.ws_begin * p.B + (int64_t)t * P.N;
+  if (n < P.N) {
+    const int4 v = unit_sum4(sm, o);
+    if (v.x | v.y | v.z | v.w) red_add_v4(ws + n, (float)v.x, (float)v.y, (float)v.z, (float)v.w);
+  }
+  // Release: the barrier orders the CTA's reductions before thread 0, whose
+  // GPU-scope fence makes them visible before its ticket increment.  The
+  // thread that completes the tile fences again (acquire) before the CTA
+  // reads the workspace back.
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    uint32_t* tk = p.tickets + (int64_t)P.ticket_begin * p.B + (int64_t)t * ntile + nt;
+    __threadfence();
+    const uint32_t prev = atomicAdd(tk, 1u);
+    const int last = prev == (uint32_t)(kch - 1);
+    if (last) {
+      atomicExch(tk, 0u);                   // every chunk has arrived: reset
+      __threadfence();
     }
-    const int total = __shfl_sync(0xffffffffu, incl, 31);
-    {
-      uint32_t w = word;
-      int rank = incl - c;
-      while (w) {
-        const int b = __ffs(w) - 1;
-        w &= w - 1u;
-        if ((rank & (kWarps - 1)) == warp) s_cols[warp][rank >> 2] = k0 + 32 * lane + b;
-        ++rank;
-      }
-    }
-    __syncwarp();
-    const int mine = (total - warp + kWarps - 1) / kWarps;   // ranks warp, warp+4, ...
-
-    // ---- 2. stream the columns of this output tile -------------------------------
-    const int ch = n0 + lane * 16;          // first channel of this lane
-    const bool lane_on = ch < P.N;
-    const int8_t* wcol = P.W + ch;
-    const int64_t ldw = P.ldw;
-    uint32_t ev[4] = {0u, 0u, 0u, 0u}, od[4] = {0u, 0u, 0u, 0u};
-    uint4* stage = &s_area[warp].stage[0][lane];     // slot b at stage[32 * b]
-    // Rounds of up to kLoadBatch + kSmemSlots columns per warp, all in flight
-    // together (one round covers a unit at 10% spikes): the columns past the
-    // register batch are copied into shared memory with cp.async first, then
-    // the register batch is loaded and added, then the shared-memory columns.
-    for (int i0 = 0; i0 < mine; i0 += kLoadBatch + kSmemSlots) {
-      const int ns = min(kSmemSlots, mine - i0 - kLoadBatch);   // warp-uniform, may be <= 0
-      if (lane_on)
-        for (int b = 0; b < ns; ++b)
-          cp_async16(stage + 32 * b, wcol + s_cols[warp][i0 + kLoadBatch + b] * ldw);
-      cp_async_commit();
-      uint4 v[kLoadBatch];
-#pragma unroll
-      for (int b = 0; b < kLoadBatch; ++b) {
-        v[b] = make_uint4(0x80808080u, 0x80808080u, 0x80808080u, 0x80808080u);
-        if (lane_on && i0 + b < mine) v[b] = ld_weights16(wcol + s_cols[warp][i0 + b] * ldw);
-      }
-#pragma unroll
-      for (int b = 0; b < kLoadBatch; ++b) {
-        acc_bytes(v[b].x, ev[0], od[0]);
-        acc_bytes(v[b].y, ev[1], od[1]);
-        acc_bytes(v[b].z, ev[2], od[2]);
-        acc_bytes(v[b].w, ev[3], od[3]);
-      }
-      cp_async_wait_all();                  // this lane's copies have landed
-      for (int b = 0; b < ns; ++b) {
-        const uint4 w = stage[32 * b];
-        acc_bytes(w.x, ev[0], od[0]);
-        acc_bytes(w.y, ev[1], od[1]);
-        acc_bytes(w.z, ev[2], od[2]);
-        acc_bytes(w.w, ev[3], od[3]);
-      }
-    }
-    // padding loads (0x80 bytes) add 0 to the biased lanes: only the `mine`
-    // real columns carry the +128 bias
-    const int nacc = mine;
-
-    // ---- 3. reduce the warps -------------------------------------------------
-    {
-      int o[16];
-      unbias16(ev[0], od[0], nacc, o + 0);
-      unbias16(ev[1], od[1], nacc, o + 4);
-      unbias16(ev[2], od[2], nacc, o + 8);
-      unbias16(ev[3], od[3], nacc, o + 12);
-      __syncwarp();                         // every lane is done with the warp's slots
-      int4* dst = reinterpret_cast<int4*>(&s_area[warp].red[lane * 16]);
-      dst[0] = make_int4(o[0], o[1], o[2], o[3]);
-      dst[1] = make_int4(o[4], o[5], o[6], o[7]);
-      dst[2] = make_int4(o[8], o[9], o[10], o[11]);
-      dst[3] = make_int4(o[12], o[13], o[14], o[15]);
-    }
-    __syncthreads();
-
-    int32_t* acc_row = p.acc ? p.acc + row * p.ld_out : nullptr;
-    float* y_row = p.y ? p.y + row * p.ld_out : nullptr;
-    if (kch == 1) {
-      for (int o = threadIdx.x; o < kGatherNT; o += kGatherThreads) {
-        const int n = n0 + o;
-        if (n >= P.N) break;
-        const int v = s_area[0].red[o] + s_area[1].red[o] + s_area[2].red[o] + s_area[3].red[o];
-        if (acc_row) acc_row[n] = v;
-        if (y_row) y_row[n] = scale_out(__ldg(P.scale + n), v);
-      }
-    } else {
-      // Partials go into the workspace as fp32 16-byte vector reductions (one
-      // per thread: channels n0 + 4i .. n0 + 4i + 3).  fp32 is exact here:
-      // every partial and every sum is an integer of magnitude <= 128 * K <
-      // 2^24, so the result does not depend on the order of the additions.
-      float* ws = reinterpret_cast<float*>(p.ws) + (int64_t)P.ws_begin * p.B + (int64_t)t * P.N;
-      const int o = threadIdx.x * 4;
-      const int n = n0 + o;                 // N % 16 == 0: the 4 channels are all valid or none
-      if (n < P.N) {
-        const int4 r0 = *reinterpret_cast<const int4*>(&s_area[0].red[o]);
-        const int4 r1 = *reinterpret_cast<const int4*>(&s_area[1].red[o]);
-        const int4 r2 = *reinterpret_cast<const int4*>(&s_area[2].red[o]);
-        const int4 r3 = *reinterpret_cast<const int4*>(&s_area[3].red[o]);
-        const int v0 = r0.x + r1.x + r2.x + r3.x, v1 = r0.y + r1.y + r2.y + r3.y;
-        const int v2 = r0.z + r1.z + r2.z + r3.z, v3 = r0.w + r1.w + r2.w + r3.w;
-        if (v0 | v1 | v2 | v3) red_add_v4(ws + n, (float)v0, (float)v1, (float)v2, (float)v3);
-      }
-      // Release: the barrier orders the CTA's reductions before thread 0, whose
-      // GPU-scope fence makes them visible before its ticket increment.  The
-      // thread that completes the tile fences again (acquire) before the CTA
-      // reads the workspace back.
-      __syncthreads();
-      if (threadIdx.x == 0) {
-        uint32_t* tk = p.tickets + (int64_t)P.ticket_begin * p.B + (int64_t)t * ntile + nt;
-        __threadfence();
-        const uint32_t prev = atomicAdd(tk, 1u);
-        const int last = prev == (uint32_t)(kch - 1);
-        if (last) {
-          atomicExch(tk, 0u);               // every chunk has arrived: reset
-          __threadfence();
-        }
-        s_last = last;
-      }
-      __syncthreads();
-      if (s_last && n < P.N) {
-        const float4 f = __ldcg(reinterpret_cast<const float4*>(ws + n));
-        __stcg(reinterpret_cast<float4*>(ws + n), make_float4(0.f, 0.f, 0.f, 0.f));
-        const int v[4] = {__float2int_rn(f.x), __float2int_rn(f.y), __float2int_rn(f.z),
-                          __float2int_rn(f.w)};
-#pragma unroll
-        for (int k = 0; k < 4; ++k) {
-          if (acc_row) acc_row[n + k] = v[k];
-          if (y_row) y_row[n + k] = scale_out(__ldg(P.scale + n + k), v[k]);
-        }
-      }
-    }
+    s_last = last;
+  }
+  __syncthreads();
+  if (s_last && n < P.N) {
+    const float4 f = __ldcg(reinterpret_cast<const float4*>(ws + n));
+    __stcg(reinterpret_cast<float4*>(ws + n), make_float4(0.f, 0.f, 0.f, 0.f));
+    write4(P, acc_row, y_row, n,
+           make_int4(__float2int_rn(f.x), __float2int_rn(f.y), __float2int_rn(f.z),
+                     __float2int_rn(f.w)));
   }
 }
 
-// Asks for the largest shared-memory carveout once per device, so that 7
-// CTAs (7 x 18 KB of shared memory) fit on an SM beside their L1.
+// ---------------------------------------------------------------------------
+// Cluster form: one token per problem, at most kGatherCluster chunks of at
+// most 1024 columns per tile.  256-thread CTAs in clusters of kGatherCluster;
+// a cluster holds tpc tiles x kch chunks of one problem (rank = tile slot *
+// kch + chunk; kch divides kGatherCluster); grid = (clusters of the largest
+// problem x kGatherCluster, problems).  The 4-channel group g of a tile
+// belongs to the CTA of chunk g % kch: every CTA stores its partial of each
+// group into the owner's shared memory (distributed shared memory), one
+// cluster barrier (release / acquire) publishes the stores, and each owner
+// adds the kch partials of its groups from its own shared memory and writes
+// acc / y.  No workspace, no atomics, and no CTA reads another's shared
+// memory, so none waits for the others after the barrier.
+constexpr int kClusterLoads = 9;                   // column loads per lane in registers (64 registers)
+constexpr int kClusterSlots = 8;                   // and in shared memory
+using ClusterSmem = UnitSmem<kGatherClusterWarps, kGatherClusterMaxCK, kClusterSlots>;
+
 template <int NP>
-cudaError_t set_carveout() {
-  static std::atomic<uint64_t> done{0};
+__global__ void __launch_bounds__(kGatherClusterThreads, 4)
+gather_cluster_kernel(const __grid_constant__ GatherParamsT<NP> p) {
+  __shared__ ClusterSmem sm;
+  // [sender chunk][owned group]: kch * ceil(128 / kch) < 128 + kch entries
+  __shared__ __align__(16) int4 s_recv[kGatherNT / 4 + kGatherCluster];
+  pdl_launch_dependents();
+  pdl_wait();
+  if (blockIdx.y == 0) prefetch_spike_rows(p);
+
+  const int j = blockIdx.y;
+  const GatherProblem& P = p.prob[j];
+  const int cl = (int)blockIdx.x / kGatherCluster;
+  const int rank = (int)blockIdx.x - cl * kGatherCluster;  // rank in the (6, 1, 1) cluster
+  if (cl >= P.ncl) return;                  // the whole cluster: no tile of this problem
+  const int kch = P.kch;
+  const int per = (kGatherNT / 4 + kch - 1) / kch;   // most groups owned by one CTA
+  const int ts = rank / kch;
+  const int kc = rank - ts * kch;
+  const int n0 = (cl * P.tpc + ts) * kGatherNT;
+  const bool work = n0 < P.N;               // tile slots past the last tile idle
+  if (work) {
+    unit_partial<kGatherClusterWarps, kGatherClusterMaxCK, kClusterLoads, kClusterSlots>(
+        sm, P, spike_row(p.spikes, p.fmt, j, p.ld_spikes), p.fmt, n0, kc * P.ck, P.ck);
+    const int g = threadIdx.x;              // the 4-channel group of this thread
+    if (g < kGatherNT / 4) {
+      const int4 v = unit_sum4(sm, 4 * g);
+      st_peer_v4((uint32_t)__cvta_generic_to_shared(&s_recv[kc * per + g / kch]),
+                 (uint32_t)(ts * kch + g % kch), v);
+    }
+  }
+  cluster_sync_all();                       // every partial is in its owner's shared memory
+  const int g_own = threadIdx.x * kch + kc; // this thread's owned group
+  const int n = n0 + 4 * g_own;
+  if (work && g_own < kGatherNT / 4 && n < P.N) {
+    int4 s = make_int4(0, 0, 0, 0);
+    for (int q = 0; q < kch; ++q) {
+      const int4 v = s_recv[q * per + threadIdx.x];
+      s.x += v.x;
+      s.y += v.y;
+      s.z += v.z;
+      s.w += v.w;
+    }
+    write4(P, p.acc ? p.acc + (int64_t)j * p.ld_out : nullptr,
+           p.y ? p.y + (int64_t)j * p.ld_out : nullptr, n, s);
+  }
+}
+
+// Asks for the largest shared-memory carveout once per device and kernel, so
+// that every resident CTA's shared memory fits beside L1.
+template <typename Kern>
+cudaError_t set_carveout(Kern kernel, std::atomic<uint64_t>& done) {
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
   const uint64_t bit = dev < 64 ? (uint64_t)1 << dev : 0;
   if (bit && (done.load(std::memory_order_relaxed) & bit)) return cudaSuccess;
-  e = cudaFuncSetAttribute(gather_kernel<NP>, cudaFuncAttributePreferredSharedMemoryCarveout,
+  e = cudaFuncSetAttribute(kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
                            (int)cudaSharedmemCarveoutMaxShared);
   if (e == cudaSuccess && bit) done.fetch_or(bit, std::memory_order_relaxed);
   return e;
 }
 
+// Clusters of the cluster form that can be resident at once (per device).
+template <int NP>
+int cluster_capacity() {
+  static std::atomic<int> cap[64];
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev >= 64) return 0;
+  int n = cap[dev].load(std::memory_order_relaxed);
+  if (n != 0) return n;
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr;
+  attr.id = cudaLaunchAttributeClusterDimension;
+  attr.val.clusterDim.x = kGatherCluster;
+  attr.val.clusterDim.y = 1;
+  attr.val.clusterDim.z = 1;
+  cfg.gridDim = dim3(kGatherCluster, 1, 1);
+  cfg.blockDim = dim3(kGatherClusterThreads, 1, 1);
+  cfg.attrs = &attr;
+  cfg.numAttrs = 1;
+  if (cudaOccupancyMaxActiveClusters(&n, gather_cluster_kernel<NP>, &cfg) != cudaSuccess || n < 1) {
+    (void)cudaGetLastError();
+    n = -1;
+  }
+  cap[dev].store(n, std::memory_order_relaxed);
+  return n;
+}
+
+// Fills the cluster-form fields of q; false when the launch does not fit the
+// cluster form (several tokens, a chunk count above the cluster size, or more
+// clusters than can be resident at once).
+template <int NP>
+bool cluster_form(GatherParamsT<NP>& q, int* grid_x) {
+  if (q.B != 1) return false;
+  int total = 0, widest = 0;
+  for (int j = 0; j < q.nprob; ++j) {
+    GatherProblem& P = q.prob[j];
+    // the fewest chunks (a divisor of the cluster size) of at most 1024 columns
+    int kch = 0;
+    for (int d = 1; d <= kGatherCluster; ++d)
+      if (kGatherCluster % d == 0 && ceil_div(P.K, d) <= kGatherClusterMaxCK) {
+        kch = d;
+        break;
+      }
+    if (kch == 0) return false;
+    P.kch = kch;
+    P.ck = ceil_div(ceil_div(P.K, kch), 32) * 32;
+    P.tpc = kGatherCluster / kch;
+    P.ncl = ceil_div(gather_ntiles(P.N), P.tpc);
+    total += P.ncl;
+    if (P.ncl > widest) widest = P.ncl;
+  }
+  if (total > cluster_capacity<NP>()) return false;
+  *grid_x = widest * kGatherCluster;
+  return true;
+}
+
 template <int NP>
 cudaError_t launch_gather_t(const GatherParamsT<NP>& p, cudaStream_t s) {
+  static std::atomic<uint64_t> carve_t{0}, carve_c{0};
   if (p.units_total <= 0 || p.B <= 0 || p.max_units <= 0) return cudaSuccess;
-  const cudaError_t e = set_carveout<NP>();
+  // the carveout first: the resident-cluster count depends on it
+  cudaError_t e = set_carveout(gather_cluster_kernel<NP>, carve_c);
+  if (e != cudaSuccess) return e;
+  GatherParamsT<NP> q = p;
+  int gx = 0;
+  if (cluster_form(q, &gx)) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)gx, (unsigned)q.nprob, 1);
+    cfg.blockDim = dim3(kGatherClusterThreads, 1, 1);
+    cfg.stream = s;
+    cudaLaunchAttribute attr[2];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = kGatherCluster;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[1].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 2;
+    return cudaLaunchKernelEx(&cfg, gather_cluster_kernel<NP>, q);
+  }
+  e = set_carveout(gather_kernel<NP>, carve_t);
   if (e != cudaSuccess) return e;
   if ((int64_t)p.max_units * p.B > 0x7fffffffll) return cudaErrorInvalidConfiguration;
   // one CTA per unit; the hardware keeps every unit of a decode step resident

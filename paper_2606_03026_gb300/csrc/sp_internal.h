@@ -45,7 +45,17 @@ struct GatherProblem {
   int32_t unit_begin;     // prefix sum of units_per_token over problems
   int32_t ws_begin;       // prefix sum of N (int32 elements of workspace)
   int32_t ticket_begin;   // prefix sum of output tiles
+  // cluster form (set by the launcher): a cluster of kGatherCluster CTAs
+  // holds tpc output tiles x kch column chunks of ck columns; ncl clusters
+  int32_t ck, kch, tpc, ncl;
 };
+
+// Cluster form of the gather (one token per problem): clusters of 6 CTAs of
+// 256 threads; a CTA sums chunks of at most 1024 columns.
+constexpr int kGatherCluster = 6;
+constexpr int kGatherClusterWarps = 8;
+constexpr int kGatherClusterThreads = 32 * kGatherClusterWarps;
+constexpr int kGatherClusterMaxCK = 1024;
 
 constexpr int kMaxProblems = SPIKE_PROJ_MAX_GROUP;
 
