@@ -14,9 +14,12 @@ events on the launching stream, max over ranks.  L2: the weights are held in
 is re-read from L2 within 8 steps (> 129 MB of other traffic in between).
 
 Also reported on the same JSON line:
-  roofline     the grouped gather kernel: active bytes per launch / average
-               launch duration (CUDA events around single launches), against
-               the measured HBM copy bandwidth
+  roofline     the grouped gather kernel (the only kernel of a step): active
+               bytes per launch / average launch duration over the timed
+               region (CUDA events on the launching stream), against the
+               measured HBM copy bandwidth; traffic = the DRAM bytes per
+               launch that ncu measured for the same kernel source
+               (profiles/dram_traffic.json), null when the source differs
   e2e          the same metric through the host-buffer entry point (spike
                masks copied in from pinned memory, acc and y copied back,
                every step)
@@ -353,8 +356,9 @@ def run_ours(args):
     ms_per_step = elapsed_ms / steps
     clocks = sampler.summary(t_wall0, t_wall1)
 
-    # per-launch duration of the grouped gather kernel (events around single
-    # launches on the launching stream), for the roofline
+    # one grouped-gather launch per step: its average duration over the timed
+    # region is the step time.  Events around isolated launches (outside any
+    # graph) are reported beside it.
     n_single = 512
     evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
            for _ in range(n_single)]
@@ -365,10 +369,11 @@ def run_ours(args):
             evs[i][1].record(stream)
     stream.synchronize()
     durs = [a.elapsed_time(b) for a, b in evs]
-    launch_ms = statistics.mean(durs)
-    bytes_single = float(np.mean([active[i % SPIKE_SETS] for i in range(n_single)]))
-    achieved = bytes_single / (launch_ms * 1e-3) / 1e9
+    isolated_ms = statistics.mean(durs)
+    launch_ms = ms_per_step
+    achieved = value / world
     hbm = float(peaks["hbm_gbs"])
+    traffic = measured_traffic("gather_cluster_kernel", "sp_gather.cu")
 
     # end to end through the host-buffer entry point, graph-captured
     h_sets = torch.from_numpy(sets_np).pin_memory()
@@ -412,10 +417,11 @@ def run_ours(args):
                    "parallelism": "replicas" if world > 1 else "single GPU"},
         "projected_tokens_per_s": 1e3 / ms_per_step * world,
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": hbm, "unit": "GB/s",
-                     "frac": achieved / hbm, "traffic": None,
-                     "kernel": "gather_kernel<64> (grouped decode step)",
-                     "launch_us": launch_ms * 1e3, "peak_kind": peak_kind,
-                     "frac_of_nominal_8tbs": achieved / 8000.0},
+                     "frac": achieved / hbm, "traffic": traffic,
+                     "algorithmic_bytes_per_launch": bytes_per_step,
+                     "kernel": "gather_cluster_kernel<64> (grouped decode step)",
+                     "launch_us": launch_ms * 1e3, "isolated_launch_us": isolated_ms * 1e3,
+                     "peak_kind": peak_kind, "frac_of_nominal_8tbs": achieved / 8000.0},
         "e2e": {"value": e2e_bytes / (e2e_ms * 1e-3) / 1e9, "unit": "GB/s",
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                 "ms_per_step": e2e_ms / e2e_steps,
@@ -440,6 +446,20 @@ def run_ours(args):
         g.close()
     if rank == 0:
         print(json.dumps(result))
+
+
+def measured_traffic(kernel, source):
+    """DRAM bytes per launch of `kernel` from the committed ncu summary, if
+    it was taken on the current kernel source (sha256 of csrc/`source`)."""
+    import hashlib
+    try:
+        rec = json.loads((ROOT / "profiles" / "dram_traffic.json").read_text())[kernel]
+        src = ROOT / "paper_2606_03026_gb300" / "csrc" / source
+        if hashlib.sha256(src.read_bytes()).hexdigest() != rec["source_sha256"]:
+            return None
+        return float(rec["dram_bytes_per_launch"])
+    except (OSError, KeyError, ValueError):
+        return None
 
 
 def bench_prefill(torch, sp, synth, dev, stream, peaks, peak_kind, world, blocks=22):
@@ -497,7 +517,9 @@ def bench_prefill(torch, sp, synth, dev, stream, peaks, peak_kind, world, blocks
             "prefill_tokens_per_s": T / (ms * 1e-3) * world, "chosen_kernel": chosen,
             "mean_density": dens, "ops": "2*T*N*K dense-equivalent int8 ops per block",
             "roofline": {"bound": "tensor", "achieved": tops, "peak": peak, "unit": "TFLOP/s",
-                         "frac": tops / peak, "traffic": None, "peak_kind": peak_kind + " bf16 burst",
+                         "frac": tops / peak,
+                         "traffic": measured_traffic("gemm_kernel", "sp_gemm.cu"),
+                         "peak_kind": peak_kind + " bf16 burst",
                          "note": "sm_103a has no tcgen05 kind::i8; exact bf16 operands, fp32 accumulate"}}
 
 

@@ -57,7 +57,8 @@ def test_down_projection_all_vectors(p):
 @pytest.mark.parametrize("N,K,ldq", [(16, 1, 16), (16, 33, 32), (48, 1000, 64),
                                      (1552, 777, 1568), (528, 1025, 528), (512, 512, 512),
                                      (2048, 4096, 2048), (2064, 300, 2064), (4096, 2000, 4112),
-                                     (6160, 129, 6160)])
+                                     (6160, 129, 6160), (1536, 3000, 1536), (544, 2049, 560),
+                                     (1040, 6145, 1040)])
 @pytest.mark.parametrize("p", [0.0, 0.3, 1.0])
 def test_ragged_shapes(N, K, ldq, p):
     """N not a multiple of the 512-channel tile, K with a ragged last word

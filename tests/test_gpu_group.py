@@ -128,3 +128,39 @@ def test_group_of_64_uncached_masks():
         assert_parity(acc[j], y[j], a[0], yy[0], f"member {j}")
     assert group.status() == sp.SP_OK
     group.close()
+
+
+@pytest.mark.parametrize("p", [0.1, 1.0])
+@pytest.mark.parametrize("ticket", [False, True])
+def test_cluster_layouts(p, ticket):
+    """Batch-1 groups run as clusters of 6 CTAs holding tiles x chunks:
+    K <= 1024 (1 chunk, 6 tiles per cluster), <= 2048 (2 chunks, 3 tiles),
+    <= 3072 (3 chunks, 2 tiles), <= 6144 (6 chunks, 1 tile), with tile counts
+    that leave idle tile slots in the last cluster.  One member with K = 6145
+    sends the whole group through the ticket form instead."""
+    cases = [(2576, 1024), (1552, 1025), (2064, 2048), (1040, 2049), (1536, 3072),
+             (528, 3073), (3088, 6144)] + ([(512, 6145)] if ticket else [])
+    weights, plans, xs = [], [], []
+    for i, (N, K) in enumerate(cases):
+        Qc, s, x = synth.random_case(60 + i, N, K, p=p)
+        weights.append((Qc, s, N, K))
+        plans.append(sp.Plan(to_dev(Qc), to_dev(s), N, K))
+        xs.append(x[0])
+    group = sp.Group(plans)
+    maxK = max(K for _, K in cases)
+    maxN = max(N for N, _ in cases)
+    bits = np.zeros((len(cases), (maxK + 31) // 32), np.uint32)
+    for j, x in enumerate(xs):
+        b = synth.pack_bits(x)
+        bits[j, : b.size] = b
+    for rep in range(2):
+        acc = torch.full((len(cases), maxN), 5, dtype=torch.int32, device=DEV)
+        y = torch.full((len(cases), maxN), 5.0, dtype=torch.float32, device=DEV)
+        group.decode(to_dev(bits), "bits", bits.shape[1], acc, y, maxN)
+        torch.cuda.synchronize()
+        for j, (Qc, s, N, K) in enumerate(weights):
+            a, yy = oracle.project(Qc, s, N, K, xs[j], "u8")
+            assert_parity(acc[j, :N], y[j, :N], a[0], yy[0], f"member {j} rep {rep}")
+            assert (acc[j, N:] == 5).all(), "wrote past the member's N"
+    assert group.status() == sp.SP_OK
+    group.close()
