@@ -41,6 +41,10 @@ struct sp_plan_s {
   float* part = nullptr;          // split-K partials, part_units x 128 x 256 fp32
   int Kp = 0, xb_rows = 0, part_units = 0;
   GemmMaps maps;
+  CUtensorMap x8map;              // u8 spike rows of the last fused call
+  const void* x8_ptr = nullptr;
+  int64_t x8_ld = 0;
+  int32_t x8_T = 0;
   sp_kernel last_kernel = SP_AUTO;
   int32_t last_active = -1;
 };
@@ -199,7 +203,19 @@ sp_status run_union(sp_plan_s* p, const void* spikes, int fmt, int B, int64_t ld
 sp_status run_gemm(sp_plan_s* p, const void* spikes, int fmt, int T, int64_t ld, int32_t* acc,
                    float* y, cudaStream_t s) {
   if (!(p->flags & SP_PLAN_GEMM)) return SP_EUNSUPPORTED;
-  SP_CUDA(launch_spikes_to_bf16(spikes, fmt, ld, T, p->K, p->Kp, p->Xb, s));
+  // u8 rows that TMA can read directly are converted inside the GEMM kernel;
+  // anything else goes through the bf16 staging copy first
+  const bool fused = fmt == SP_SPIKES_U8 && aligned(spikes, 16) && ld % 16 == 0;
+  if (fused) {
+    if (spikes != p->x8_ptr || ld != p->x8_ld || T != p->x8_T) {
+      SP_CUDA(gemm_make_x8_map(spikes, ld, T, p->K, &p->x8map));
+      p->x8_ptr = spikes;
+      p->x8_ld = ld;
+      p->x8_T = T;
+    }
+  } else {
+    SP_CUDA(launch_spikes_to_bf16(spikes, fmt, ld, T, p->K, p->Kp, p->Xb, s));
+  }
   GemmParams g;
   g.scale = p->scale;
   g.acc = acc;
@@ -210,7 +226,7 @@ sp_status run_gemm(sp_plan_s* p, const void* spikes, int fmt, int T, int64_t ld,
   g.err = p->err;
   g.part = p->part;
   g.part_units = p->part_units;
-  SP_CUDA(launch_gemm(p->maps, T, p->N, p->Kp, g, s));
+  SP_CUDA(launch_gemm(fused ? p->x8map : p->maps.a, p->maps.b, fused, T, p->N, p->Kp, g, s));
   return SP_OK;
 }
 

@@ -49,7 +49,11 @@ constexpr int A_BYTES = BM * BK * 2;          // 16 KB
 constexpr int B_BYTES = BN * BK * 2;          // 32 KB
 constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
 constexpr int TMEM_COLS = 2 * BN;             // double-buffered accumulator
-constexpr int kGemmThreads = 192;
+constexpr int kGemmThreads = 192;             // TMA, MMA and 4 epilogue warps
+constexpr int kConvThreads = 256;             // 8 warps converting u8 spikes to bf16
+constexpr int kGemmThreadsFused = kGemmThreads + kConvThreads;
+constexpr int X8_BYTES = BM * BK;             // one u8 spike tile (8 KB)
+constexpr int X8_OFFSET = A_BYTES - X8_BYTES; // lands in the upper half of the A slot
 constexpr int TR_STRIDE = 33;                 // padded transpose rows (words)
 constexpr size_t SMEM_RING = (size_t)STAGES * STAGE_BYTES;
 constexpr size_t SMEM_TR = (size_t)4 * 32 * TR_STRIDE * 4;
@@ -152,7 +156,54 @@ __device__ __forceinline__ void store_chunk(const GemmParams& p, uint32_t* tr,
   __syncwarp();
 }
 
-__global__ void __launch_bounds__(kGemmThreads, 1)
+// True on all converter threads if `v` is true on any of them (named barrier
+// 1 with a predicate reduction): the converter warps take every abort
+// decision together, so none can be left waiting at barrier 1.
+__device__ __forceinline__ bool converters_any(bool v) {
+  uint32_t r;
+  asm volatile(
+      "{\n\t.reg .pred p, q;\n\tsetp.ne.u32 p, %1, 0;\n\t"
+      "bar.red.or.pred q, 1, %2, p;\n\tselp.u32 %0, 1, 0, q;\n\t}"
+      : "=r"(r)
+      : "r"((uint32_t)v), "n"(kConvThreads)
+      : "memory");
+  return r != 0;
+}
+
+// 128 u8 spike rows x 64 columns (TMA-loaded at X8_OFFSET of the A slot) ->
+// the slot's bf16 0/1 tile in the 128-byte-swizzle layout the MMA descriptor
+// expects (16-byte chunk j of row r at r * 128 + (j ^ (r % 8)) * 16).
+// Thread t (0..255) converts half h = t % 2 of row r = t / 2 (columns 32h ..
+// 32h + 31).  Every thread reads before any writes (named barrier 1), since
+// the bf16 rows 64..127 cover the u8 tile.
+__device__ __forceinline__ void convert_x8_tile(uint8_t* slot, int t) {
+  const int r = t >> 1, h = t & 1;
+  const uint4* src = reinterpret_cast<const uint4*>(slot + X8_OFFSET + r * BK + h * 32);
+  const uint4 u0 = src[0], u1 = src[1];
+  asm volatile("bar.sync 1, %0;" ::"n"(kConvThreads) : "memory");
+  const uint32_t w[8] = {u0.x, u0.y, u0.z, u0.w, u1.x, u1.y, u1.z, u1.w};
+  uint8_t* row = slot + r * 128;
+#pragma unroll
+  for (int jj = 0; jj < 4; ++jj) {            // chunk j = 4h + jj: columns 8j .. 8j + 7
+    uint32_t o[4];
+#pragma unroll
+    for (int e = 0; e < 2; ++e) {
+      const uint32_t v = w[2 * jj + e];
+      // 0x80 in every nonzero byte (the low byte of bf16 1.0 = 0x3f80), 0 elsewhere
+      const uint32_t lo = (((v & 0x7f7f7f7fu) + 0x7f7f7f7fu) | v) & 0x80808080u;
+      const uint32_t hi = (lo >> 7) * 0x3fu;
+      o[2 * e] = __byte_perm(lo, hi, 0x5140);
+      o[2 * e + 1] = __byte_perm(lo, hi, 0x7362);
+    }
+    const int j = 4 * h + jj;
+    *reinterpret_cast<uint4*>(row + ((j ^ (r & 7)) << 4)) = make_uint4(o[0], o[1], o[2], o[3]);
+  }
+}
+
+// kFusedX: operand A is u8 spikes (converted in shared memory by warps 6-13)
+// instead of the bf16 staging copy.
+template <bool kFusedX>
+__global__ void __launch_bounds__(kFusedX ? kGemmThreadsFused : kGemmThreads, 1)
 gemm_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB,
             const __grid_constant__ GemmArgs a) {
   extern __shared__ uint8_t smem_raw[];
@@ -168,7 +219,8 @@ gemm_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CU
   uint64_t* tempty = tfull + 2;          // [2] epilogue -> MMA
   uint64_t* done = tempty + 2;           // all MMAs retired
   uint64_t* pfull = done + 1;            // split K: peers' partials landed
-  uint32_t* s_tmem = reinterpret_cast<uint32_t*>(pfull + 1);
+  uint64_t* conv = pfull + 1;            // [STAGES] converted A tile ready (fused)
+  uint32_t* s_tmem = reinterpret_cast<uint32_t*>(conv + STAGES);
   volatile int* s_abort = reinterpret_cast<volatile int*>(s_tmem + 1);
 
   const int warp = threadIdx.x >> 5;
@@ -185,6 +237,7 @@ gemm_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CU
     }
     mbar_init(done, 1);
     mbar_init(pfull, 1);
+    for (int s = 0; s < STAGES; ++s) mbar_init(&conv[s], kConvThreads / 32);  // per converter warp
     *s_abort = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     tma_prefetch_desc(&mapA);
@@ -211,8 +264,14 @@ gemm_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CU
             atomicExch(a.p.err, kErrMbarTimeout);
             break;
           }
-          mbar_arrive_expect_tx(&full[stage], STAGE_BYTES);
-          tma_load_2d(sA + (size_t)stage * A_BYTES, &mapA, &full[stage], kb * BK, mb * BM);
+          if (kFusedX) {
+            mbar_arrive_expect_tx(&full[stage], X8_BYTES + B_BYTES);
+            tma_load_2d(sA + (size_t)stage * A_BYTES + X8_OFFSET, &mapA, &full[stage], kb * BK,
+                        mb * BM);
+          } else {
+            mbar_arrive_expect_tx(&full[stage], STAGE_BYTES);
+            tma_load_2d(sA + (size_t)stage * A_BYTES, &mapA, &full[stage], kb * BK, mb * BM);
+          }
           tma_load_2d(sB + (size_t)stage * B_BYTES, &mapB, &full[stage], kb * BK, nb * BN);
           ++issued;
           if (++stage == STAGES) { stage = 0; ph ^= 1u; }
@@ -246,7 +305,7 @@ gemm_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CU
         const uint32_t d = tmem_base + (uint32_t)(ab * BN);
         bool ok = true;
         for (int kb = kb0; kb < kb1; ++kb) {
-          if (!mbar_wait(&full[stage], ph)) {
+          if (!mbar_wait(kFusedX ? &conv[stage] : &full[stage], ph)) {
             ok = false;
             break;
           }
@@ -269,6 +328,33 @@ gemm_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CU
       }
       mma_commit(done);                      // retire every issued MMA
       mbar_wait(done, 0);
+    }
+  } else if (kFusedX && warp >= 6) {
+    // ------------------------- spike converters (fused) -----------------------
+    // Same (unit, K block) sequence as the producer: wait for the u8 tile,
+    // expand it in place, make the writes visible to the tensor core (async
+    // proxy) and release the slot to the MMA warp.
+    const int ct = threadIdx.x - kGemmThreads;   // 0 .. kConvThreads - 1
+    int stage = 0;
+    uint32_t ph = 0;
+    bool ok = true;
+    for (int u = blockIdx.x; u < a.units && ok; u += gridDim.x) {
+      int tile, mb, nb, kb0, kb1;
+      unit_coords(a, u, tile, mb, nb, kb0, kb1);
+      for (int kb = kb0; kb < kb1; ++kb) {
+        const bool bad = *s_abort || !mbar_wait(&full[stage], ph);
+        if (converters_any(bad)) {
+          *s_abort = 1;
+          if (ct == 0) atomicExch(a.p.err, kErrMbarTimeout);
+          ok = false;
+          break;
+        }
+        convert_x8_tile(sA + (size_t)stage * A_BYTES, ct);
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&conv[stage]);
+        if (++stage == STAGES) { stage = 0; ph ^= 1u; }
+      }
     }
   } else if (a.splits == 1) {
     // ------------------------------ epilogue (whole K) ------------------------
@@ -317,7 +403,7 @@ gemm_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CU
     // of its quarter) per store, and each (r, c) partial is 16 KB contiguous.
     const int S = a.splits;
     const int rank = (int)cluster_ctarank();
-    const bool epi = warp >= 2;
+    const bool epi = warp >= 2 && warp < 6;
     const int q = warp & 3;
     int tile, mb, nb, kb0, kb1;
     unit_coords(a, blockIdx.x, tile, mb, nb, kb0, kb1);
@@ -484,6 +570,109 @@ bool encode_2d(CUtensorMap* map, const void* base, uint64_t inner, uint64_t oute
              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+template <bool kFusedX>
+constexpr int gemm_threads() {
+  return kFusedX ? kGemmThreadsFused : kGemmThreads;
+}
+
+// Largest number of clusters of `size` CTAs that can be resident at once.
+template <bool kFusedX>
+int max_active_clusters(int size) {
+  static int cache[9] = {0};
+  if (cache[size] == 0) {
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute attr;
+    attr.id = cudaLaunchAttributeClusterDimension;
+    attr.val.clusterDim.x = size;
+    attr.val.clusterDim.y = 1;
+    attr.val.clusterDim.z = 1;
+    cfg.gridDim = dim3(size, 1, 1);
+    cfg.blockDim = dim3(gemm_threads<kFusedX>(), 1, 1);
+    cfg.dynamicSmemBytes = kGemmSmem;
+    cfg.attrs = &attr;
+    cfg.numAttrs = 1;
+    int n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, gemm_kernel<kFusedX>, &cfg) != cudaSuccess || n < 1) {
+      (void)cudaGetLastError();
+      n = -1;
+    }
+    cache[size] = n;
+  }
+  return cache[size];
+}
+
+template <bool kFusedX>
+cudaError_t set_gemm_attrs() {
+  static bool done = false;
+  if (done) return cudaSuccess;
+  cudaError_t e = cudaFuncSetAttribute(gemm_kernel<kFusedX>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kGemmSmem);
+  if (e != cudaSuccess) return e;
+  e = cudaFuncSetAttribute(gemm_kernel<kFusedX>, cudaFuncAttributeNonPortableClusterSizeAllowed, 0);
+  if (e != cudaSuccess) return e;
+  done = true;
+  return cudaSuccess;
+}
+
+template <bool kFusedX>
+cudaError_t launch_gemm_t(const CUtensorMap& mapA, const CUtensorMap& mapB, int T, int N, int Kp,
+                          const GemmParams& p, cudaStream_t s) {
+  if (!g_attr_set) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    e = cudaDeviceGetAttribute(&g_num_sms, cudaDevAttrMultiProcessorCount, dev);
+    if (e != cudaSuccess) return e;
+    g_attr_set = true;
+  }
+  cudaError_t e = set_gemm_attrs<kFusedX>();
+  if (e != cudaSuccess) return e;
+  GemmArgs a;
+  a.p = p;
+  a.tiles_m = ceil_div(T, BM);
+  a.tiles_n = ceil_div(N, BN);
+  a.nkb = Kp / BK;
+  const int tiles = a.tiles_m * a.tiles_n;
+  // Split K over a cluster only when the tiles alone leave SMs idle, and only
+  // as far as every cluster stays resident in a single wave.
+  int S = 1;
+  if (tiles < g_num_sms) {
+    S = g_num_sms / tiles;
+    if (S > 8) S = 8;
+    if (S > a.nkb / 4) S = a.nkb / 4;
+    if (S < 1) S = 1;
+    while (S > 1) {
+      const int kbps = ceil_div(a.nkb, S);
+      const int exact = ceil_div(a.nkb, kbps);          // splits with work
+      if (exact == S && max_active_clusters<kFusedX>(S) >= tiles && tiles * S <= p.part_units)
+        break;
+      --S;
+    }
+  }
+  a.kb_per_split = ceil_div(a.nkb, S);
+  a.splits = S;
+  a.units = tiles * S;
+  const int threads = gemm_threads<kFusedX>();
+  if (S == 1) {
+    const int grid = a.units < g_num_sms ? a.units : g_num_sms;
+    gemm_kernel<kFusedX><<<grid, threads, kGemmSmem, s>>>(mapA, mapB, a);
+    return cudaGetLastError();
+  }
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr;
+  attr.id = cudaLaunchAttributeClusterDimension;
+  attr.val.clusterDim.x = S;
+  attr.val.clusterDim.y = 1;
+  attr.val.clusterDim.z = 1;
+  cfg.gridDim = dim3(a.units, 1, 1);
+  cfg.blockDim = dim3(threads, 1, 1);
+  cfg.dynamicSmemBytes = kGemmSmem;
+  cfg.stream = s;
+  cfg.attrs = &attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, gemm_kernel<kFusedX>, mapA, mapB, a);
+}
+
 }  // namespace
 
 int gemm_k_pad(int K) { return ceil_div(K, BK) * BK; }
@@ -519,88 +708,23 @@ cudaError_t launch_spikes_to_bf16(const void* spikes, int fmt, int64_t ld, int T
   return cudaGetLastError();
 }
 
-// Largest number of clusters of `size` CTAs that can be resident at once.
-int max_active_clusters(int size) {
-  static int cache[9] = {0};
-  if (cache[size] == 0) {
-    cudaLaunchConfig_t cfg = {};
-    cudaLaunchAttribute attr;
-    attr.id = cudaLaunchAttributeClusterDimension;
-    attr.val.clusterDim.x = size;
-    attr.val.clusterDim.y = 1;
-    attr.val.clusterDim.z = 1;
-    cfg.gridDim = dim3(size, 1, 1);
-    cfg.blockDim = dim3(kGemmThreads, 1, 1);
-    cfg.dynamicSmemBytes = kGemmSmem;
-    cfg.attrs = &attr;
-    cfg.numAttrs = 1;
-    int n = 0;
-    if (cudaOccupancyMaxActiveClusters(&n, gemm_kernel, &cfg) != cudaSuccess || n < 1) {
-      (void)cudaGetLastError();
-      n = -1;
-    }
-    cache[size] = n;
-  }
-  return cache[size];
+cudaError_t gemm_make_x8_map(const void* X, int64_t ldx, int T, int K, CUtensorMap* out) {
+  auto enc = get_encode();
+  if (!enc) return cudaErrorUnknown;
+  const cuuint64_t dims[2] = {(cuuint64_t)K, (cuuint64_t)T};
+  const cuuint64_t strides[1] = {(cuuint64_t)ldx};
+  const cuuint32_t box[2] = {BK, BM};
+  const cuuint32_t estr[2] = {1, 1};
+  const CUresult r = enc(out, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<void*>(X), dims, strides,
+                         box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+                         CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
 }
 
-cudaError_t launch_gemm(const GemmMaps& maps, int T, int N, int Kp, const GemmParams& p,
-                        cudaStream_t s) {
-  if (!g_attr_set) {
-    int dev = 0;
-    cudaError_t e = cudaGetDevice(&dev);
-    if (e != cudaSuccess) return e;
-    e = cudaDeviceGetAttribute(&g_num_sms, cudaDevAttrMultiProcessorCount, dev);
-    if (e != cudaSuccess) return e;
-    e = cudaFuncSetAttribute(gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             (int)kGemmSmem);
-    if (e != cudaSuccess) return e;
-    e = cudaFuncSetAttribute(gemm_kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 0);
-    if (e != cudaSuccess) return e;
-    g_attr_set = true;
-  }
-  GemmArgs a;
-  a.p = p;
-  a.tiles_m = ceil_div(T, BM);
-  a.tiles_n = ceil_div(N, BN);
-  a.nkb = Kp / BK;
-  const int tiles = a.tiles_m * a.tiles_n;
-  // Split K over a cluster only when the tiles alone leave SMs idle, and only
-  // as far as every cluster stays resident in a single wave.
-  int S = 1;
-  if (tiles < g_num_sms) {
-    S = g_num_sms / tiles;
-    if (S > 8) S = 8;
-    if (S > a.nkb / 4) S = a.nkb / 4;
-    if (S < 1) S = 1;
-    while (S > 1) {
-      const int kbps = ceil_div(a.nkb, S);
-      const int exact = ceil_div(a.nkb, kbps);          // splits with work
-      if (exact == S && max_active_clusters(S) >= tiles && tiles * S <= p.part_units) break;
-      --S;
-    }
-  }
-  a.kb_per_split = ceil_div(a.nkb, S);
-  a.splits = S;
-  a.units = tiles * S;
-  if (S == 1) {
-    const int grid = a.units < g_num_sms ? a.units : g_num_sms;
-    gemm_kernel<<<grid, kGemmThreads, kGemmSmem, s>>>(maps.a, maps.b, a);
-    return cudaGetLastError();
-  }
-  cudaLaunchConfig_t cfg = {};
-  cudaLaunchAttribute attr;
-  attr.id = cudaLaunchAttributeClusterDimension;
-  attr.val.clusterDim.x = S;
-  attr.val.clusterDim.y = 1;
-  attr.val.clusterDim.z = 1;
-  cfg.gridDim = dim3(a.units, 1, 1);
-  cfg.blockDim = dim3(kGemmThreads, 1, 1);
-  cfg.dynamicSmemBytes = kGemmSmem;
-  cfg.stream = s;
-  cfg.attrs = &attr;
-  cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, gemm_kernel, maps.a, maps.b, a);
+cudaError_t launch_gemm(const CUtensorMap& mapA, const CUtensorMap& mapB, bool fused_x, int T,
+                        int N, int Kp, const GemmParams& p, cudaStream_t s) {
+  return fused_x ? launch_gemm_t<true>(mapA, mapB, T, N, Kp, p, s)
+                 : launch_gemm_t<false>(mapA, mapB, T, N, Kp, p, s);
 }
 
 }  // namespace sp

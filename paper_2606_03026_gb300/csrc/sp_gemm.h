@@ -19,12 +19,18 @@ cudaError_t gemm_make_maps(const __nv_bfloat16* Xb, int rows_alloc, const __nv_b
                            int N, int Kp, GemmMaps* out);
 cudaError_t launch_w_to_bf16(const int8_t* W, int64_t ldw, int N, int K, __nv_bfloat16* Wb,
                              cudaStream_t s);
+// TMA descriptor of u8 spike rows X [T][ldx] (nonzero = spike) read in
+// 64-column x 128-row boxes, zero past K and T.  X 16-byte aligned,
+// ldx % 16 == 0.
+cudaError_t gemm_make_x8_map(const void* X, int64_t ldx, int T, int K, CUtensorMap* out);
 // fp32 elements of one split-K partial (one 128 x 256 output tile).
 constexpr int kGemmPartialElems = 128 * 256;
-// ACC = X W^T on the tensor cores with the acc / y epilogue.  Splits K over
-// a thread-block cluster when the output has fewer tiles than SMs; the
+// ACC = X W^T on the tensor cores with the acc / y epilogue.  mapA is the
+// bf16 staging copy of X (gemm_make_maps), or with fused_x the u8 spike rows
+// themselves (gemm_make_x8_map), converted to bf16 inside the kernel.  Splits
+// K over a thread-block cluster when the output has fewer tiles than SMs; the
 // partials meet in p.part (at least one per SM: p.part_units >= SM count).
-cudaError_t launch_gemm(const GemmMaps& maps, int T, int N, int Kp, const GemmParams& p,
-                        cudaStream_t s);
+cudaError_t launch_gemm(const CUtensorMap& mapA, const CUtensorMap& mapB, bool fused_x, int T,
+                        int N, int Kp, const GemmParams& p, cudaStream_t s);
 
 }  // namespace sp

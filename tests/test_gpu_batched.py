@@ -83,6 +83,25 @@ def test_gemm_ragged(T, N, K, ldq):
         assert_parity(acc, y, want_acc, want_y, f"T={T} N={N} K={K} {strategy}")
 
 
+@pytest.mark.parametrize("T,N,K", [(1, 16, 1), (5, 48, 100), (129, 272, 1000), (300, 1552, 777),
+                                   (257, 512, 6143)])
+def test_gemm_u8_rows_read_in_kernel(T, N, K):
+    """u8 spike rows with a 16-byte-aligned row stride are read by the
+    tensor-core kernel itself (no bf16 staging copy): any nonzero byte is a
+    spike, bytes past K in each row are ignored, rows and K-blocks ragged."""
+    Qc, s, X = synth.random_case(80 + T, N, K, T=T, p=0.3)
+    ldx = (K + 15) // 16 * 16 + 16
+    rng = synth.rng_for(81, T, K)
+    Xs = rng.integers(1, 256, size=(T, ldx)).astype(np.uint8)     # garbage past K
+    Xs[:, :K] = np.where(X != 0, rng.integers(1, 256, size=(T, K)), 0).astype(np.uint8)
+    want_acc, want_y = oracle.project(Qc, s, N, K, X, "u8")
+    plan = sp.Plan(to_dev(Qc), to_dev(s), N, K, max_batch=T, gemm=True)
+    for rep in range(2):
+        acc, y = run_batched(plan, to_dev(Xs), "u8", T, ldx, N, "gemm")
+        assert_parity(acc, y, want_acc, want_y, f"T={T} N={N} K={K} rep {rep}")
+    assert plan.status() == sp.SP_OK
+
+
 def test_gemm_extremes():
     """All-ones spikes against -128 / +127 weights: the largest sums the
     tensor-core path must carry exactly (|acc| = 128 * K)."""
