@@ -203,9 +203,15 @@ sp_status run_union(sp_plan_s* p, const void* spikes, int fmt, int B, int64_t ld
 sp_status run_gemm(sp_plan_s* p, const void* spikes, int fmt, int T, int64_t ld, int32_t* acc,
                    float* y, cudaStream_t s) {
   if (!(p->flags & SP_PLAN_GEMM)) return SP_EUNSUPPORTED;
-  // u8 rows that TMA can read directly are converted inside the GEMM kernel;
-  // anything else goes through the bf16 staging copy first
-  const bool fused = fmt == SP_SPIKES_U8 && aligned(spikes, 16) && ld % 16 == 0;
+  // u8 rows that TMA can read directly are converted inside the GEMM kernel
+  // when K is split (the fused form's shape); anything else goes through the
+  // bf16 staging copy first
+  bool fused = fmt == SP_SPIKES_U8 && aligned(spikes, 16) && ld % 16 == 0;
+  int S = gemm_splits(fused, T, p->N, p->Kp, p->part_units);
+  if (fused && S < 2) {
+    fused = false;
+    S = gemm_splits(false, T, p->N, p->Kp, p->part_units);
+  }
   if (fused) {
     if (spikes != p->x8_ptr || ld != p->x8_ld || T != p->x8_T) {
       SP_CUDA(gemm_make_x8_map(spikes, ld, T, p->K, &p->x8map));
@@ -226,7 +232,7 @@ sp_status run_gemm(sp_plan_s* p, const void* spikes, int fmt, int T, int64_t ld,
   g.err = p->err;
   g.part = p->part;
   g.part_units = p->part_units;
-  SP_CUDA(launch_gemm(fused ? p->x8map : p->maps.a, p->maps.b, fused, T, p->N, p->Kp, g, s));
+  SP_CUDA(launch_gemm(fused ? p->x8map : p->maps.a, p->maps.b, fused, S, T, p->N, p->Kp, g, s));
   return SP_OK;
 }
 

@@ -53,12 +53,24 @@ constexpr int kGemmThreads = 192;             // TMA, MMA and 4 epilogue warps
 constexpr int kConvThreads = 256;             // 8 warps converting u8 spikes to bf16
 constexpr int kGemmThreadsFused = kGemmThreads + kConvThreads;
 constexpr int X8_BYTES = BM * BK;             // one u8 spike tile (8 KB)
-constexpr int X8_OFFSET = A_BYTES - X8_BYTES; // lands in the upper half of the A slot
 constexpr int TR_STRIDE = 33;                 // padded transpose rows (words)
 constexpr size_t SMEM_RING = (size_t)STAGES * STAGE_BYTES;
 constexpr size_t SMEM_TR = (size_t)4 * 32 * TR_STRIDE * 4;
+constexpr size_t SMEM_X8 = (size_t)STAGES * X8_BYTES;   // u8 spike ring (fused form)
 constexpr size_t SMEM_BARS = 256;
-constexpr size_t kGemmSmem = 1024 + SMEM_RING + SMEM_TR + SMEM_BARS;
+// Past the operand ring: the epilogue transpose buffer, or in the fused form
+// the u8 spike ring, which the transpose buffer reuses once the K loop is done
+// (the fused form always splits K, so its epilogue runs after the K loop).
+template <bool kFusedX>
+__host__ __device__ constexpr size_t gemm_smem_extra() {
+  return kFusedX ? SMEM_X8 : SMEM_TR;
+}
+template <bool kFusedX>
+__host__ __device__ constexpr size_t gemm_smem() {
+  return 1024 + SMEM_RING + gemm_smem_extra<kFusedX>() + SMEM_BARS;
+}
+static_assert(SMEM_X8 >= SMEM_TR, "the transpose buffer fits the idle u8 ring");
+static_assert(gemm_smem<true>() <= 227 * 1024, "shared memory of the fused form");
 
 // Shared-memory matrix descriptor (tcgen05 format): K-major operand whose rows
 // are 128 bytes (64 bf16) laid out by TMA with the 128-byte swizzle; 8-row
@@ -156,63 +168,71 @@ __device__ __forceinline__ void store_chunk(const GemmParams& p, uint32_t* tr,
   __syncwarp();
 }
 
-// True on all converter threads if `v` is true on any of them (named barrier
-// 1 with a predicate reduction): the converter warps take every abort
-// decision together, so none can be left waiting at barrier 1.
-__device__ __forceinline__ bool converters_any(bool v) {
-  uint32_t r;
-  asm volatile(
-      "{\n\t.reg .pred p, q;\n\tsetp.ne.u32 p, %1, 0;\n\t"
-      "bar.red.or.pred q, 1, %2, p;\n\tselp.u32 %0, 1, 0, q;\n\t}"
-      : "=r"(r)
-      : "r"((uint32_t)v), "n"(kConvThreads)
-      : "memory");
-  return r != 0;
-}
+// One u8 spike tile (128 rows x 64 columns, 64-byte rows, TMA-loaded into
+// the u8 ring) -> the A slot's bf16 0/1 tile in the 128-byte-swizzle layout
+// the MMA descriptor expects (16-byte chunk j of row r at
+// r * 128 + (j ^ (r % 8)) * 16).  Item i = (row i / 8, chunk i % 8): 8 u8
+// bytes in, one 16-byte bf16 chunk out; thread t converts items t, t + 256,
+// t + 512, t + 768, so every 8 consecutive threads read 64 contiguous bytes
+// and write one whole 128-byte row (no shared-memory bank conflicts).
+// Split in two so that the u8 slot can be released between them.
+constexpr int kConvItems = BM * 8 / kConvThreads;   // 4
 
-// 128 u8 spike rows x 64 columns (TMA-loaded at X8_OFFSET of the A slot) ->
-// the slot's bf16 0/1 tile in the 128-byte-swizzle layout the MMA descriptor
-// expects (16-byte chunk j of row r at r * 128 + (j ^ (r % 8)) * 16).
-// Thread t (0..255) converts half h = t % 2 of row r = t / 2 (columns 32h ..
-// 32h + 31).  Every thread reads before any writes (named barrier 1), since
-// the bf16 rows 64..127 cover the u8 tile.
-__device__ __forceinline__ void convert_x8_tile(uint8_t* slot, int t) {
-  const int r = t >> 1, h = t & 1;
-  const uint4* src = reinterpret_cast<const uint4*>(slot + X8_OFFSET + r * BK + h * 32);
-  const uint4 u0 = src[0], u1 = src[1];
-  asm volatile("bar.sync 1, %0;" ::"n"(kConvThreads) : "memory");
-  const uint32_t w[8] = {u0.x, u0.y, u0.z, u0.w, u1.x, u1.y, u1.z, u1.w};
-  uint8_t* row = slot + r * 128;
+__device__ __forceinline__ void convert_x8_load(const uint8_t* x8, int t, uint4 (&o)[kConvItems]) {
+  uint2 u[kConvItems];
 #pragma unroll
-  for (int jj = 0; jj < 4; ++jj) {            // chunk j = 4h + jj: columns 8j .. 8j + 7
-    uint32_t o[4];
+  for (int k = 0; k < kConvItems; ++k) {
+    const int i = t + k * kConvThreads;
+    u[k] = *reinterpret_cast<const uint2*>(x8 + (i >> 3) * BK + (i & 7) * 8);
+  }
+#pragma unroll
+  for (int k = 0; k < kConvItems; ++k) {
+    uint32_t w[4];
 #pragma unroll
     for (int e = 0; e < 2; ++e) {
-      const uint32_t v = w[2 * jj + e];
+      const uint32_t v = e ? u[k].y : u[k].x;
       // 0x80 in every nonzero byte (the low byte of bf16 1.0 = 0x3f80), 0 elsewhere
       const uint32_t lo = (((v & 0x7f7f7f7fu) + 0x7f7f7f7fu) | v) & 0x80808080u;
       const uint32_t hi = (lo >> 7) * 0x3fu;
-      o[2 * e] = __byte_perm(lo, hi, 0x5140);
-      o[2 * e + 1] = __byte_perm(lo, hi, 0x7362);
+      w[2 * e] = __byte_perm(lo, hi, 0x5140);
+      w[2 * e + 1] = __byte_perm(lo, hi, 0x7362);
     }
-    const int j = 4 * h + jj;
-    *reinterpret_cast<uint4*>(row + ((j ^ (r & 7)) << 4)) = make_uint4(o[0], o[1], o[2], o[3]);
+    o[k] = make_uint4(w[0], w[1], w[2], w[3]);
   }
 }
 
-// kFusedX: operand A is u8 spikes (converted in shared memory by warps 6-13)
-// instead of the bf16 staging copy.
+__device__ __forceinline__ void convert_x8_store(uint8_t* slot, int t, const uint4 (&o)[kConvItems]) {
+#pragma unroll
+  for (int k = 0; k < kConvItems; ++k) {
+    const int i = t + k * kConvThreads;
+    const int r = i >> 3, j = i & 7;
+    *reinterpret_cast<uint4*>(slot + r * 128 + ((j ^ (r & 7)) << 4)) = o[k];
+  }
+}
+
+// kFusedX: operand A is u8 spikes instead of the bf16 staging copy.  Lane 1
+// of the TMA warp streams the u8 tiles into their own ring; warps 6-13 read
+// and convert each tile into registers, hand the u8 slot back at once (so
+// the u8 stream runs up to two rings ahead of the tensor core), and write
+// the bf16 tile into its A slot as soon as the MMA has released that slot.
+// The fused form is launched with split K only (its epilogue transpose
+// buffer is the idle u8 ring).
 template <bool kFusedX>
 __global__ void __launch_bounds__(kFusedX ? kGemmThreadsFused : kGemmThreads, 1)
 gemm_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB,
             const __grid_constant__ GemmArgs a) {
+  if (kFusedX && a.splits < 2) {            // launch error: nothing has started yet
+    if (threadIdx.x == 0) atomicExch(a.p.err, kErrBadUnit);
+    return;
+  }
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
   uint8_t* sA = smem;
   uint8_t* sB = smem + (size_t)STAGES * A_BYTES;
   uint32_t* s_tr = reinterpret_cast<uint32_t*>(smem + SMEM_RING);
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + SMEM_RING + SMEM_TR);
+  uint8_t* sX8 = smem + SMEM_RING;          // fused form: u8 spike ring (aliases s_tr)
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + SMEM_RING + gemm_smem_extra<kFusedX>());
   uint64_t* full = bars;                 // [STAGES] TMA -> MMA
   uint64_t* empty = bars + STAGES;       // [STAGES] MMA -> TMA
   uint64_t* tfull = bars + 2 * STAGES;   // [2] MMA -> epilogue
@@ -220,7 +240,9 @@ gemm_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CU
   uint64_t* done = tempty + 2;           // all MMAs retired
   uint64_t* pfull = done + 1;            // split K: peers' partials landed
   uint64_t* conv = pfull + 1;            // [STAGES] converted A tile ready (fused)
-  uint32_t* s_tmem = reinterpret_cast<uint32_t*>(conv + STAGES);
+  uint64_t* full8 = conv + STAGES;       // [STAGES] u8 tile landed (fused)
+  uint64_t* empty8 = full8 + STAGES;     // [STAGES] u8 slot consumed (fused)
+  uint32_t* s_tmem = reinterpret_cast<uint32_t*>(empty8 + STAGES);
   volatile int* s_abort = reinterpret_cast<volatile int*>(s_tmem + 1);
 
   const int warp = threadIdx.x >> 5;
@@ -237,7 +259,11 @@ gemm_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CU
     }
     mbar_init(done, 1);
     mbar_init(pfull, 1);
-    for (int s = 0; s < STAGES; ++s) mbar_init(&conv[s], kConvThreads / 32);  // per converter warp
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(&conv[s], kConvThreads / 32);     // one arrive per converter warp
+      mbar_init(&full8[s], 1);
+      mbar_init(&empty8[s], kConvThreads / 32);
+    }
     *s_abort = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     tma_prefetch_desc(&mapA);
@@ -251,7 +277,11 @@ gemm_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CU
 
   if (warp == 0) {
     // ------------------------------ TMA producer ------------------------------
-    if (lane == 0) {
+    // lane 0: the W tiles (and the bf16 A tiles); lane 1 (fused): the u8 tiles
+    if (lane == 0 || (kFusedX && lane == 1)) {
+      const bool x8 = lane == 1;
+      uint64_t* fb = x8 ? full8 : full;
+      uint64_t* eb = x8 ? empty8 : empty;
       int stage = 0;
       uint32_t ph = 0;
       int issued = 0;                       // ring slots filled, for the drain
@@ -259,20 +289,21 @@ gemm_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CU
         int tile, mb, nb, kb0, kb1;
         unit_coords(a, u, tile, mb, nb, kb0, kb1);
         for (int kb = kb0; kb < kb1; ++kb) {
-          if (!mbar_wait(&empty[stage], ph ^ 1u)) {
+          if (!mbar_wait(&eb[stage], ph ^ 1u)) {
             *s_abort = 1;
             atomicExch(a.p.err, kErrMbarTimeout);
             break;
           }
-          if (kFusedX) {
-            mbar_arrive_expect_tx(&full[stage], X8_BYTES + B_BYTES);
-            tma_load_2d(sA + (size_t)stage * A_BYTES + X8_OFFSET, &mapA, &full[stage], kb * BK,
-                        mb * BM);
+          if (x8) {
+            mbar_arrive_expect_tx(&fb[stage], X8_BYTES);
+            tma_load_2d(sX8 + (size_t)stage * X8_BYTES, &mapA, &fb[stage], kb * BK, mb * BM);
+          } else if (kFusedX) {
+            mbar_arrive_expect_tx(&fb[stage], B_BYTES);
           } else {
-            mbar_arrive_expect_tx(&full[stage], STAGE_BYTES);
-            tma_load_2d(sA + (size_t)stage * A_BYTES, &mapA, &full[stage], kb * BK, mb * BM);
+            mbar_arrive_expect_tx(&fb[stage], STAGE_BYTES);
+            tma_load_2d(sA + (size_t)stage * A_BYTES, &mapA, &fb[stage], kb * BK, mb * BM);
           }
-          tma_load_2d(sB + (size_t)stage * B_BYTES, &mapB, &full[stage], kb * BK, nb * BN);
+          if (!x8) tma_load_2d(sB + (size_t)stage * B_BYTES, &mapB, &fb[stage], kb * BK, nb * BN);
           ++issued;
           if (++stage == STAGES) { stage = 0; ph ^= 1u; }
         }
@@ -283,7 +314,7 @@ gemm_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CU
       uint32_t q = ph;
       for (int i = 0; i < STAGES && i < issued; ++i) {
         if (--s < 0) { s = STAGES - 1; q ^= 1u; }
-        mbar_wait(&full[s], q);
+        mbar_wait(&fb[s], q);
       }
     }
   } else if (warp == 1) {
@@ -305,7 +336,7 @@ gemm_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CU
         const uint32_t d = tmem_base + (uint32_t)(ab * BN);
         bool ok = true;
         for (int kb = kb0; kb < kb1; ++kb) {
-          if (!mbar_wait(kFusedX ? &conv[stage] : &full[stage], ph)) {
+          if (!mbar_wait(&full[stage], ph) || (kFusedX && !mbar_wait(&conv[stage], ph))) {
             ok = false;
             break;
           }
@@ -331,9 +362,10 @@ gemm_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CU
     }
   } else if (kFusedX && warp >= 6) {
     // ------------------------- spike converters (fused) -----------------------
-    // Same (unit, K block) sequence as the producer: wait for the u8 tile,
-    // expand it in place, make the writes visible to the tensor core (async
-    // proxy) and release the slot to the MMA warp.
+    // Same (unit, K block) sequence as the producer: once the u8 tile has
+    // landed and the MMA has released the A slot, expand the tile into the
+    // slot, make the writes visible to the tensor core (async proxy), and
+    // release the A slot to the MMA warp and the u8 slot to the producer.
     const int ct = threadIdx.x - kGemmThreads;   // 0 .. kConvThreads - 1
     int stage = 0;
     uint32_t ph = 0;
@@ -342,14 +374,25 @@ gemm_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CU
       int tile, mb, nb, kb0, kb1;
       unit_coords(a, u, tile, mb, nb, kb0, kb1);
       for (int kb = kb0; kb < kb1; ++kb) {
-        const bool bad = *s_abort || !mbar_wait(&full[stage], ph);
-        if (converters_any(bad)) {
+        if (*s_abort || !mbar_wait(&full8[stage], ph)) {
           *s_abort = 1;
-          if (ct == 0) atomicExch(a.p.err, kErrMbarTimeout);
+          if (lane == 0) atomicExch(a.p.err, kErrMbarTimeout);
           ok = false;
           break;
         }
-        convert_x8_tile(sA + (size_t)stage * A_BYTES, ct);
+        // the converted tile is in registers (it depends on every u8 load),
+        // so the u8 slot goes back to the producer before the A slot is free
+        uint4 o[kConvItems];
+        convert_x8_load(sX8 + (size_t)stage * X8_BYTES, ct, o);
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&empty8[stage]);
+        if (!mbar_wait(&empty[stage], ph ^ 1u)) {
+          *s_abort = 1;
+          if (lane == 0) atomicExch(a.p.err, kErrMbarTimeout);
+          ok = false;
+          break;
+        }
+        convert_x8_store(sA + (size_t)stage * A_BYTES, ct, o);
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
         __syncwarp();
         if (lane == 0) mbar_arrive(&conv[stage]);
@@ -588,7 +631,7 @@ int max_active_clusters(int size) {
     attr.val.clusterDim.z = 1;
     cfg.gridDim = dim3(size, 1, 1);
     cfg.blockDim = dim3(gemm_threads<kFusedX>(), 1, 1);
-    cfg.dynamicSmemBytes = kGemmSmem;
+    cfg.dynamicSmemBytes = gemm_smem<kFusedX>();
     cfg.attrs = &attr;
     cfg.numAttrs = 1;
     int n = 0;
@@ -606,7 +649,7 @@ cudaError_t set_gemm_attrs() {
   static bool done = false;
   if (done) return cudaSuccess;
   cudaError_t e = cudaFuncSetAttribute(gemm_kernel<kFusedX>,
-                                       cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kGemmSmem);
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, (int)gemm_smem<kFusedX>());
   if (e != cudaSuccess) return e;
   e = cudaFuncSetAttribute(gemm_kernel<kFusedX>, cudaFuncAttributeNonPortableClusterSizeAllowed, 0);
   if (e != cudaSuccess) return e;
@@ -614,17 +657,42 @@ cudaError_t set_gemm_attrs() {
   return cudaSuccess;
 }
 
+cudaError_t init_sms() {
+  if (g_attr_set) return cudaSuccess;
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  e = cudaDeviceGetAttribute(&g_num_sms, cudaDevAttrMultiProcessorCount, dev);
+  if (e != cudaSuccess) return e;
+  g_attr_set = true;
+  return cudaSuccess;
+}
+
+// K splits for a T x N output: split only when the tiles alone leave SMs
+// idle, and only as far as every cluster stays resident in a single wave.
 template <bool kFusedX>
-cudaError_t launch_gemm_t(const CUtensorMap& mapA, const CUtensorMap& mapB, int T, int N, int Kp,
-                          const GemmParams& p, cudaStream_t s) {
-  if (!g_attr_set) {
-    int dev = 0;
-    cudaError_t e = cudaGetDevice(&dev);
-    if (e != cudaSuccess) return e;
-    e = cudaDeviceGetAttribute(&g_num_sms, cudaDevAttrMultiProcessorCount, dev);
-    if (e != cudaSuccess) return e;
-    g_attr_set = true;
+int pick_splits(int T, int N, int Kp, int part_units) {
+  const int tiles = ceil_div(T, BM) * ceil_div(N, BN);
+  const int nkb = Kp / BK;
+  int S = 1;
+  if (tiles < g_num_sms) {
+    S = g_num_sms / tiles;
+    if (S > 8) S = 8;
+    if (S > nkb / 4) S = nkb / 4;
+    if (S < 1) S = 1;
+    while (S > 1) {
+      const int kbps = ceil_div(nkb, S);
+      const int exact = ceil_div(nkb, kbps);            // splits with work
+      if (exact == S && max_active_clusters<kFusedX>(S) >= tiles && tiles * S <= part_units) break;
+      --S;
+    }
   }
+  return S;
+}
+
+template <bool kFusedX>
+cudaError_t launch_gemm_t(const CUtensorMap& mapA, const CUtensorMap& mapB, int S, int T, int N,
+                          int Kp, const GemmParams& p, cudaStream_t s) {
   cudaError_t e = set_gemm_attrs<kFusedX>();
   if (e != cudaSuccess) return e;
   GemmArgs a;
@@ -632,30 +700,14 @@ cudaError_t launch_gemm_t(const CUtensorMap& mapA, const CUtensorMap& mapB, int 
   a.tiles_m = ceil_div(T, BM);
   a.tiles_n = ceil_div(N, BN);
   a.nkb = Kp / BK;
-  const int tiles = a.tiles_m * a.tiles_n;
-  // Split K over a cluster only when the tiles alone leave SMs idle, and only
-  // as far as every cluster stays resident in a single wave.
-  int S = 1;
-  if (tiles < g_num_sms) {
-    S = g_num_sms / tiles;
-    if (S > 8) S = 8;
-    if (S > a.nkb / 4) S = a.nkb / 4;
-    if (S < 1) S = 1;
-    while (S > 1) {
-      const int kbps = ceil_div(a.nkb, S);
-      const int exact = ceil_div(a.nkb, kbps);          // splits with work
-      if (exact == S && max_active_clusters<kFusedX>(S) >= tiles && tiles * S <= p.part_units)
-        break;
-      --S;
-    }
-  }
   a.kb_per_split = ceil_div(a.nkb, S);
   a.splits = S;
-  a.units = tiles * S;
+  a.units = a.tiles_m * a.tiles_n * S;
   const int threads = gemm_threads<kFusedX>();
+  const size_t smem = gemm_smem<kFusedX>();
   if (S == 1) {
     const int grid = a.units < g_num_sms ? a.units : g_num_sms;
-    gemm_kernel<kFusedX><<<grid, threads, kGemmSmem, s>>>(mapA, mapB, a);
+    gemm_kernel<kFusedX><<<grid, threads, smem, s>>>(mapA, mapB, a);
     return cudaGetLastError();
   }
   cudaLaunchConfig_t cfg = {};
@@ -666,7 +718,7 @@ cudaError_t launch_gemm_t(const CUtensorMap& mapA, const CUtensorMap& mapB, int 
   attr.val.clusterDim.z = 1;
   cfg.gridDim = dim3(a.units, 1, 1);
   cfg.blockDim = dim3(threads, 1, 1);
-  cfg.dynamicSmemBytes = kGemmSmem;
+  cfg.dynamicSmemBytes = smem;
   cfg.stream = s;
   cfg.attrs = &attr;
   cfg.numAttrs = 1;
@@ -721,10 +773,23 @@ cudaError_t gemm_make_x8_map(const void* X, int64_t ldx, int T, int K, CUtensorM
   return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
 }
 
-cudaError_t launch_gemm(const CUtensorMap& mapA, const CUtensorMap& mapB, bool fused_x, int T,
-                        int N, int Kp, const GemmParams& p, cudaStream_t s) {
-  return fused_x ? launch_gemm_t<true>(mapA, mapB, T, N, Kp, p, s)
-                 : launch_gemm_t<false>(mapA, mapB, T, N, Kp, p, s);
+int gemm_splits(bool fused_x, int T, int N, int Kp, int part_units) {
+  if (init_sms() != cudaSuccess) return 1;
+  if (fused_x) {
+    if (set_gemm_attrs<true>() != cudaSuccess) return 1;
+    return pick_splits<true>(T, N, Kp, part_units);
+  }
+  if (set_gemm_attrs<false>() != cudaSuccess) return 1;
+  return pick_splits<false>(T, N, Kp, part_units);
+}
+
+cudaError_t launch_gemm(const CUtensorMap& mapA, const CUtensorMap& mapB, bool fused_x, int S,
+                        int T, int N, int Kp, const GemmParams& p, cudaStream_t s) {
+  cudaError_t e = init_sms();
+  if (e != cudaSuccess) return e;
+  if (fused_x && S < 2) return cudaErrorInvalidValue;
+  return fused_x ? launch_gemm_t<true>(mapA, mapB, S, T, N, Kp, p, s)
+                 : launch_gemm_t<false>(mapA, mapB, S, T, N, Kp, p, s);
 }
 
 }  // namespace sp

@@ -25,12 +25,15 @@ cudaError_t launch_w_to_bf16(const int8_t* W, int64_t ldw, int N, int K, __nv_bf
 cudaError_t gemm_make_x8_map(const void* X, int64_t ldx, int T, int K, CUtensorMap* out);
 // fp32 elements of one split-K partial (one 128 x 256 output tile).
 constexpr int kGemmPartialElems = 128 * 256;
-// ACC = X W^T on the tensor cores with the acc / y epilogue.  mapA is the
-// bf16 staging copy of X (gemm_make_maps), or with fused_x the u8 spike rows
-// themselves (gemm_make_x8_map), converted to bf16 inside the kernel.  Splits
-// K over a thread-block cluster when the output has fewer tiles than SMs; the
-// partials meet in p.part (at least one per SM: p.part_units >= SM count).
-cudaError_t launch_gemm(const CUtensorMap& mapA, const CUtensorMap& mapB, bool fused_x, int T,
-                        int N, int Kp, const GemmParams& p, cudaStream_t s);
+// K splits the launch will use for a T x N output (1 = no split): as many as
+// leave no SM idle while every cluster of splits stays resident at once.
+int gemm_splits(bool fused_x, int T, int N, int Kp, int part_units);
+// ACC = X W^T on the tensor cores with the acc / y epilogue, K split S ways
+// (gemm_splits) over a thread-block cluster; the partials meet in p.part (at
+// least one per SM: p.part_units >= SM count).  mapA is the bf16 staging copy
+// of X (gemm_make_maps), or with fused_x (requires S >= 2) the u8 spike rows
+// themselves (gemm_make_x8_map), converted to bf16 inside the kernel.
+cudaError_t launch_gemm(const CUtensorMap& mapA, const CUtensorMap& mapB, bool fused_x, int S,
+                        int T, int N, int Kp, const GemmParams& p, cudaStream_t s);
 
 }  // namespace sp
