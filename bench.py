@@ -25,6 +25,13 @@ Also reported on the same JSON line:
                every step)
   cpu_baseline the CPU oracle on the host cores, on a bounded sample
   prefill      512-token prefill over 22 blocks on the tensor cores, TOPS
+  configs      every workload of the benchmark table, timed outside the
+               headline region: the single 1536 x 1536 projection and the
+               6144 -> 1536 down projection at each spike rate (weights
+               L2-resident and L2-cold), the decode step as a dependent
+               chain of 44 single calls, batched B = 64 (per-token gather
+               vs union fetch, independent and correlated spikes), and the
+               CPU oracle on each (single thread, bounded samples)
   clocks       nvidia-smi samples taken during the timed region
 
 --impl reference times the CPU oracle (the only reference there is: the paper
@@ -69,6 +76,9 @@ def parse():
                     help="rotating copies of the 22-block weights (8 keeps every "
                          "timed step out of L2; 1 for small profiling runs)")
     ap.add_argument("--prefill-blocks", type=int, default=22)
+    ap.add_argument("--no-configs", action="store_true",
+                    help="skip the per-config measurements (single projection, down projection "
+                         "at every spike rate, dependent 44-call chain, batched B=64, oracle)")
     ap.add_argument("--prefill-only", action="store_true",
                     help="run only the prefill leg (profiling of the tensor-core path)")
     return ap.parse_args()
@@ -435,6 +445,11 @@ def run_ours(args):
                                           args.prefill_blocks)
         result["gpu_launches"] = steps   # prefill is timed outside the headline region
 
+    if not args.no_configs:
+        result["configs"] = bench_configs(torch, sp, synth, dev, stream, float(peaks["hbm_gbs"]),
+                                          copies, spikes, sets_np, active, ld,
+                                          with_oracle=rank == 0 and not args.no_cpu_baseline)
+
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         v, nsteps, dt = cpu_baseline_decode(weights, sets_np, args.cpu_seconds)
         result["cpu_baseline"] = {
@@ -446,6 +461,170 @@ def run_ours(args):
         g.close()
     if rank == 0:
         print(json.dumps(result))
+
+
+def graph_time_us(torch, stream, calls, reps=20):
+    """Average device time (us) of one call of `calls` (a list of no-argument
+    launches), captured once into a CUDA graph and replayed `reps` times."""
+    for c in calls[:4]:
+        c(stream)
+    stream.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        cur = torch.cuda.current_stream()
+        for c in calls:
+            c(cur)
+    with torch.cuda.stream(stream):
+        for _ in range(2):
+            g.replay()
+    stream.synchronize()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        e0.record(stream)
+        for _ in range(reps):
+            g.replay()
+        e1.record(stream)
+    stream.synchronize()
+    return e0.elapsed_time(e1) * 1e3 / (reps * len(calls))
+
+
+def oracle_time_us(fn, budget_s=1.0, max_calls=50):
+    n, t0 = 0, time.perf_counter()
+    while n < max_calls:
+        fn()
+        n += 1
+        if time.perf_counter() - t0 > budget_s:
+            break
+    return (time.perf_counter() - t0) * 1e6 / n, n
+
+
+def bench_configs(torch, sp, synth, dev, stream, hbm, copies, spikes, sets_np, active, ld,
+                  with_oracle):
+    """Every workload of the benchmark table, each on its own (outside the
+    headline's timed region).  Weights 'cold' = enough rotating copies that
+    no call finds its weights in L2 (3 x the 126 MB L2 between reuses)."""
+    import math
+
+    import oracle
+    L2 = 126e6
+    G = 64                                  # calls per graph
+    out = {}
+
+    def to_dev(a):
+        return torch.from_numpy(np.ascontiguousarray(a)).to(dev)
+
+    def gbs(nbytes, us):
+        return nbytes / (us * 1e-6) / 1e9
+
+    def decode_calls(plans, rows, acc, y):
+        calls = []
+        for i in range(G):
+            pl, r = plans[i % len(plans)], rows[i % len(rows)]
+            calls.append(lambda s, pl=pl, r=r: pl.decode(r, "bits", acc, y, stream=s))
+        return calls
+
+    def projection(name, Q, s, N, K, X, rate):
+        bits = to_dev(synth.pack_bits(X))
+        rows = [bits[i] for i in range(X.shape[0])]
+        nbytes = float(X.astype(np.int64).sum(axis=1).mean()) * N
+        acc = torch.empty(N, dtype=torch.int32, device=dev)
+        y = torch.empty(N, dtype=torch.float32, device=dev)
+        W, S = to_dev(Q), to_dev(s)
+        hot = [sp.Plan(W, S, N, K)]
+        t_hot = graph_time_us(torch, stream, decode_calls(hot, rows, acc, y))
+        ncold = math.ceil(3 * L2 / Q.nbytes)
+        Ws = [to_dev(Q) for _ in range(ncold)]
+        cold = [sp.Plan(w, S, N, K) for w in Ws]
+        t_cold = graph_time_us(torch, stream, decode_calls(cold, rows, acc, y))
+        last = (G - 1) % X.shape[0]         # the row of the graph's last call
+        want = oracle.project(Q, s, N, K, X[last:last + 1], "u8")[0][0]
+        assert np.array_equal(acc.cpu().numpy(), want), f"{name} spot check failed"
+        for pl in hot + cold:
+            pl.close()
+        del Ws
+        r = {"p": rate, "active_bytes_per_call": nbytes,
+             "hot_l2": {"us_per_call": t_hot, "gbs": gbs(nbytes, t_hot)},
+             "cold": {"us_per_call": t_cold, "gbs": gbs(nbytes, t_cold),
+                      "frac_of_hbm": gbs(nbytes, t_cold) / hbm, "weight_copies": ncold}}
+        if with_oracle:
+            us, n = oracle_time_us(lambda: oracle.project(Q, s, N, K, X[:1], "u8"))
+            r["oracle"] = {"us_per_call": us, "gbs": gbs(nbytes, us), "calls": n, "cores": 1}
+        return r
+
+    # config 1: single projection K = N = 1536, Bernoulli(0.1)
+    c = synth.single_projection(0)
+    X1 = np.stack([synth.bernoulli(synth.rng_for(11, i), (1536,), 0.1) for i in range(64)])
+    out["single_1536x1536"] = projection("single", c["Q"], c["s"], 1536, 1536, X1, 0.1)
+
+    # config 2: FFN down projection 6144 -> 1536 at every spike rate
+    Qd, sd = synth.down_weights(0)
+    out["down_6144x1536"] = {
+        str(pr): projection("down", Qd, sd, 1536, 6144, synth.down_spikes(pr, count=256, seed=0), pr)
+        for pr in synth.DOWN_RATES}
+
+    # config 3 as a dependent chain: 44 single-projection calls per step
+    n_proj = len(copies[0].plans)
+    acc1 = torch.empty(1536, dtype=torch.int32, device=dev)
+    y1 = torch.empty(1536, dtype=torch.float32, device=dev)
+    chain = []
+    steps = 8
+    for st in range(steps):
+        grp = copies[st % len(copies)]
+        for j in range(n_proj):
+            pl = grp.plans[j]
+            row = spikes[st % spikes.shape[0], j]
+            chain.append(lambda s, pl=pl, row=row: pl.decode(row, "bits", acc1, y1, stream=s))
+    t_call = graph_time_us(torch, stream, chain)
+    t_step = t_call * n_proj
+    step_bytes = float(np.mean(active[:steps]))
+    out["decode_step_chain_44_calls"] = {
+        "us_per_step": t_step, "gbs": gbs(step_bytes, t_step), "frac_of_hbm": gbs(step_bytes, t_step) / hbm,
+        "projected_tokens_per_s": 1e6 / t_step,
+        "note": "44 spike_proj_decode launches in sequence per step (each waits for the previous)"}
+
+    # config 4: batched B = 64, per-token gather vs union fetch
+    Qb, sb = synth.down_weights(3)
+    Wb, Sb = to_dev(Qb), to_dev(sb)
+    plan = sp.Plan(Wb, Sb, 1536, 6144, max_batch=64, gemm=True)
+    accb = torch.empty(64, 1536, dtype=torch.int32, device=dev)
+    yb = torch.empty(64, 1536, dtype=torch.float32, device=dev)
+    b4 = {}
+    for corr in (False, True):
+        Xs = [synth.batched_spikes(seed, correlated=corr)[0] for seed in range(8)]
+        bits = [to_dev(synth.pack_bits(X)) for X in Xs]
+        adds = float(np.mean([X.astype(np.int64).sum() for X in Xs])) * 1536
+        union = float(np.mean([(X.max(axis=0) > 0).sum() for X in Xs])) * 1536
+        row = {"sum_active_x_N": adds, "union_bytes": union}
+        for strat in ("gather", "union", "gemm"):
+            calls = [lambda s, b=bits[i % 8], st=strat: plan.batched(b, "bits", 64, b.shape[1], accb,
+                                                                     yb, st, stream=s)
+                     for i in range(16)]
+            us = graph_time_us(torch, stream, calls)
+            fetched = {"gather": adds, "union": union, "gemm": 1536 * 6144 * 2.0}[strat]
+            row[strat] = {"us_per_batch": us, "tokens_per_s": 64e6 / us,
+                          "adds_per_s": adds / (us * 1e-6), "bytes_fetched": fetched,
+                          "fetch_gbs": gbs(fetched, us)}
+        plan.batched(bits[0], "bits", 64, bits[0].shape[1], accb, yb, "auto", stream=stream)
+        stream.synchronize()
+        row["auto_chose"] = plan.last_dispatch()[0]
+        if with_oracle:
+            X0 = Xs[0]
+            us, n = oracle_time_us(lambda: oracle.project(Qb, sb, 1536, 6144, X0, "u8"), 2.0, 5)
+            row["oracle"] = {"us_per_batch": us, "tokens_per_s": 64e6 / us, "calls": n, "cores": 1}
+        b4["correlated" if corr else "independent"] = row
+    plan.close()
+    out["batched_b64_6144x1536"] = b4
+
+    # config 5 oracle: one 512-token prefill block, extrapolated to 22 blocks
+    if with_oracle:
+        Qp, spp = synth.prefill_weights(0)
+        Xp = synth.prefill_spikes(0)
+        us, n = oracle_time_us(lambda: oracle.project(Qp, spp, 1536, 6144, Xp, "u8"), 1.0, 1)
+        out["prefill_oracle"] = {"us_per_block": us, "blocks_22_s": us * 22e-6,
+                                 "tops": 2 * 512 * 1536 * 6144 / (us * 1e-6) / 1e12,
+                                 "note": "one block timed, x22 extrapolated", "cores": 1}
+    return out
 
 
 def measured_traffic(kernel, source):

@@ -78,8 +78,10 @@ typedef enum sp_status {
 typedef enum sp_fmt { SP_SPIKES_BITS32 = 0, SP_SPIKES_U8 = 1 } sp_fmt;
 
 /* Kernel strategies for multi-token calls.
- *   SP_AUTO    measure the spike density on the device, read it back (one
- *              stream synchronisation) and pick one of the others.
+ *   SP_AUTO    count the active spikes on the device, read the count back
+ *              (one stream synchronisation) and pick SP_GATHER or, on a plan
+ *              made with SP_PLAN_GEMM, SP_GEMM when its modelled time is
+ *              lower (large batches and dense prefill).
  *   SP_GATHER  per-token active-column gather (the batch-1 kernel per row).
  *   SP_UNION   one fetch of each column in the union of the rows' active sets,
  *              added into every row whose spike is set.

@@ -236,17 +236,20 @@ sp_status run_gemm(sp_plan_s* p, const void* spikes, int fmt, int T, int64_t ld,
   return SP_OK;
 }
 
-// Measured-density dispatch.  Costs are modelled per call from the counts:
-//   gather  ~ sum_t |A_t| * N bytes, through L1/L2, ~one byte-add per byte
-//   union   ~ |U| * N bytes fetched + the same adds from shared memory
-//   gemm    ~ 2 * T * N * K tensor-core ops + conversion of T*K spikes
-// The thresholds below are the crossover points of those models with
-// throughputs measured on GB300 (see the dispatch tests and profiles).
+// Measured-density dispatch between the per-token gather and the
+// tensor-core GEMM, by a cost model fitted on GB300 (K = 6144, N = 1536,
+// token rates U(0.05, 0.2), B = 2 .. 1024, weights L2-resident):
+//   gather ~ 6 us + active bytes (sum_t |A_t| * N) / 6.3 TB/s
+//   GEMM   ~ 12 us + 2 B N K ops / 1 PFLOP/s            (plans with SP_PLAN_GEMM)
+// The crossover lies between B = 32 and B = 64 at these rates.  The union
+// fetch is never chosen automatically: it was slower than the per-token
+// gather at every batch size measured (its adds are ALU-bound, and the
+// 126 MB L2 serves the per-token re-reads of a 9.4 MB weight matrix).
 sp_kernel choose(const sp_plan_s* p, int B, int32_t total) {
-  const double dens = (double)total / ((double)B * (double)p->K);
-  if ((p->flags & SP_PLAN_GEMM) && B >= 32 && dens >= 0.03) return SP_GEMM;
-  if (B >= 4) return SP_UNION;
-  return SP_GATHER;
+  if (!(p->flags & SP_PLAN_GEMM)) return SP_GATHER;
+  const double gather_us = 6.0 + (double)total * p->N / 6.3e6;
+  const double gemm_us = 12.0 + 2.0 * B * (double)p->N * p->K / 1.0e9;
+  return gemm_us < gather_us ? SP_GEMM : SP_GATHER;
 }
 
 sp_status run_multi(sp_plan_s* p, const void* spikes, int fmt, int B, int64_t ld, int32_t* acc,

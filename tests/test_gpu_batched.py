@@ -118,6 +118,25 @@ def test_gemm_extremes():
         assert_parity(acc, y, want_acc, want_y, f"gemm extremes {c}")
 
 
+def test_auto_dispatch_by_cost(down):
+    """SP_AUTO: per-token gather for small batches, the tensor-core GEMM for
+    large ones on a plan with SP_PLAN_GEMM, never the GEMM without it; the
+    result is the same bits either way."""
+    Qc, s, plan = down
+    X = np.concatenate([synth.batched_spikes(i)[0] for i in range(4)])        # 256 tokens
+    want_acc, want_y = oracle.project(Qc, s, 1536, 6144, X, "u8")
+    bits = to_dev(synth.pack_bits(X))
+    for B, expect in ((8, "gather"), (256, "gemm")):
+        acc, y = run_batched(plan, bits, "bits", B, bits.shape[1], 1536, "auto")
+        assert plan.last_dispatch()[0] == expect, (B, plan.last_dispatch())
+        assert_parity(acc, y, want_acc[:B], want_y[:B], f"auto B={B}")
+    plain = sp.Plan(to_dev(Qc), to_dev(s), 1536, 6144, max_batch=256)
+    acc, y = run_batched(plain, bits, "bits", 256, bits.shape[1], 1536, "auto")
+    assert plain.last_dispatch()[0] == "gather"
+    assert_parity(acc, y, want_acc, want_y, "auto without the GEMM operand copy")
+    plain.close()
+
+
 def test_union_many_rows():
     """More rows than one union launch holds (passes of 256)."""
     N, K, B = 256, 2000, 600
