@@ -35,6 +35,9 @@ def noalloc_decode(W, ldw, S, N, K, spikes, fmt):
     (2064, 1025, 2080, 0.5),          # ragged tile, ragged chunk, ldw > N
     (16, 1, 16, 1.0),                 # smallest shape
     (sp.SPIKE_PROJ_NOALLOC_MAX_N, 1100, sp.SPIKE_PROJ_NOALLOC_MAX_N, 0.3),  # largest N
+    # K above 6144: split-K partials pass through the fixed scratch
+    (2064, 8000, 2080, 0.2),
+    (sp.SPIKE_PROJ_NOALLOC_MAX_N, 7000, sp.SPIKE_PROJ_NOALLOC_MAX_N, 0.1),
 ])
 @pytest.mark.parametrize("fmt", ["bits", "u8"])
 def test_noalloc_matches_plan_decode(N, K, ldq, p, fmt):
