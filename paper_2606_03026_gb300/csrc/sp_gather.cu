@@ -73,7 +73,9 @@ __device__ __forceinline__ void st_peer_v4(uint32_t local, uint32_t rank, int4 v
 }
 
 // CTA x of the first grid row prefetches rows x, x + gridDim.x, ... of the
-// (problem, token) spike rows into L2, one 128-byte line per thread.
+// (problem, token) spike rows into L2, one 128-byte line per thread, and the
+// scales of problems x, x + gridDim.x, ... (read only at the very end, when a
+// DRAM round trip would add to the kernel's tail).
 template <int NP>
 __device__ __forceinline__ void prefetch_spike_rows(const GatherParamsT<NP>& p) {
   const int rows = p.nprob * p.B;
@@ -84,6 +86,12 @@ __device__ __forceinline__ void prefetch_spike_rows(const GatherParamsT<NP>& p) 
     const char* row = static_cast<const char*>(spike_row(p.spikes, p.fmt, r, p.ld_spikes));
     for (int64_t off = (int64_t)threadIdx.x * 128; off < bytes; off += (int64_t)blockDim.x * 128)
       asm volatile("prefetch.global.L2 [%0];" ::"l"(row + off));
+  }
+  if (p.y == nullptr) return;
+  for (int j = blockIdx.x; j < p.nprob; j += gridDim.x) {
+    const char* sc = reinterpret_cast<const char*>(p.prob[j].scale);
+    for (int off = threadIdx.x * 128; off < p.prob[j].N * 4; off += blockDim.x * 128)
+      asm volatile("prefetch.global.L2 [%0];" ::"l"(sc + off));
   }
 }
 
@@ -239,14 +247,16 @@ __global__ void __launch_bounds__(kGatherThreads, 7)
 gather_kernel(const __grid_constant__ GatherParamsT<NP> p) {
   __shared__ TicketSmem sm;
   __shared__ int s_last;
-  // the next launch may take free SM slots now; this grid's own memory work
-  // starts once the previous kernel has finished
+  // The next launch may take free SM slots now.  The first grid row starts
+  // first: it pulls every spike row of the launch into L2 before the
+  // column-load burst fills the DRAM queues, so that units that start late
+  // do not wait behind that burst for their spike words.  A prefetch hands
+  // no data to the kernel, so it may run before the wait for the previous
+  // kernel (if that kernel writes the rows, L2 simply holds its writes);
+  // every load and store of this grid comes after the wait.
   pdl_launch_dependents();
-  pdl_wait();
-  // The first grid row starts first: it pulls every spike row of the launch
-  // into L2 before the column-load burst fills the DRAM queues, so that units
-  // that start late do not wait behind that burst for their spike words.
   if (blockIdx.y == 0) prefetch_spike_rows(p);
+  pdl_wait();
 
   const int j = blockIdx.y;
   const int t = (int)(blockIdx.x / (unsigned)p.max_units);
@@ -328,8 +338,8 @@ gather_cluster_kernel(const __grid_constant__ GatherParamsT<NP> p) {
   // [sender chunk][owned group]: kch * ceil(128 / kch) < 128 + kch entries
   __shared__ __align__(16) int4 s_recv[kGatherNT / 4 + kGatherCluster];
   pdl_launch_dependents();
+  if (blockIdx.y == 0) prefetch_spike_rows(p);   // before the wait: see gather_kernel
   pdl_wait();
-  if (blockIdx.y == 0) prefetch_spike_rows(p);
 
   const int j = blockIdx.y;
   const GatherProblem& P = p.prob[j];
