@@ -45,6 +45,7 @@ namespace sp {
 namespace {
 
 constexpr int BM = 128, BN = 256, BK = 64, STAGES = 4;
+constexpr int CPT = BN / 32;                  // 32-column chunks per output tile
 constexpr int A_BYTES = BM * BK * 2;          // 16 KB
 constexpr int B_BYTES = BN * BK * 2;          // 32 KB
 constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
@@ -105,12 +106,21 @@ __device__ __forceinline__ void cluster_sync() {
 }
 
 // Split-K exchange: one partial chunk (32 columns x 128 rows fp32) is 16 KB;
-// a rank owns at most kMaxOwned of the 8 chunks (S >= 2), and the S - 1
-// incoming partials of its chunks fit the idle ring: (S - 1) * ceil(8 / S)
-// chunks <= 12 for S <= 8.
+// a rank owns at most kMaxOwned of the CPT chunks of a tile (S >= 2), and the
+// S - 1 incoming partials of its chunks fit the idle ring.
 constexpr int kPartChunkBytes = 32 * BM * 4;
-constexpr int kMaxOwned = 4;
-static_assert(12 * kPartChunkBytes <= (int)SMEM_RING, "split-K partials fit the ring");
+constexpr int kMaxOwned = (CPT + 1) / 2;
+// most peer partials an owner receives: max over S of (S - 1) * ceil(CPT / S)
+constexpr int max_incoming_chunks() {
+  int m = 0;
+  for (int S = 2; S <= 8; ++S) {
+    const int n = (S - 1) * ((CPT + S - 1) / S);
+    if (n > m) m = n;
+  }
+  return m;
+}
+static_assert(max_incoming_chunks() * kPartChunkBytes <= (int)SMEM_RING,
+              "split-K partials fit the ring");
 
 struct GemmArgs {
   GemmParams p;
@@ -441,7 +451,7 @@ gemm_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CU
 
   if (a.splits > 1) {
     // Partial of cluster rank r for chunk c, quarter q: 32 columns x 32 rows
-    // at part + ((tile * S + r) * 8 + c) * 4096 + q * 1024, column-major with
+    // at part + ((tile * S + r) * CPT + c) * 4096 + q * 1024, column-major with
     // the row fastest, so that a warp writes 128 contiguous bytes (one column
     // of its quarter) per store, and each (r, c) partial is 16 KB contiguous.
     const int S = a.splits;
@@ -487,7 +497,7 @@ gemm_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CU
         for (int r = 0; r < S; ++r)
           if (r != rank)
             bulk_load(smem + (size_t)(slot++) * kPartChunkBytes,
-                      tile_part + ((size_t)r * 8 + c) * 4096, kPartChunkBytes, pfull);
+                      tile_part + ((size_t)r * CPT + c) * 4096, kPartChunkBytes, pfull);
     }
     if (epi && !*s_abort) {
       if (!mbar_wait(pfull, 0)) {
