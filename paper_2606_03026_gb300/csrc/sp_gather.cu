@@ -341,10 +341,15 @@ gather_cluster_kernel(const __grid_constant__ GatherParamsT<NP> p) {
   if (blockIdx.y == 0) prefetch_spike_rows(p);   // before the wait: see gather_kernel
   pdl_wait();
 
-  const int j = blockIdx.y;
+  const int c = (int)blockIdx.x / kGatherCluster;
+  const int rank = (int)blockIdx.x - c * kGatherCluster;   // rank in the (6, 1, 1) cluster
+  int j = blockIdx.y, cl = c;
+  if (p.ncl_list > 0) {                     // listed clusters: no idle CTAs
+    const int e = p.cl_list[c];
+    j = e >> 8;
+    cl = e & 0xff;
+  }
   const GatherProblem& P = p.prob[j];
-  const int cl = (int)blockIdx.x / kGatherCluster;
-  const int rank = (int)blockIdx.x - cl * kGatherCluster;  // rank in the (6, 1, 1) cluster
   if (cl >= P.ncl) return;                  // the whole cluster: no tile of this problem
   const int kch = P.kch;
   const int per = (kGatherNT / 4 + kch - 1) / kch;   // most groups owned by one CTA
@@ -422,9 +427,12 @@ int cluster_capacity() {
 
 // Fills the cluster-form fields of q; false when the launch does not fit the
 // cluster form (several tokens, a chunk count above the cluster size, or more
-// clusters than can be resident at once).
+// clusters than can be resident at once).  Up to kGatherMaxClusterList
+// clusters are listed one by one (a 1-D grid of exactly the clusters with
+// work, all resident together); more take a (clusters x 6, problems) grid in
+// which the problems with fewer clusters leave idle CTAs.
 template <int NP>
-bool cluster_form(GatherParamsT<NP>& q, int* grid_x) {
+bool cluster_form(GatherParamsT<NP>& q, int* grid_x, int* grid_y) {
   if (q.B != 1) return false;
   int total = 0, widest = 0;
   for (int j = 0; j < q.nprob; ++j) {
@@ -445,7 +453,18 @@ bool cluster_form(GatherParamsT<NP>& q, int* grid_x) {
     if (P.ncl > widest) widest = P.ncl;
   }
   if (total > cluster_capacity<NP>()) return false;
-  *grid_x = widest * kGatherCluster;
+  q.ncl_list = 0;
+  if (total <= kGatherMaxClusterList && widest <= 0xff) {
+    int c = 0;
+    for (int j = 0; j < q.nprob; ++j)
+      for (int cl = 0; cl < q.prob[j].ncl; ++cl) q.cl_list[c++] = (uint16_t)((j << 8) | cl);
+    q.ncl_list = total;
+    *grid_x = total * kGatherCluster;
+    *grid_y = 1;
+  } else {
+    *grid_x = widest * kGatherCluster;
+    *grid_y = q.nprob;
+  }
   return true;
 }
 
@@ -457,10 +476,10 @@ cudaError_t launch_gather_t(const GatherParamsT<NP>& p, cudaStream_t s) {
   cudaError_t e = set_carveout(gather_cluster_kernel<NP>, carve_c);
   if (e != cudaSuccess) return e;
   GatherParamsT<NP> q = p;
-  int gx = 0;
-  if (cluster_form(q, &gx)) {
+  int gx = 0, gy = 0;
+  if (cluster_form(q, &gx, &gy)) {
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3((unsigned)gx, (unsigned)q.nprob, 1);
+    cfg.gridDim = dim3((unsigned)gx, (unsigned)gy, 1);
     cfg.blockDim = dim3(kGatherClusterThreads, 1, 1);
     cfg.stream = s;
     cudaLaunchAttribute attr[2];

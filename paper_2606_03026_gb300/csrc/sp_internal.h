@@ -56,6 +56,7 @@ constexpr int kGatherCluster = 6;
 constexpr int kGatherClusterWarps = 8;
 constexpr int kGatherClusterThreads = 32 * kGatherClusterWarps;
 constexpr int kGatherClusterMaxCK = 1024;
+constexpr int kGatherMaxClusterList = 256;   // clusters of a launch listed one by one
 
 constexpr int kMaxProblems = SPIKE_PROJ_MAX_GROUP;
 
@@ -77,6 +78,10 @@ struct GatherParamsT {
   int32_t* ws;            // problem j token t: ws + (ws_begin_j*B + t*N_j); the gather kernel adds fp32 into it
   uint32_t* tickets;      // problem j token t tile n: ticket_begin_j*B + t*ntile_j + n
   int* err;
+  // cluster form: cluster c of a 1-D grid is cluster (cl_list[c] & 0xff) of
+  // problem (cl_list[c] >> 8); ncl_list == 0: grid (clusters x 6, problems)
+  int32_t ncl_list;
+  uint16_t cl_list[kGatherMaxClusterList];
 };
 using GatherParams1 = GatherParamsT<1>;
 using GatherParamsG = GatherParamsT<kMaxProblems>;
