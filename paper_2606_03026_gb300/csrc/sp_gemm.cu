@@ -284,6 +284,10 @@ gemm_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CU
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *s_tmem;
+  // The set-up above overlaps the previous kernel of the stream (programmatic
+  // dependent launch); every global access below comes after it has finished.
+  pdl_launch_dependents();
+  pdl_wait();
 
   if (warp == 0) {
     // ------------------------------ TMA producer ------------------------------
@@ -559,6 +563,8 @@ __global__ void w_to_bf16_kernel(const int8_t* __restrict__ W, int64_t ldw, int 
 template <bool kVec>
 __global__ void spikes_to_bf16_kernel(const void* __restrict__ spikes, int fmt, int64_t ld, int T,
                                       int K, int Kp, __nv_bfloat16* __restrict__ Xb) {
+  pdl_launch_dependents();
+  pdl_wait();
   const int per_row = Kp / 16;
   const int64_t total = (int64_t)T * per_row;
   for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < total;
@@ -717,21 +723,22 @@ cudaError_t launch_gemm_t(const CUtensorMap& mapA, const CUtensorMap& mapB, int 
   const size_t smem = gemm_smem<kFusedX>();
   if (S == 1) {
     const int grid = a.units < g_num_sms ? a.units : g_num_sms;
-    gemm_kernel<kFusedX><<<grid, threads, smem, s>>>(mapA, mapB, a);
-    return cudaGetLastError();
+    return launch_pdl(gemm_kernel<kFusedX>, dim3(grid), dim3(threads), smem, s, mapA, mapB, a);
   }
   cudaLaunchConfig_t cfg = {};
-  cudaLaunchAttribute attr;
-  attr.id = cudaLaunchAttributeClusterDimension;
-  attr.val.clusterDim.x = S;
-  attr.val.clusterDim.y = 1;
-  attr.val.clusterDim.z = 1;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = S;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.gridDim = dim3(a.units, 1, 1);
   cfg.blockDim = dim3(threads, 1, 1);
   cfg.dynamicSmemBytes = smem;
   cfg.stream = s;
-  cfg.attrs = &attr;
-  cfg.numAttrs = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 2;
   return cudaLaunchKernelEx(&cfg, gemm_kernel<kFusedX>, mapA, mapB, a);
 }
 
@@ -764,10 +771,10 @@ cudaError_t launch_spikes_to_bf16(const void* spikes, int fmt, int64_t ld, int T
   const bool vec = fmt == SP_SPIKES_U8 && (reinterpret_cast<uintptr_t>(spikes) & 15u) == 0 &&
                    ld % 16 == 0;
   if (vec)
-    spikes_to_bf16_kernel<true><<<(int)blocks, threads, 0, s>>>(spikes, fmt, ld, T, K, Kp, Xb);
-  else
-    spikes_to_bf16_kernel<false><<<(int)blocks, threads, 0, s>>>(spikes, fmt, ld, T, K, Kp, Xb);
-  return cudaGetLastError();
+    return launch_pdl(spikes_to_bf16_kernel<true>, dim3((unsigned)blocks), dim3(threads), 0, s, spikes,
+                      fmt, ld, T, K, Kp, Xb);
+  return launch_pdl(spikes_to_bf16_kernel<false>, dim3((unsigned)blocks), dim3(threads), 0, s, spikes,
+                    fmt, ld, T, K, Kp, Xb);
 }
 
 cudaError_t gemm_make_x8_map(const void* X, int64_t ldx, int T, int K, CUtensorMap* out) {
