@@ -20,9 +20,9 @@ Also reported on the same JSON line:
                measured HBM copy bandwidth; traffic = the DRAM bytes per
                launch that ncu measured for the same kernel source
                (profiles/dram_traffic.json), null when the source differs
-  e2e          the same metric through the host-buffer entry point (spike
-               masks copied in from pinned memory, acc and y copied back,
-               every step)
+  e2e          the same metric through the host-buffer entry point: spike
+               masks read from and acc / y written to page-locked host memory
+               every step (the bytes cross the CPU-GPU link inside the step)
   cpu_baseline the CPU oracle on the host cores, on a bounded sample
   prefill      512-token prefill over 22 blocks on the tensor cores, TOPS
   configs      every workload of the benchmark table, timed outside the
@@ -435,7 +435,9 @@ def run_ours(args):
         "e2e": {"value": e2e_bytes / (e2e_ms * 1e-3) / 1e9, "unit": "GB/s",
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                 "ms_per_step": e2e_ms / e2e_steps,
-                "api": "spike_proj_group_decode_host (pinned host buffers, copies each step)"},
+                "api": "spike_proj_group_decode_host on page-locked host buffers: every step the "
+                       "kernel reads the spike words from and writes acc and y to host memory "
+                       "over the CPU-GPU link"},
         "gpu_launches": steps,
         "clocks": clocks,
     }

@@ -206,11 +206,14 @@ sp_status spike_proj_group_decode(sp_group_t group, const void *spikes,
                                   sp_fmt fmt, int64_t ld_spikes, int32_t *acc,
                                   float *y, int64_t ld_out, sp_stream_t stream);
 
-/* spike_proj_group_decode_host: the same with HOST buffers (page-locked
- * memory recommended).  Enqueues on `stream`: the copy of count rows of
- * spikes into group-owned device staging, the kernel, and the copies of
- * acc / y back to the host.  Returns once enqueued; the host buffers must
- * not be touched until `stream` has been synchronised. */
+/* spike_proj_group_decode_host: the same with HOST buffers.  Page-locked
+ * buffers (cudaHostAlloc, cudaHostRegister, torch pin_memory) are read and
+ * written by the kernel in place, over the CPU-GPU link, with no copy; for
+ * pageable buffers the call enqueues the copy of count rows of spikes into
+ * group-owned device staging, the kernel, and the copies of acc / y back.
+ * Returns once enqueued; the host buffers must not be touched until `stream`
+ * has been synchronised.  Errors as spike_proj_group_decode (SP_EALIGN for a
+ * spike word or output pointer that is not 4-byte aligned). */
 sp_status spike_proj_group_decode_host(sp_group_t group, const void *h_spikes,
                                        sp_fmt fmt, int64_t ld_spikes,
                                        int32_t *h_acc, float *h_y,

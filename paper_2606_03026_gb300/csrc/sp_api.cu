@@ -134,6 +134,17 @@ void group_free(sp_group_s* g) {
   delete g;
 }
 
+// Device address of page-locked host memory that the current device can
+// reach (cudaHostAlloc, cudaHostRegister, torch pin_memory), else nullptr.
+void* device_view(const void* h) {
+  cudaPointerAttributes a;
+  if (cudaPointerGetAttributes(&a, h) != cudaSuccess) {
+    (void)cudaGetLastError();
+    return nullptr;
+  }
+  return a.type == cudaMemoryTypeHost ? a.devicePointer : nullptr;
+}
+
 // Spike / output argument checks shared by the per-plan calls.
 sp_status check_io(const void* spikes, int fmt, const int32_t* acc, const float* y) {
   if (!spikes || !fmt_ok(fmt)) return SP_EINVAL;
@@ -531,19 +542,40 @@ sp_status spike_proj_group_decode_host(sp_group_t g, const void* h_spikes, sp_fm
   if (!g || !h_spikes || !fmt_ok(fmt) || (!h_acc && !h_y)) return SP_EINVAL;
   const int64_t need = row_elems(fmt, g->maxK);
   if (ld_spikes < need || ld_out < g->maxN) return SP_EINVAL;
+  if ((fmt == SP_SPIKES_BITS32 && !aligned(h_spikes, 4)) || (h_acc && !aligned(h_acc, 4)) ||
+      (h_y && !aligned(h_y, 4)))
+    return SP_EALIGN;
   cudaStream_t s = as_stream(stream);
   const size_t elem = fmt == SP_SPIKES_BITS32 ? 4 : 1;
   const size_t row_bytes = (size_t)need * elem;
-  SP_CUDA(cudaMemcpy2DAsync(g->d_spikes, g->spike_row_bytes, h_spikes, (size_t)ld_spikes * elem,
-                            row_bytes, (size_t)g->count, cudaMemcpyHostToDevice, s));
   GatherParamsG& P = g->params;
   P.fmt = fmt;
-  P.spikes = g->d_spikes;
-  P.ld_spikes = (int64_t)(g->spike_row_bytes / elem);
-  P.acc = h_acc ? g->d_acc : nullptr;
-  P.y = h_y ? g->d_y : nullptr;
-  P.ld_out = g->maxN;
+  // Page-locked host buffers are read and written by the kernel in place;
+  // pageable ones go through the group's device staging.
+  const void* m_spikes = device_view(h_spikes);
+  if (m_spikes) {
+    P.spikes = m_spikes;
+    P.ld_spikes = ld_spikes;
+  } else {
+    SP_CUDA(cudaMemcpy2DAsync(g->d_spikes, g->spike_row_bytes, h_spikes, (size_t)ld_spikes * elem,
+                              row_bytes, (size_t)g->count, cudaMemcpyHostToDevice, s));
+    P.spikes = g->d_spikes;
+    P.ld_spikes = (int64_t)(g->spike_row_bytes / elem);
+  }
+  int32_t* m_acc = h_acc ? static_cast<int32_t*>(device_view(h_acc)) : nullptr;
+  float* m_y = h_y ? static_cast<float*>(device_view(h_y)) : nullptr;
+  const bool out_mapped = (!h_acc || m_acc) && (!h_y || m_y);
+  if (out_mapped) {
+    P.acc = m_acc;
+    P.y = m_y;
+    P.ld_out = ld_out;
+  } else {
+    P.acc = h_acc ? g->d_acc : nullptr;
+    P.y = h_y ? g->d_y : nullptr;
+    P.ld_out = g->maxN;
+  }
   SP_CUDA(launch_gather(P, s));
+  if (out_mapped) return SP_OK;
   const size_t out_row = (size_t)g->maxN * 4;
   if (h_acc)
     SP_CUDA(cudaMemcpy2DAsync(h_acc, (size_t)ld_out * 4, g->d_acc, out_row, out_row,

@@ -77,6 +77,28 @@ def test_host_buffer_entry_point(step):
         assert_parity(h_acc, h_y, want_acc, want_y, "host buffers")
 
 
+def test_host_buffer_pageable_and_page_locked(step):
+    """Pageable host buffers go through device staging copies, page-locked
+    ones are read and written in place by the kernel; both give the oracle's
+    bits, with an output row stride wider than N."""
+    weights, plans, group = step
+    xs, bits, u8 = step_inputs(weights, 9)
+    want_acc, want_y = oracle_step(weights, xs)
+    n, ld = len(weights), 1600
+    for locked in (False, True):
+        for fmt, rows in (("bits", bits), ("u8", u8)):
+            h_rows = torch.from_numpy(np.ascontiguousarray(rows))
+            h_acc = torch.full((n, ld), -3, dtype=torch.int32)
+            h_y = torch.full((n, ld), -3.0, dtype=torch.float32)
+            if locked:
+                h_rows, h_acc, h_y = h_rows.pin_memory(), h_acc.pin_memory(), h_y.pin_memory()
+            group.decode_host(h_rows, fmt, rows.shape[1], h_acc, h_y, ld)
+            torch.cuda.synchronize()
+            assert_parity(h_acc[:, :1536], h_y[:, :1536], want_acc, want_y,
+                          f"host buffers locked={locked} {fmt}")
+            assert (h_acc[:, 1536:] == -3).all() and (h_y[:, 1536:] == -3.0).all()
+
+
 def test_mixed_group_shapes():
     """Projections of different N, K and ldw in one group, sparse and dense."""
     cases = [(16, 1), (48, 1000), (1552, 777), (512, 6144), (2048, 33)]
