@@ -218,6 +218,17 @@ __device__ __forceinline__ int4 unit_sum4(const UnitSmem<W, MAXCK, S>& sm, int o
 
 __device__ __forceinline__ void write4(const GatherProblem& P, int32_t* acc_row, float* y_row,
                                        int n, int4 v) {
+  // one 16-byte store each where the rows allow it (the output may also be
+  // page-locked host memory, where every transaction crosses the link)
+  const bool v4 = ((reinterpret_cast<uintptr_t>(acc_row) | reinterpret_cast<uintptr_t>(y_row)) & 15u) == 0;
+  if (v4) {
+    if (acc_row) *reinterpret_cast<int4*>(acc_row + n) = v;
+    if (y_row)
+      *reinterpret_cast<float4*>(y_row + n) =
+          make_float4(scale_out(__ldg(P.scale + n), v.x), scale_out(__ldg(P.scale + n + 1), v.y),
+                      scale_out(__ldg(P.scale + n + 2), v.z), scale_out(__ldg(P.scale + n + 3), v.w));
+    return;
+  }
   if (acc_row) {
     acc_row[n] = v.x;
     acc_row[n + 1] = v.y;
@@ -319,10 +330,11 @@ gather_kernel(const __grid_constant__ GatherParamsT<NP> p) {
 // Cluster form: one token per problem, at most kGatherCluster chunks of at
 // most 1024 columns per tile.  256-thread CTAs in clusters of kGatherCluster;
 // a cluster holds tpc tiles x kch chunks of one problem (rank = tile slot *
-// kch + chunk; kch divides kGatherCluster); grid = (clusters of the largest
-// problem x kGatherCluster, problems).  The 4-channel group g of a tile
-// belongs to the CTA of chunk g % kch: every CTA stores its partial of each
-// group into the owner's shared memory (distributed shared memory), one
+// kch + chunk; kch divides kGatherCluster); the grid lists the clusters one
+// by one (or is (clusters of the largest problem x kGatherCluster,
+// problems)).  The 128 4-channel groups of a tile are split into kch
+// contiguous runs, run c owned by the CTA of chunk c: every CTA stores its
+// partial of each group into the owner's shared memory (distributed shared memory), one
 // cluster barrier (release / acquire) publishes the stores, and each owner
 // adds the kch partials of its groups from its own shared memory and writes
 // acc / y.  No workspace, no atomics, and no CTA reads another's shared
@@ -363,14 +375,15 @@ gather_cluster_kernel(const __grid_constant__ GatherParamsT<NP> p) {
     const int g = threadIdx.x;              // the 4-channel group of this thread
     if (g < kGatherNT / 4) {
       const int4 v = unit_sum4(sm, 4 * g);
-      st_peer_v4((uint32_t)__cvta_generic_to_shared(&s_recv[kc * per + g / kch]),
-                 (uint32_t)(ts * kch + g % kch), v);
+      const int owner = g / per;
+      st_peer_v4((uint32_t)__cvta_generic_to_shared(&s_recv[kc * per + (g - owner * per)]),
+                 (uint32_t)(ts * kch + owner), v);
     }
   }
   cluster_sync_all();                       // every partial is in its owner's shared memory
-  const int g_own = threadIdx.x * kch + kc; // this thread's owned group
+  const int g_own = kc * per + threadIdx.x; // this thread's owned group (a contiguous run)
   const int n = n0 + 4 * g_own;
-  if (work && g_own < kGatherNT / 4 && n < P.N) {
+  if (work && (int)threadIdx.x < per && g_own < kGatherNT / 4 && n < P.N) {
     int4 s = make_int4(0, 0, 0, 0);
     for (int q = 0; q < kch; ++q) {
       const int4 v = s_recv[q * per + threadIdx.x];
