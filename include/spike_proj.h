@@ -13,7 +13,7 @@
  *       at W[k * ldw + m], so each active column is one contiguous read of N
  *       bytes across the output channels (Section 2.2).
  *   s   FP32 scale per output channel, length N (Section 2.3 quantiser).
- *   x   binary spikes, one row per token, in one of two formats (sp_fmt).
+ *   x   binary spikes, one row per token, in one of three formats (sp_fmt).
  *
  * Only the active columns are read on the gather paths; the dense
  * tensor-core path (SP_GEMM) reads all of Q and is chosen only where the
@@ -74,8 +74,20 @@ typedef enum sp_status {
  *                     ignored.  A row holds ceil(K/32) words; row stride
  *                     (ld_spikes) is counted in words.
  *   SP_SPIKES_U8:     one byte per column, any nonzero byte is a spike; row
- *                     stride counted in bytes. */
-typedef enum sp_fmt { SP_SPIKES_BITS32 = 0, SP_SPIKES_U8 = 1 } sp_fmt;
+ *                     stride counted in bytes.
+ *   SP_SPIKES_BOOL8:  one byte per column holding exactly 0 or 1 (the bytes
+ *                     of a C bool array or a torch.bool tensor); row stride
+ *                     counted in bytes.  Every path accepts it; SP_GEMM reads
+ *                     such rows in place when the base is 16-byte aligned and
+ *                     the row stride a multiple of 16 (other formats go
+ *                     through a 0/1 staging pass first).  A byte other than 0
+ *                     or 1 gives an unspecified result on that path (no
+ *                     fault); the gather and union paths treat it as U8. */
+typedef enum sp_fmt {
+    SP_SPIKES_BITS32 = 0,
+    SP_SPIKES_U8 = 1,
+    SP_SPIKES_BOOL8 = 2
+} sp_fmt;
 
 /* Kernel strategies for multi-token calls.
  *   SP_AUTO    count the active spikes on the device, read the count back
@@ -85,10 +97,11 @@ typedef enum sp_fmt { SP_SPIKES_BITS32 = 0, SP_SPIKES_U8 = 1 } sp_fmt;
  *   SP_GATHER  per-token active-column gather (the batch-1 kernel per row).
  *   SP_UNION   one fetch of each column in the union of the rows' active sets,
  *              added into every row whose spike is set.
- *   SP_GEMM    dense tensor-core contraction over all columns (tcgen05,
- *              bf16 operands holding the exact integers, fp32 accumulation
- *              in tensor memory: exact because every partial sum is an
- *              integer below 2^24). */
+ *   SP_GEMM    dense tensor-core contraction over all columns (tcgen05
+ *              e4m3 x e4m3 with fp32 accumulation in tensor memory: spike
+ *              bytes 0 / 1 read as 0 and 2^-9, each weight split into two
+ *              e4m3-exact planes 16 h + l; exact because every partial sum
+ *              is a multiple of 2^-9 with at most 24 significant bits). */
 typedef enum sp_kernel {
     SP_AUTO = 0,
     SP_GATHER = 1,
@@ -98,7 +111,8 @@ typedef enum sp_kernel {
 
 /* Plan flags. */
 #define SP_PLAN_GEMM 0x1u  /* also build the tensor-core operand copy of W:
-                              N*K bf16 (2 bytes per weight), owned by the plan */
+                              two e4m3 planes, 2*N*Kp bytes (Kp = K rounded up
+                              to a multiple of 64), owned by the plan */
 
 /* ---------------------------------------------------------------------------
  * spike_proj_plan -- describe one projection and allocate its workspace.
@@ -115,7 +129,8 @@ typedef enum sp_kernel {
  *   K          input columns, 1 <= K <= SPIKE_PROJ_MAX_K (else SP_ERANGE).
  *   max_batch  largest B / T accepted by spike_proj_batched / _prefill on this
  *              plan (>= 1; sizes the workspace: 4*N*max_batch bytes, plus
- *              2*K*max_batch with SP_PLAN_GEMM).
+ *              Kp*ceil(max_batch/128)*128 bytes of 0/1 spike staging with
+ *              SP_PLAN_GEMM).
  *   flags      0 or SP_PLAN_GEMM.
  *   stream     used for the workspace clear and the operand copy; the call
  *              synchronises it before returning.
@@ -145,7 +160,8 @@ sp_status spike_proj_decode(sp_plan_t plan, const void *spikes, sp_fmt fmt,
  * spike_proj_batched -- B independent spike rows sharing the plan's W.
  *
  *   spikes     device, B rows, row b at spikes + b*ld_spikes (words for
- *              BITS32, bytes for U8); ld_spikes >= ceil(K/32) or >= K.
+ *              BITS32, bytes for U8 and BOOL8); ld_spikes >= ceil(K/32) or
+ *              >= K.
  *   B          1 <= B <= plan's max_batch (else SP_ERANGE).
  *   acc, y     device [B][N] row-major (either may be NULL, not both).
  *   strategy   SP_AUTO, SP_GATHER, SP_UNION or SP_GEMM (SP_GEMM needs a plan
@@ -198,7 +214,7 @@ sp_status spike_proj_group_create(sp_group_t *group, const sp_plan_t *plans,
 sp_status spike_proj_group_destroy(sp_group_t group);
 
 /* spike_proj_group_decode: projection j reads its spike row at
- *   spikes + j*ld_spikes   (words for BITS32, bytes for U8)
+ *   spikes + j*ld_spikes   (words for BITS32, bytes for U8 and BOOL8)
  * and writes acc + j*ld_out, y + j*ld_out (device; either may be NULL, not
  * both).  ld_spikes must cover the largest K of the group; ld_out >= the
  * largest N. */

@@ -36,15 +36,15 @@ struct sp_plan_s {
   int32_t* d_counts = nullptr;    // density probe result [2]
   int32_t* h_counts = nullptr;    // page-locked copy
   // tensor-core path
-  __nv_bfloat16* Wb = nullptr;    // [N][Kp] bf16 K-major
-  __nv_bfloat16* Xb = nullptr;    // [xb_rows][Kp] bf16 spike staging
+  uint8_t* Wq = nullptr;          // [N][2 Kp] e4m3 weight planes (16 h, l)
+  uint8_t* Xs = nullptr;          // [xs_rows][Kp] 0/1 spike staging
   float* part = nullptr;          // split-K partials, part_units x 128 x 256 fp32
-  int Kp = 0, xb_rows = 0, part_units = 0;
+  int Kp = 0, xs_rows = 0, part_units = 0;
   GemmMaps maps;
-  CUtensorMap x8map;              // u8 spike rows of the last fused call
-  const void* x8_ptr = nullptr;
-  int64_t x8_ld = 0;
-  int32_t x8_T = 0;
+  CUtensorMap rows_map;           // caller's 0/1 rows of the last in-place call
+  const void* rows_ptr = nullptr;
+  int64_t rows_ld = 0;
+  int32_t rows_T = 0;
   sp_kernel last_kernel = SP_AUTO;
   int32_t last_active = -1;
 };
@@ -84,7 +84,9 @@ inline bool aligned(const void* p, uintptr_t a) {
 inline cudaStream_t as_stream(sp_stream_t s) { return reinterpret_cast<cudaStream_t>(s); }
 inline int64_t words_for(int K) { return ((int64_t)K + 31) / 32; }
 inline int64_t row_elems(sp_fmt fmt, int K) { return fmt == SP_SPIKES_BITS32 ? words_for(K) : K; }
-inline bool fmt_ok(int fmt) { return fmt == SP_SPIKES_BITS32 || fmt == SP_SPIKES_U8; }
+inline bool fmt_ok(int fmt) {
+  return fmt == SP_SPIKES_BITS32 || fmt == SP_SPIKES_U8 || fmt == SP_SPIKES_BOOL8;
+}
 
 sp_status check_device(int* dev_out) {
   int dev = 0, major = 0, minor = 0;
@@ -117,8 +119,8 @@ void plan_free(sp_plan_s* p) {
   cudaFree(p->err);
   cudaFree(p->d_counts);
   if (p->h_counts) cudaFreeHost(p->h_counts);
-  cudaFree(p->Wb);
-  cudaFree(p->Xb);
+  cudaFree(p->Wq);
+  cudaFree(p->Xs);
   cudaFree(p->part);
   delete p;
 }
@@ -214,24 +216,19 @@ sp_status run_union(sp_plan_s* p, const void* spikes, int fmt, int B, int64_t ld
 sp_status run_gemm(sp_plan_s* p, const void* spikes, int fmt, int T, int64_t ld, int32_t* acc,
                    float* y, cudaStream_t s) {
   if (!(p->flags & SP_PLAN_GEMM)) return SP_EUNSUPPORTED;
-  // u8 rows that TMA can read directly are converted inside the GEMM kernel
-  // when K is split (the fused form's shape); anything else goes through the
-  // bf16 staging copy first
-  bool fused = fmt == SP_SPIKES_U8 && aligned(spikes, 16) && ld % 16 == 0;
-  int S = gemm_splits(fused, T, p->N, p->Kp, p->part_units);
-  if (fused && S < 2) {
-    fused = false;
-    S = gemm_splits(false, T, p->N, p->Kp, p->part_units);
-  }
-  if (fused) {
-    if (spikes != p->x8_ptr || ld != p->x8_ld || T != p->x8_T) {
-      SP_CUDA(gemm_make_x8_map(spikes, ld, T, p->K, &p->x8map));
-      p->x8_ptr = spikes;
-      p->x8_ld = ld;
-      p->x8_T = T;
+  // 0/1 byte rows that TMA can address are the MMA's spike operand as they
+  // stand; any other input is first written as 0/1 bytes into the staging copy
+  const bool in_place = fmt == SP_SPIKES_BOOL8 && aligned(spikes, 16) && ld % 16 == 0;
+  const int S = gemm_splits(T, p->N, p->Kp, p->part_units);
+  if (in_place) {
+    if (spikes != p->rows_ptr || ld != p->rows_ld || T != p->rows_T) {
+      SP_CUDA(gemm_make_rows_map(spikes, ld, T, p->K, &p->rows_map));
+      p->rows_ptr = spikes;
+      p->rows_ld = ld;
+      p->rows_T = T;
     }
   } else {
-    SP_CUDA(launch_spikes_to_bf16(spikes, fmt, ld, T, p->K, p->Kp, p->Xb, s));
+    SP_CUDA(launch_spikes_to_01(spikes, fmt, ld, T, p->K, p->Kp, p->Xs, s));
   }
   GemmParams g;
   g.scale = p->scale;
@@ -243,7 +240,7 @@ sp_status run_gemm(sp_plan_s* p, const void* spikes, int fmt, int T, int64_t ld,
   g.err = p->err;
   g.part = p->part;
   g.part_units = p->part_units;
-  SP_CUDA(launch_gemm(fused ? p->x8map : p->maps.a, p->maps.b, fused, S, T, p->N, p->Kp, g, s));
+  SP_CUDA(launch_gemm(in_place ? p->rows_map : p->maps.a, p->maps.b, S, T, p->N, p->Kp, g, s));
   return SP_OK;
 }
 
@@ -360,7 +357,7 @@ sp_status spike_proj_plan(sp_plan_t* plan, const int8_t* W, int64_t ldw, const f
   }
   if (flags & SP_PLAN_GEMM) {
     p->Kp = gemm_k_pad(K);
-    p->xb_rows = ceil_div(max_batch, 128) * 128;
+    p->xs_rows = ceil_div(max_batch, 128) * 128;
     // a split-K launch has at most one unit per SM
     int sms = 0;
     e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
@@ -369,14 +366,14 @@ sp_status spike_proj_plan(sp_plan_t* plan, const int8_t* W, int64_t ldw, const f
       return cuda_fail(e);
     }
     p->part_units = sms;
-    if ((st = dev_alloc_zero(&p->Wb, (size_t)N * p->Kp, s)) != SP_OK ||
-        (st = dev_alloc_zero(&p->Xb, (size_t)p->xb_rows * p->Kp, s)) != SP_OK ||
+    if ((st = dev_alloc_zero(&p->Wq, (size_t)2 * N * p->Kp, s)) != SP_OK ||
+        (st = dev_alloc_zero(&p->Xs, (size_t)p->xs_rows * p->Kp, s)) != SP_OK ||
         (st = dev_alloc_zero(&p->part, (size_t)p->part_units * kGemmPartialElems, s)) != SP_OK) {
       plan_free(p);
       return st;
     }
-    e = launch_w_to_bf16(W, ldw, N, K, p->Wb, s);
-    if (e == cudaSuccess) e = gemm_make_maps(p->Xb, p->xb_rows, p->Wb, N, p->Kp, &p->maps);
+    e = launch_w_to_e4m3(W, ldw, N, K, p->Wq, s);
+    if (e == cudaSuccess) e = gemm_make_maps(p->Xs, p->xs_rows, p->Wq, N, p->Kp, &p->maps);
     if (e != cudaSuccess) {
       plan_free(p);
       return cuda_fail(e);

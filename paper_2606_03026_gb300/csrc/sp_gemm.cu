@@ -5,23 +5,35 @@
 // i.e. Eq. (sparse) for every row of a dense spike matrix (prompt prefill).
 //
 // The 5th-generation tensor cores of sm_103a have no integer MMA
-// (ptxas rejects tcgen05.mma .kind::i8 for this target), so the contraction
-// runs as tcgen05.mma .kind::f16 with bf16 operands and fp32 accumulation in
-// tensor memory.  It is exact: spikes 0/1 and weights in [-128, 127] are bf16
-// integers, every product is an integer, and every partial sum is an integer
-// of magnitude <= 128 * K < 2^24, so no fp32 addition ever rounds.  The
-// epilogue converts the accumulator to INT32 without loss.
+// (ptxas rejects tcgen05.mma .kind::i8 for this target).  The contraction runs
+// as tcgen05.mma .kind::f8f6f4 with both operands e4m3 and fp32 accumulation
+// in tensor memory, and it is exact:
+//   * spikes are bytes 0 / 1, which e4m3 reads as 0 and 2^-9 (its smallest
+//     subnormal), so a 0/1 spike matrix is an MMA operand as it stands;
+//   * a weight w in [-128, 127] is split as w = 16 h + l, h = floor(w / 16) in
+//     [-8, 7], l in [0, 15].  16 h and l have at most four significant bits
+//     and |16 h| <= 128, so both are e4m3 values exactly.  The weight operand
+//     holds the two planes side by side along K, and every K step issues one
+//     MMA per plane into the same accumulator;
+//   * every product is a multiple of 2^-9 and every partial sum n 2^-9 with
+//     |n| <= 128 K <= 2^24 (K <= 2^17): an fp32 value, so no addition
+//     rounds.  The epilogue scales by 2^9 (exact) and converts to INT32.
+// An fp8 MMA runs at twice the bf16 rate, so the two planes take the time of
+// one bf16 MMA, while the spike operand is one byte per element and needs no
+// conversion pass.
 //
-// Kernel structure:
-//   warp 0      TMA producer: 128x64 (X) and 256x64 (W) bf16 boxes, 128-byte
-//               swizzle, into a 4-stage shared-memory ring (mbarriers)
-//   warp 1      allocates 512 TMEM columns (two 128x256 fp32 accumulators) and
-//               issues tcgen05.mma (M=128, N=256, K=16) from one thread;
-//               tcgen05.commit frees ring slots and publishes accumulators
+// Kernel structure (192 threads):
+//   warp 0      TMA producer: per 64-column K block, a 128 x 64 spike box
+//               (64-byte swizzle) and a 256 x 128 weight box (both planes,
+//               128-byte swizzle) into a 5-stage shared-memory ring
+//   warp 1      allocates 512 TMEM columns (two 128 x 256 fp32 accumulators)
+//               and issues tcgen05.mma (M = 128, N = 256, K = 32) from one
+//               thread; tcgen05.commit frees ring slots and publishes
+//               accumulators
 //   warps 2-5   epilogue: warp w reads TMEM lane quarter w % 4 (32 rows),
 //               32 columns per tcgen05.ld
 // Whole K (enough output tiles for every SM): one CTA per SM, persistent over
-// 128x256 tiles; the epilogue of one tile overlaps the next tile's MMAs
+// 128 x 256 tiles; the epilogue of one tile overlaps the next tile's MMAs
 // (double-buffered accumulator) and writes acc / y through a shared-memory
 // transpose so that every store covers 128 contiguous bytes of a row.
 // Split K (few output tiles, e.g. T = 512 rows give 4 x 6 tiles for N =
@@ -44,53 +56,41 @@
 namespace sp {
 namespace {
 
-constexpr int BM = 128, BN = 256, BK = 64, STAGES = 4;
+constexpr int BM = 128, BN = 256, BK = 64, STAGES = 5;
 constexpr int CPT = BN / 32;                  // 32-column chunks per output tile
-constexpr int A_BYTES = BM * BK * 2;          // 16 KB
-constexpr int B_BYTES = BN * BK * 2;          // 32 KB
+constexpr int A_BYTES = BM * BK;              // 8 KB: 0/1 spike bytes
+constexpr int B_BYTES = BN * BK * 2;          // 32 KB: the 16h and l planes
 constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
 constexpr int TMEM_COLS = 2 * BN;             // double-buffered accumulator
 constexpr int kGemmThreads = 192;             // TMA, MMA and 4 epilogue warps
-constexpr int kConvThreads = 256;             // 8 warps converting u8 spikes to bf16
-constexpr int kGemmThreadsFused = kGemmThreads + kConvThreads;
-constexpr int X8_BYTES = BM * BK;             // one u8 spike tile (8 KB)
 constexpr int TR_STRIDE = 33;                 // padded transpose rows (words)
 constexpr size_t SMEM_RING = (size_t)STAGES * STAGE_BYTES;
 constexpr size_t SMEM_TR = (size_t)4 * 32 * TR_STRIDE * 4;
-constexpr size_t SMEM_X8 = (size_t)STAGES * X8_BYTES;   // u8 spike ring (fused form)
 constexpr size_t SMEM_BARS = 256;
-// Past the operand ring: the epilogue transpose buffer, or in the fused form
-// the u8 spike ring, which the transpose buffer reuses once the K loop is done
-// (the fused form always splits K, so its epilogue runs after the K loop).
-template <bool kFusedX>
-__host__ __device__ constexpr size_t gemm_smem_extra() {
-  return kFusedX ? SMEM_X8 : SMEM_TR;
-}
-template <bool kFusedX>
-__host__ __device__ constexpr size_t gemm_smem() {
-  return 1024 + SMEM_RING + gemm_smem_extra<kFusedX>() + SMEM_BARS;
-}
-static_assert(SMEM_X8 >= SMEM_TR, "the transpose buffer fits the idle u8 ring");
-static_assert(gemm_smem<true>() <= 227 * 1024, "shared memory of the fused form");
+constexpr size_t kGemmSmem = 1024 + SMEM_RING + SMEM_TR + SMEM_BARS;
+static_assert(kGemmSmem <= 227 * 1024, "shared memory per CTA");
+// accumulator units per spike: e4m3 0x01 = 2^-9
+constexpr float kUnitsPerSpike = 512.f;
 
-// Shared-memory matrix descriptor (tcgen05 format): K-major operand whose rows
-// are 128 bytes (64 bf16) laid out by TMA with the 128-byte swizzle; 8-row
-// groups are 1024 bytes apart (stride byte offset).  Stage buffers are
-// 1024-byte aligned, so the base-offset field is 0.  Advancing K by 16
-// elements inside the swizzle atom adds 32 bytes to the start address.
-__device__ __forceinline__ uint64_t smem_desc_k128(const void* p) {
+// Shared-memory matrix descriptors (tcgen05 format) of K-major operands laid
+// out by TMA with a swizzle: rows of 128 bytes (128-byte swizzle, 8-row groups
+// 1024 bytes apart) or of 64 bytes (64-byte swizzle, 8-row groups 512 bytes
+// apart).  Stage buffers are 1024-byte aligned, so the base-offset field is 0.
+// Advancing K by 32 e4m3 elements inside a swizzle row adds 32 bytes to the
+// start address.
+__device__ __forceinline__ uint64_t smem_desc(const void* p, uint32_t group_bytes, uint64_t mode) {
   const uint64_t addr = smem_u32(p);
   uint64_t d = (addr >> 4) & 0x3FFFull;    // start address
   d |= (uint64_t)1 << 16;                  // leading byte offset (unused here)
-  d |= (uint64_t)(1024 >> 4) << 32;        // stride byte offset
+  d |= (uint64_t)(group_bytes >> 4) << 32; // stride byte offset
   d |= (uint64_t)1 << 46;                  // descriptor version for tcgen05
-  d |= (uint64_t)2 << 61;                  // 128-byte swizzle
+  d |= mode << 61;                         // swizzle mode
   return d;
 }
-// Instruction descriptor, kind::f16: D fp32, A and B bf16, both K-major,
-// N = 256, M = 128.
-constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(BN >> 3) << 17) |
-                            ((uint32_t)(BM >> 4) << 24);
+constexpr uint64_t kSwizzle128 = 2, kSwizzle64 = 4;
+// Instruction descriptor, kind::f8f6f4: D fp32, A and B e4m3 (format 0), both
+// K-major, N = 256, M = 128.
+constexpr uint32_t kIdesc = (1u << 4) | ((uint32_t)(BN >> 3) << 17) | ((uint32_t)(BM >> 4) << 24);
 
 __device__ __forceinline__ uint32_t cluster_ctarank() {
   uint32_t r;
@@ -142,10 +142,10 @@ __device__ __forceinline__ float column_scale(const GemmParams& p, int n) {
   return (p.y && n < p.N) ? __ldg(p.scale + n) : 0.f;
 }
 
-// One warp writes a 32-row x 32-column chunk of integer-valued fp32 sums
-// (v[i] = column col0 + i of row row0 + lane): transposed through shared
+// One warp writes a 32-row x 32-column chunk of fp32 sums in accumulator
+// units (v[i] = column col0 + i of row row0 + lane): transposed through shared
 // memory so that each store instruction covers 32 consecutive columns of one
-// row; acc = exact int conversion, y = s * float(acc) with sc = the scale of
+// row; acc = the exact integer, y = s * float(acc) with sc = the scale of
 // column col0 + lane.
 __device__ __forceinline__ void store_chunk(const GemmParams& p, uint32_t* tr,
                                             const uint32_t (&v)[32], int row0, int col0,
@@ -163,13 +163,13 @@ __device__ __forceinline__ void store_chunk(const GemmParams& p, uint32_t* tr,
       // full chunk: unrolled, so the 32 shared-memory reads are in flight together
 #pragma unroll
       for (int rr = 0; rr < 32; ++rr) {
-        const int val = __float2int_rn(__uint_as_float(tr[rr * TR_STRIDE + lane]));
+        const int val = __float2int_rn(__uint_as_float(tr[rr * TR_STRIDE + lane]) * kUnitsPerSpike);
         if (acc) acc[(int64_t)rr * p.N] = val;
         if (y) y[(int64_t)rr * p.N] = scale_out(sc, val);
       }
     } else {
       for (int rr = 0; rr < nrows; ++rr) {
-        const int val = __float2int_rn(__uint_as_float(tr[rr * TR_STRIDE + lane]));
+        const int val = __float2int_rn(__uint_as_float(tr[rr * TR_STRIDE + lane]) * kUnitsPerSpike);
         if (acc) acc[(int64_t)rr * p.N] = val;
         if (y) y[(int64_t)rr * p.N] = scale_out(sc, val);
       }
@@ -178,81 +178,23 @@ __device__ __forceinline__ void store_chunk(const GemmParams& p, uint32_t* tr,
   __syncwarp();
 }
 
-// One u8 spike tile (128 rows x 64 columns, 64-byte rows, TMA-loaded into
-// the u8 ring) -> the A slot's bf16 0/1 tile in the 128-byte-swizzle layout
-// the MMA descriptor expects (16-byte chunk j of row r at
-// r * 128 + (j ^ (r % 8)) * 16).  Item i = (row i / 8, chunk i % 8): 8 u8
-// bytes in, one 16-byte bf16 chunk out; thread t converts items t, t + 256,
-// t + 512, t + 768, so every 8 consecutive threads read 64 contiguous bytes
-// and write one whole 128-byte row (no shared-memory bank conflicts).
-// Split in two so that the u8 slot can be released between them.
-constexpr int kConvItems = BM * 8 / kConvThreads;   // 4
-
-__device__ __forceinline__ void convert_x8_load(const uint8_t* x8, int t, uint4 (&o)[kConvItems]) {
-  uint2 u[kConvItems];
-#pragma unroll
-  for (int k = 0; k < kConvItems; ++k) {
-    const int i = t + k * kConvThreads;
-    u[k] = *reinterpret_cast<const uint2*>(x8 + (i >> 3) * BK + (i & 7) * 8);
-  }
-#pragma unroll
-  for (int k = 0; k < kConvItems; ++k) {
-    uint32_t w[4];
-#pragma unroll
-    for (int e = 0; e < 2; ++e) {
-      const uint32_t v = e ? u[k].y : u[k].x;
-      // 0x80 in every nonzero byte (the low byte of bf16 1.0 = 0x3f80), 0 elsewhere
-      const uint32_t lo = (((v & 0x7f7f7f7fu) + 0x7f7f7f7fu) | v) & 0x80808080u;
-      const uint32_t hi = (lo >> 7) * 0x3fu;
-      w[2 * e] = __byte_perm(lo, hi, 0x5140);
-      w[2 * e + 1] = __byte_perm(lo, hi, 0x7362);
-    }
-    o[k] = make_uint4(w[0], w[1], w[2], w[3]);
-  }
-}
-
-__device__ __forceinline__ void convert_x8_store(uint8_t* slot, int t, const uint4 (&o)[kConvItems]) {
-#pragma unroll
-  for (int k = 0; k < kConvItems; ++k) {
-    const int i = t + k * kConvThreads;
-    const int r = i >> 3, j = i & 7;
-    *reinterpret_cast<uint4*>(slot + r * 128 + ((j ^ (r & 7)) << 4)) = o[k];
-  }
-}
-
-// kFusedX: operand A is u8 spikes instead of the bf16 staging copy.  Lane 1
-// of the TMA warp streams the u8 tiles into their own ring; warps 6-13 read
-// and convert each tile into registers, hand the u8 slot back at once (so
-// the u8 stream runs up to two rings ahead of the tensor core), and write
-// the bf16 tile into its A slot as soon as the MMA has released that slot.
-// The fused form is launched with split K only (its epilogue transpose
-// buffer is the idle u8 ring).
-template <bool kFusedX>
-__global__ void __launch_bounds__(kFusedX ? kGemmThreadsFused : kGemmThreads, 1)
+__global__ void __launch_bounds__(kGemmThreads, 1)
 gemm_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CUtensorMap mapB,
             const __grid_constant__ GemmArgs a) {
-  if (kFusedX && a.splits < 2) {            // launch error: nothing has started yet
-    if (threadIdx.x == 0) atomicExch(a.p.err, kErrBadUnit);
-    return;
-  }
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
   uint8_t* sA = smem;
   uint8_t* sB = smem + (size_t)STAGES * A_BYTES;
   uint32_t* s_tr = reinterpret_cast<uint32_t*>(smem + SMEM_RING);
-  uint8_t* sX8 = smem + SMEM_RING;          // fused form: u8 spike ring (aliases s_tr)
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + SMEM_RING + gemm_smem_extra<kFusedX>());
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + SMEM_RING + SMEM_TR);
   uint64_t* full = bars;                 // [STAGES] TMA -> MMA
   uint64_t* empty = bars + STAGES;       // [STAGES] MMA -> TMA
   uint64_t* tfull = bars + 2 * STAGES;   // [2] MMA -> epilogue
   uint64_t* tempty = tfull + 2;          // [2] epilogue -> MMA
   uint64_t* done = tempty + 2;           // all MMAs retired
   uint64_t* pfull = done + 1;            // split K: peers' partials landed
-  uint64_t* conv = pfull + 1;            // [STAGES] converted A tile ready (fused)
-  uint64_t* full8 = conv + STAGES;       // [STAGES] u8 tile landed (fused)
-  uint64_t* empty8 = full8 + STAGES;     // [STAGES] u8 slot consumed (fused)
-  uint32_t* s_tmem = reinterpret_cast<uint32_t*>(empty8 + STAGES);
+  uint32_t* s_tmem = reinterpret_cast<uint32_t*>(pfull + 1);
   volatile int* s_abort = reinterpret_cast<volatile int*>(s_tmem + 1);
 
   const int warp = threadIdx.x >> 5;
@@ -269,11 +211,6 @@ gemm_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CU
     }
     mbar_init(done, 1);
     mbar_init(pfull, 1);
-    for (int s = 0; s < STAGES; ++s) {
-      mbar_init(&conv[s], kConvThreads / 32);     // one arrive per converter warp
-      mbar_init(&full8[s], 1);
-      mbar_init(&empty8[s], kConvThreads / 32);
-    }
     *s_abort = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     tma_prefetch_desc(&mapA);
@@ -291,11 +228,7 @@ gemm_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CU
 
   if (warp == 0) {
     // ------------------------------ TMA producer ------------------------------
-    // lane 0: the W tiles (and the bf16 A tiles); lane 1 (fused): the u8 tiles
-    if (lane == 0 || (kFusedX && lane == 1)) {
-      const bool x8 = lane == 1;
-      uint64_t* fb = x8 ? full8 : full;
-      uint64_t* eb = x8 ? empty8 : empty;
+    if (lane == 0) {
       int stage = 0;
       uint32_t ph = 0;
       int issued = 0;                       // ring slots filled, for the drain
@@ -303,21 +236,14 @@ gemm_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CU
         int tile, mb, nb, kb0, kb1;
         unit_coords(a, u, tile, mb, nb, kb0, kb1);
         for (int kb = kb0; kb < kb1; ++kb) {
-          if (!mbar_wait(&eb[stage], ph ^ 1u)) {
+          if (!mbar_wait(&empty[stage], ph ^ 1u)) {
             *s_abort = 1;
             atomicExch(a.p.err, kErrMbarTimeout);
             break;
           }
-          if (x8) {
-            mbar_arrive_expect_tx(&fb[stage], X8_BYTES);
-            tma_load_2d(sX8 + (size_t)stage * X8_BYTES, &mapA, &fb[stage], kb * BK, mb * BM);
-          } else if (kFusedX) {
-            mbar_arrive_expect_tx(&fb[stage], B_BYTES);
-          } else {
-            mbar_arrive_expect_tx(&fb[stage], STAGE_BYTES);
-            tma_load_2d(sA + (size_t)stage * A_BYTES, &mapA, &fb[stage], kb * BK, mb * BM);
-          }
-          if (!x8) tma_load_2d(sB + (size_t)stage * B_BYTES, &mapB, &fb[stage], kb * BK, nb * BN);
+          mbar_arrive_expect_tx(&full[stage], STAGE_BYTES);
+          tma_load_2d(sA + (size_t)stage * A_BYTES, &mapA, &full[stage], kb * BK, mb * BM);
+          tma_load_2d(sB + (size_t)stage * B_BYTES, &mapB, &full[stage], kb * 2 * BK, nb * BN);
           ++issued;
           if (++stage == STAGES) { stage = 0; ph ^= 1u; }
         }
@@ -328,7 +254,7 @@ gemm_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CU
       uint32_t q = ph;
       for (int i = 0; i < STAGES && i < issued; ++i) {
         if (--s < 0) { s = STAGES - 1; q ^= 1u; }
-        mbar_wait(&fb[s], q);
+        mbar_wait(&full[s], q);
       }
     }
   } else if (warp == 1) {
@@ -350,16 +276,20 @@ gemm_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CU
         const uint32_t d = tmem_base + (uint32_t)(ab * BN);
         bool ok = true;
         for (int kb = kb0; kb < kb1; ++kb) {
-          if (!mbar_wait(&full[stage], ph) || (kFusedX && !mbar_wait(&conv[stage], ph))) {
+          if (!mbar_wait(&full[stage], ph)) {
             ok = false;
             break;
           }
           tc_fence_after();
-          const uint64_t ad = smem_desc_k128(sA + (size_t)stage * A_BYTES);
-          const uint64_t bd = smem_desc_k128(sB + (size_t)stage * B_BYTES);
+          const uint64_t ad = smem_desc(sA + (size_t)stage * A_BYTES, 512, kSwizzle64);
+          const uint64_t bd = smem_desc(sB + (size_t)stage * B_BYTES, 1024, kSwizzle128);
+          // descriptor addresses count 16-byte units: +2 = 32 bytes (next 32
+          // K elements), +4 = 64 bytes (the l plane of the weight row)
 #pragma unroll
-          for (int k = 0; k < BK / 16; ++k)
-            mma_bf16(d, ad + 2u * k, bd + 2u * k, kIdesc, (kb > kb0 || k > 0) ? 1u : 0u);
+          for (int k = 0; k < BK / 32; ++k) {
+            mma_e4m3(d, ad + 2u * k, bd + 2u * k, kIdesc, (kb > kb0 || k > 0) ? 1u : 0u);
+            mma_e4m3(d, ad + 2u * k, bd + 4u + 2u * k, kIdesc, 1u);
+          }
           mma_commit(&empty[stage]);
           if (++stage == STAGES) { stage = 0; ph ^= 1u; }
         }
@@ -373,45 +303,6 @@ gemm_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CU
       }
       mma_commit(done);                      // retire every issued MMA
       mbar_wait(done, 0);
-    }
-  } else if (kFusedX && warp >= 6) {
-    // ------------------------- spike converters (fused) -----------------------
-    // Same (unit, K block) sequence as the producer: once the u8 tile has
-    // landed and the MMA has released the A slot, expand the tile into the
-    // slot, make the writes visible to the tensor core (async proxy), and
-    // release the A slot to the MMA warp and the u8 slot to the producer.
-    const int ct = threadIdx.x - kGemmThreads;   // 0 .. kConvThreads - 1
-    int stage = 0;
-    uint32_t ph = 0;
-    bool ok = true;
-    for (int u = blockIdx.x; u < a.units && ok; u += gridDim.x) {
-      int tile, mb, nb, kb0, kb1;
-      unit_coords(a, u, tile, mb, nb, kb0, kb1);
-      for (int kb = kb0; kb < kb1; ++kb) {
-        if (*s_abort || !mbar_wait(&full8[stage], ph)) {
-          *s_abort = 1;
-          if (lane == 0) atomicExch(a.p.err, kErrMbarTimeout);
-          ok = false;
-          break;
-        }
-        // the converted tile is in registers (it depends on every u8 load),
-        // so the u8 slot goes back to the producer before the A slot is free
-        uint4 o[kConvItems];
-        convert_x8_load(sX8 + (size_t)stage * X8_BYTES, ct, o);
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&empty8[stage]);
-        if (!mbar_wait(&empty[stage], ph ^ 1u)) {
-          *s_abort = 1;
-          if (lane == 0) atomicExch(a.p.err, kErrMbarTimeout);
-          ok = false;
-          break;
-        }
-        convert_x8_store(sA + (size_t)stage * A_BYTES, ct, o);
-        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&conv[stage]);
-        if (++stage == STAGES) { stage = 0; ph ^= 1u; }
-      }
     }
   } else if (a.splits == 1) {
     // ------------------------------ epilogue (whole K) ------------------------
@@ -460,7 +351,7 @@ gemm_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CU
     // of its quarter) per store, and each (r, c) partial is 16 KB contiguous.
     const int S = a.splits;
     const int rank = (int)cluster_ctarank();
-    const bool epi = warp >= 2 && warp < 6;
+    const bool epi = warp >= 2;
     const int q = warp & 3;
     int tile, mb, nb, kb0, kb1;
     unit_coords(a, blockIdx.x, tile, mb, nb, kb0, kb1);
@@ -538,10 +429,23 @@ gemm_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CU
 
 // ---- operand preparation ------------------------------------------------------
 
-// W column-major INT8 [K][ldw] -> bf16 K-major [N][Kp] (zero for k >= K):
-// 32x32 tiles transposed through shared memory.
-__global__ void w_to_bf16_kernel(const int8_t* __restrict__ W, int64_t ldw, int N, int K, int Kp,
-                                 __nv_bfloat16* __restrict__ Wb) {
+// e4m3 encoding (1 sign bit, 4 exponent bits with bias 7, 3 mantissa bits) of
+// an integer v with at most four significant bits and |v| <= 448 (exact).
+__device__ __forceinline__ uint8_t e4m3_of_small_int(int v) {
+  if (v == 0) return 0;
+  const uint32_t sign = v < 0 ? 0x80u : 0u;
+  const uint32_t m = (uint32_t)(v < 0 ? -v : v);
+  const int e = 31 - __clz((int)m);                    // 2^e <= m < 2^(e+1)
+  const uint32_t frac = ((m << 3) >> e) & 7u;          // the three bits below the leading one
+  return (uint8_t)(sign | (uint32_t)(e + 7) << 3 | frac);
+}
+
+// W column-major INT8 [K][ldw] -> the weight operand [N][2 Kp] bytes: for
+// every 64-column K block, 64 bytes of e4m3(16 h) then 64 bytes of e4m3(l),
+// w = 16 h + l (zero for k >= K).  32 x 32 tiles transposed through shared
+// memory.
+__global__ void w_to_e4m3_kernel(const int8_t* __restrict__ W, int64_t ldw, int N, int K, int Kp,
+                                 uint8_t* __restrict__ Wq) {
   __shared__ int8_t tile[32][33];
   const int k0 = blockIdx.x * 32, m0 = blockIdx.y * 32;
   const int tx = threadIdx.x, ty = threadIdx.y;     // 32 x 8
@@ -552,17 +456,23 @@ __global__ void w_to_bf16_kernel(const int8_t* __restrict__ W, int64_t ldw, int 
   __syncthreads();
   for (int i = ty; i < 32; i += 8) {
     const int m = m0 + i, k = k0 + tx;
-    if (m < N && k < Kp) Wb[(int64_t)m * Kp + k] = __float2bfloat16_rn((float)tile[tx][i]);
+    if (m < N && k < Kp) {
+      const int w = tile[tx][i];
+      const int h = w >> 4;                  // floor(w / 16)
+      uint8_t* row = Wq + (int64_t)m * 2 * Kp + (k / BK) * (2 * BK) + (k % BK);
+      row[0] = e4m3_of_small_int(16 * h);
+      row[BK] = e4m3_of_small_int(w - 16 * h);
+    }
   }
 }
 
-// Spike rows (either format) -> bf16 0/1 [T][Kp], zero past K.  One thread
-// per 16 consecutive columns of a row: one 16-byte load of u8 spikes (or a
-// half word of bits), two 16-byte stores.  kVec: u8 rows are 16-byte aligned
-// (base and leading dimension), so whole 16-column groups load as one vector.
+// Spike rows (any format) -> 0/1 bytes [T][Kp], zero past K.  One thread per
+// 16 consecutive columns of a row: one 16-byte store.  kVec: byte rows are
+// 16-byte aligned (base and leading dimension), so whole 16-column groups
+// load as one vector.
 template <bool kVec>
-__global__ void spikes_to_bf16_kernel(const void* __restrict__ spikes, int fmt, int64_t ld, int T,
-                                      int K, int Kp, __nv_bfloat16* __restrict__ Xb) {
+__global__ void spikes_to_01_kernel(const void* __restrict__ spikes, int fmt, int64_t ld, int T,
+                                    int K, int Kp, uint8_t* __restrict__ Xs) {
   pdl_launch_dependents();
   pdl_wait();
   const int per_row = Kp / 16;
@@ -571,32 +481,33 @@ __global__ void spikes_to_bf16_kernel(const void* __restrict__ spikes, int fmt, 
        i += (int64_t)gridDim.x * blockDim.x) {
     const int t = (int)(i / per_row);
     const int k = (int)(i - (int64_t)t * per_row) * 16;
-    uint32_t bits = 0u;                      // spikes of columns k .. k+15
+    uint4 o = make_uint4(0u, 0u, 0u, 0u);
     if (k < K) {
       const void* row = spike_row(spikes, fmt, t, ld);
-      if (fmt == SP_SPIKES_BITS32) {
-        bits = (__ldg(reinterpret_cast<const uint32_t*>(row) + (k >> 5)) >> (k & 31)) & 0xffffu;
+      if (fmt != SP_SPIKES_BITS32 && kVec && K - k >= 16) {
+        const uint4 w = __ldg(reinterpret_cast<const uint4*>(static_cast<const uint8_t*>(row) + k));
+        o = make_uint4(nonzero_bytes_to_01(w.x), nonzero_bytes_to_01(w.y), nonzero_bytes_to_01(w.z),
+                       nonzero_bytes_to_01(w.w));
       } else {
-        const uint8_t* x = reinterpret_cast<const uint8_t*>(row) + k;
-        if (kVec && K - k >= 16) {
-          const uint4 w = __ldg(reinterpret_cast<const uint4*>(x));
-          bits = nonzero_bytes_to_bits(w.x) | (nonzero_bytes_to_bits(w.y) << 4) |
-                 (nonzero_bytes_to_bits(w.z) << 8) | (nonzero_bytes_to_bits(w.w) << 12);
+        uint32_t bits = 0u;                  // spikes of columns k .. k+15
+        if (fmt == SP_SPIKES_BITS32) {
+          bits = (__ldg(reinterpret_cast<const uint32_t*>(row) + (k >> 5)) >> (k & 31)) & 0xffffu;
         } else {
+          const uint8_t* x = static_cast<const uint8_t*>(row) + k;
           const int n = K - k < 16 ? K - k : 16;
           for (int j = 0; j < n; ++j) bits |= (uint32_t)(__ldg(x + j) != 0) << j;
         }
-      }
-      if (K - k < 16) bits &= (1u << (K - k)) - 1u;
-    }
-    // bf16 1.0 = 0x3F80; two columns per 32-bit word
-    uint32_t o[8];
+        if (K - k < 16) bits &= (1u << (K - k)) - 1u;
+        uint32_t w[4];
 #pragma unroll
-    for (int j = 0; j < 8; ++j)
-      o[j] = ((bits >> (2 * j)) & 1u ? 0x3F80u : 0u) | ((bits >> (2 * j + 1)) & 1u ? 0x3F800000u : 0u);
-    uint4* dst = reinterpret_cast<uint4*>(Xb + (int64_t)t * Kp + k);
-    dst[0] = make_uint4(o[0], o[1], o[2], o[3]);
-    dst[1] = make_uint4(o[4], o[5], o[6], o[7]);
+        for (int j = 0; j < 4; ++j) {
+          const uint32_t nib = (bits >> (4 * j)) & 0xfu;
+          w[j] = (nib & 1u) | (nib & 2u) << 7 | (nib & 4u) << 14 | (nib & 8u) << 21;
+        }
+        o = make_uint4(w[0], w[1], w[2], w[3]);
+      }
+    }
+    *reinterpret_cast<uint4*>(Xs + (int64_t)t * Kp + k) = o;
   }
 }
 
@@ -616,26 +527,23 @@ PFN_cuTensorMapEncodeTiled_v12000 get_encode() {
   return fn;
 }
 
-bool encode_2d(CUtensorMap* map, const void* base, uint64_t inner, uint64_t outer,
-               uint32_t box_inner, uint32_t box_outer) {
+// 2-D byte matrix [outer][inner] with rows `stride` bytes apart, read in
+// box_inner x box_outer boxes, zero past the extents.
+bool encode_u8_2d(CUtensorMap* map, const void* base, uint64_t inner, uint64_t outer,
+                  uint64_t stride, uint32_t box_inner, uint32_t box_outer,
+                  CUtensorMapSwizzle swizzle) {
   auto enc = get_encode();
   if (!enc) return false;
   const cuuint64_t dims[2] = {inner, outer};
-  const cuuint64_t strides[1] = {inner * 2};
+  const cuuint64_t strides[1] = {stride};
   const cuuint32_t box[2] = {box_inner, box_outer};
   const cuuint32_t estr[2] = {1, 1};
-  return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box,
-             estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
-}
-
-template <bool kFusedX>
-constexpr int gemm_threads() {
-  return kFusedX ? kGemmThreadsFused : kGemmThreads;
+  return enc(map, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<void*>(base), dims, strides, box,
+             estr, CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
 // Largest number of clusters of `size` CTAs that can be resident at once.
-template <bool kFusedX>
 int max_active_clusters(int size) {
   static int cache[9] = {0};
   if (cache[size] == 0) {
@@ -646,12 +554,12 @@ int max_active_clusters(int size) {
     attr.val.clusterDim.y = 1;
     attr.val.clusterDim.z = 1;
     cfg.gridDim = dim3(size, 1, 1);
-    cfg.blockDim = dim3(gemm_threads<kFusedX>(), 1, 1);
-    cfg.dynamicSmemBytes = gemm_smem<kFusedX>();
+    cfg.blockDim = dim3(kGemmThreads, 1, 1);
+    cfg.dynamicSmemBytes = kGemmSmem;
     cfg.attrs = &attr;
     cfg.numAttrs = 1;
     int n = 0;
-    if (cudaOccupancyMaxActiveClusters(&n, gemm_kernel<kFusedX>, &cfg) != cudaSuccess || n < 1) {
+    if (cudaOccupancyMaxActiveClusters(&n, gemm_kernel, &cfg) != cudaSuccess || n < 1) {
       (void)cudaGetLastError();
       n = -1;
     }
@@ -660,14 +568,13 @@ int max_active_clusters(int size) {
   return cache[size];
 }
 
-template <bool kFusedX>
 cudaError_t set_gemm_attrs() {
   static bool done = false;
   if (done) return cudaSuccess;
-  cudaError_t e = cudaFuncSetAttribute(gemm_kernel<kFusedX>,
-                                       cudaFuncAttributeMaxDynamicSharedMemorySize, (int)gemm_smem<kFusedX>());
+  cudaError_t e = cudaFuncSetAttribute(gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)kGemmSmem);
   if (e != cudaSuccess) return e;
-  e = cudaFuncSetAttribute(gemm_kernel<kFusedX>, cudaFuncAttributeNonPortableClusterSizeAllowed, 0);
+  e = cudaFuncSetAttribute(gemm_kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 0);
   if (e != cudaSuccess) return e;
   done = true;
   return cudaSuccess;
@@ -686,7 +593,6 @@ cudaError_t init_sms() {
 
 // K splits for a T x N output: split only when the tiles alone leave SMs
 // idle, and only as far as every cluster stays resident in a single wave.
-template <bool kFusedX>
 int pick_splits(int T, int N, int Kp, int part_units) {
   const int tiles = ceil_div(T, BM) * ceil_div(N, BN);
   const int nkb = Kp / BK;
@@ -699,17 +605,69 @@ int pick_splits(int T, int N, int Kp, int part_units) {
     while (S > 1) {
       const int kbps = ceil_div(nkb, S);
       const int exact = ceil_div(nkb, kbps);            // splits with work
-      if (exact == S && max_active_clusters<kFusedX>(S) >= tiles && tiles * S <= part_units) break;
+      if (exact == S && max_active_clusters(S) >= tiles && tiles * S <= part_units) break;
       --S;
     }
   }
   return S;
 }
 
-template <bool kFusedX>
-cudaError_t launch_gemm_t(const CUtensorMap& mapA, const CUtensorMap& mapB, int S, int T, int N,
-                          int Kp, const GemmParams& p, cudaStream_t s) {
-  cudaError_t e = set_gemm_attrs<kFusedX>();
+}  // namespace
+
+int gemm_k_pad(int K) { return ceil_div(K, BK) * BK; }
+
+cudaError_t gemm_make_maps(const uint8_t* Xs, int rows_alloc, const uint8_t* Wq, int N, int Kp,
+                           GemmMaps* out) {
+  if (!encode_u8_2d(&out->a, Xs, (uint64_t)Kp, (uint64_t)rows_alloc, (uint64_t)Kp, BK, BM,
+                    CU_TENSOR_MAP_SWIZZLE_64B))
+    return cudaErrorUnknown;
+  if (!encode_u8_2d(&out->b, Wq, (uint64_t)2 * Kp, (uint64_t)N, (uint64_t)2 * Kp, 2 * BK, BN,
+                    CU_TENSOR_MAP_SWIZZLE_128B))
+    return cudaErrorUnknown;
+  return cudaSuccess;
+}
+
+cudaError_t gemm_make_rows_map(const void* X, int64_t ldx, int T, int K, CUtensorMap* out) {
+  return encode_u8_2d(out, X, (uint64_t)K, (uint64_t)T, (uint64_t)ldx, BK, BM,
+                      CU_TENSOR_MAP_SWIZZLE_64B)
+             ? cudaSuccess
+             : cudaErrorInvalidValue;
+}
+
+cudaError_t launch_w_to_e4m3(const int8_t* W, int64_t ldw, int N, int K, uint8_t* Wq,
+                             cudaStream_t s) {
+  const int Kp = gemm_k_pad(K);
+  dim3 grid(ceil_div(Kp, 32), ceil_div(N, 32)), block(32, 8);
+  w_to_e4m3_kernel<<<grid, block, 0, s>>>(W, ldw, N, K, Kp, Wq);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_spikes_to_01(const void* spikes, int fmt, int64_t ld, int T, int K, int Kp,
+                                uint8_t* Xs, cudaStream_t s) {
+  const int64_t total = (int64_t)T * (Kp / 16);
+  const int threads = 256;
+  int64_t blocks = (total + threads - 1) / threads;
+  if (blocks > 8192) blocks = 8192;
+  if (blocks < 1) blocks = 1;
+  const bool vec = fmt != SP_SPIKES_BITS32 && (reinterpret_cast<uintptr_t>(spikes) & 15u) == 0 &&
+                   ld % 16 == 0;
+  if (vec)
+    return launch_pdl(spikes_to_01_kernel<true>, dim3((unsigned)blocks), dim3(threads), 0, s, spikes,
+                      fmt, ld, T, K, Kp, Xs);
+  return launch_pdl(spikes_to_01_kernel<false>, dim3((unsigned)blocks), dim3(threads), 0, s, spikes,
+                    fmt, ld, T, K, Kp, Xs);
+}
+
+int gemm_splits(int T, int N, int Kp, int part_units) {
+  if (init_sms() != cudaSuccess || set_gemm_attrs() != cudaSuccess) return 1;
+  return pick_splits(T, N, Kp, part_units);
+}
+
+cudaError_t launch_gemm(const CUtensorMap& mapA, const CUtensorMap& mapB, int S, int T, int N,
+                        int Kp, const GemmParams& p, cudaStream_t s) {
+  cudaError_t e = init_sms();
+  if (e != cudaSuccess) return e;
+  e = set_gemm_attrs();
   if (e != cudaSuccess) return e;
   GemmArgs a;
   a.p = p;
@@ -719,11 +677,9 @@ cudaError_t launch_gemm_t(const CUtensorMap& mapA, const CUtensorMap& mapB, int 
   a.kb_per_split = ceil_div(a.nkb, S);
   a.splits = S;
   a.units = a.tiles_m * a.tiles_n * S;
-  const int threads = gemm_threads<kFusedX>();
-  const size_t smem = gemm_smem<kFusedX>();
   if (S == 1) {
     const int grid = a.units < g_num_sms ? a.units : g_num_sms;
-    return launch_pdl(gemm_kernel<kFusedX>, dim3(grid), dim3(threads), smem, s, mapA, mapB, a);
+    return launch_pdl(gemm_kernel, dim3(grid), dim3(kGemmThreads), kGemmSmem, s, mapA, mapB, a);
   }
   cudaLaunchConfig_t cfg = {};
   cudaLaunchAttribute attr[2];
@@ -734,79 +690,12 @@ cudaError_t launch_gemm_t(const CUtensorMap& mapA, const CUtensorMap& mapB, int 
   attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.gridDim = dim3(a.units, 1, 1);
-  cfg.blockDim = dim3(threads, 1, 1);
-  cfg.dynamicSmemBytes = smem;
+  cfg.blockDim = dim3(kGemmThreads, 1, 1);
+  cfg.dynamicSmemBytes = kGemmSmem;
   cfg.stream = s;
   cfg.attrs = attr;
   cfg.numAttrs = 2;
-  return cudaLaunchKernelEx(&cfg, gemm_kernel<kFusedX>, mapA, mapB, a);
-}
-
-}  // namespace
-
-int gemm_k_pad(int K) { return ceil_div(K, BK) * BK; }
-
-cudaError_t gemm_make_maps(const __nv_bfloat16* Xb, int rows_alloc, const __nv_bfloat16* Wb, int N,
-                           int Kp, GemmMaps* out) {
-  if (!encode_2d(&out->a, Xb, (uint64_t)Kp, (uint64_t)rows_alloc, BK, BM)) return cudaErrorUnknown;
-  if (!encode_2d(&out->b, Wb, (uint64_t)Kp, (uint64_t)N, BK, BN)) return cudaErrorUnknown;
-  return cudaSuccess;
-}
-
-cudaError_t launch_w_to_bf16(const int8_t* W, int64_t ldw, int N, int K, __nv_bfloat16* Wb,
-                             cudaStream_t s) {
-  const int Kp = gemm_k_pad(K);
-  dim3 grid(ceil_div(Kp, 32), ceil_div(N, 32)), block(32, 8);
-  w_to_bf16_kernel<<<grid, block, 0, s>>>(W, ldw, N, K, Kp, Wb);
-  return cudaGetLastError();
-}
-
-cudaError_t launch_spikes_to_bf16(const void* spikes, int fmt, int64_t ld, int T, int K, int Kp,
-                                  __nv_bfloat16* Xb, cudaStream_t s) {
-  const int64_t total = (int64_t)T * (Kp / 16);
-  const int threads = 256;
-  int64_t blocks = (total + threads - 1) / threads;
-  if (blocks > 8192) blocks = 8192;
-  if (blocks < 1) blocks = 1;
-  const bool vec = fmt == SP_SPIKES_U8 && (reinterpret_cast<uintptr_t>(spikes) & 15u) == 0 &&
-                   ld % 16 == 0;
-  if (vec)
-    return launch_pdl(spikes_to_bf16_kernel<true>, dim3((unsigned)blocks), dim3(threads), 0, s, spikes,
-                      fmt, ld, T, K, Kp, Xb);
-  return launch_pdl(spikes_to_bf16_kernel<false>, dim3((unsigned)blocks), dim3(threads), 0, s, spikes,
-                    fmt, ld, T, K, Kp, Xb);
-}
-
-cudaError_t gemm_make_x8_map(const void* X, int64_t ldx, int T, int K, CUtensorMap* out) {
-  auto enc = get_encode();
-  if (!enc) return cudaErrorUnknown;
-  const cuuint64_t dims[2] = {(cuuint64_t)K, (cuuint64_t)T};
-  const cuuint64_t strides[1] = {(cuuint64_t)ldx};
-  const cuuint32_t box[2] = {BK, BM};
-  const cuuint32_t estr[2] = {1, 1};
-  const CUresult r = enc(out, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<void*>(X), dims, strides,
-                         box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
-                         CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-  return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
-}
-
-int gemm_splits(bool fused_x, int T, int N, int Kp, int part_units) {
-  if (init_sms() != cudaSuccess) return 1;
-  if (fused_x) {
-    if (set_gemm_attrs<true>() != cudaSuccess) return 1;
-    return pick_splits<true>(T, N, Kp, part_units);
-  }
-  if (set_gemm_attrs<false>() != cudaSuccess) return 1;
-  return pick_splits<false>(T, N, Kp, part_units);
-}
-
-cudaError_t launch_gemm(const CUtensorMap& mapA, const CUtensorMap& mapB, bool fused_x, int S,
-                        int T, int N, int Kp, const GemmParams& p, cudaStream_t s) {
-  cudaError_t e = init_sms();
-  if (e != cudaSuccess) return e;
-  if (fused_x && S < 2) return cudaErrorInvalidValue;
-  return fused_x ? launch_gemm_t<true>(mapA, mapB, S, T, N, Kp, p, s)
-                 : launch_gemm_t<false>(mapA, mapB, S, T, N, Kp, p, s);
+  return cudaLaunchKernelEx(&cfg, gemm_kernel, mapA, mapB, a);
 }
 
 }  // namespace sp

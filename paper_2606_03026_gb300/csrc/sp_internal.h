@@ -3,7 +3,6 @@
 #pragma once
 
 #include <cuda_runtime.h>
-#include <cuda_bf16.h>
 #include <stdint.h>
 
 #include "spike_proj.h"
@@ -147,8 +146,8 @@ cudaError_t launch_union(const UnionParams& p, cudaStream_t s);
 // Counts active spikes: out[0] = sum over the B rows of |A_t| (out[1] unused).
 cudaError_t launch_density(const void* spikes, int fmt, int64_t ld, int B, int K,
                            int32_t* out, cudaStream_t s);
-// Spike rows in either format -> bf16 0/1 [T][Kp] (zero past K).
-cudaError_t launch_spikes_to_bf16(const void* spikes, int fmt, int64_t ld, int T, int K,
-                                  int Kp, __nv_bfloat16* Xb, cudaStream_t s);
+// Spike rows in any format -> bytes 0 / 1 [T][Kp] (zero past K).
+cudaError_t launch_spikes_to_01(const void* spikes, int fmt, int64_t ld, int T, int K, int Kp,
+                                uint8_t* Xs, cudaStream_t s);
 
 }  // namespace sp

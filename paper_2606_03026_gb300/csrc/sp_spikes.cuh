@@ -10,13 +10,16 @@ namespace sp {
 
 // --- spike words -------------------------------------------------------------
 
-// Four u8 spikes (one per byte of v) -> four bits, byte b -> bit b.
-__device__ __forceinline__ uint32_t nonzero_bytes_to_bits(uint32_t v) {
+// Four u8 spikes (one per byte of v) -> the same four bytes as 0 / 1.
+__device__ __forceinline__ uint32_t nonzero_bytes_to_01(uint32_t v) {
   v |= v >> 4;          // fold each byte onto its low bit; bits that leak in
   v |= v >> 2;          // from the next byte land above bit 3 of the byte and
   v |= v >> 1;          // are masked off below
-  v &= 0x01010101u;
-  return (v * 0x01020408u) >> 24;   // gather bit 0 of bytes 0..3 into bits 0..3
+  return v & 0x01010101u;
+}
+// Four u8 spikes (one per byte of v) -> four bits, byte b -> bit b.
+__device__ __forceinline__ uint32_t nonzero_bytes_to_bits(uint32_t v) {
+  return (nonzero_bytes_to_01(v) * 0x01020408u) >> 24;   // bit 0 of bytes 0..3 -> bits 0..3
 }
 
 // Word of the spike row covering columns [kw, kw + 32), bits at or past K

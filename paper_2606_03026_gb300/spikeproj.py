@@ -16,7 +16,7 @@ LIB_PATH = Path(__file__).resolve().parent / "_build" / "libspikeproj.so"
 SP_OK, SP_EINVAL, SP_EALIGN, SP_EDEVICE, SP_ECUDA, SP_ENOMEM, SP_ERANGE, \
     SP_EKERNEL, SP_EUNSUPPORTED, SP_ESCRATCH = range(10)
 # sp_fmt
-SP_SPIKES_BITS32, SP_SPIKES_U8 = 0, 1
+SP_SPIKES_BITS32, SP_SPIKES_U8, SP_SPIKES_BOOL8 = 0, 1, 2
 # sp_kernel
 SP_AUTO, SP_GATHER, SP_UNION, SP_GEMM = 0, 1, 2, 3
 SP_PLAN_GEMM = 0x1
@@ -24,7 +24,7 @@ SPIKE_PROJ_MAX_K = 131072
 SPIKE_PROJ_MAX_GROUP = 64
 SPIKE_PROJ_NOALLOC_MAX_N = 32768
 
-FMTS = {"bits": SP_SPIKES_BITS32, "u8": SP_SPIKES_U8}
+FMTS = {"bits": SP_SPIKES_BITS32, "u8": SP_SPIKES_U8, "bool8": SP_SPIKES_BOOL8}
 KERNELS = {"auto": SP_AUTO, "gather": SP_GATHER, "union": SP_UNION, "gemm": SP_GEMM}
 KERNEL_NAMES = {v: k for k, v in KERNELS.items()}
 

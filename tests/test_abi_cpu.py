@@ -30,6 +30,18 @@ def test_header_declares_the_boundary():
         assert required in names
 
 
+def test_header_enums_match_the_binding():
+    """Every enumerator of the header's enums has the binding's value."""
+    text = re.sub(r"/\*.*?\*/", "", HEADER.read_text(), flags=re.S)
+    found = {}
+    for body in re.findall(r"typedef enum \w+ \{(.*?)\}", text, flags=re.S):
+        for name, val in re.findall(r"\b(SP_\w+)\s*=\s*(\d+)", body):
+            found[name] = int(val)
+    assert found["SP_SPIKES_BOOL8"] == spikeproj.SP_SPIKES_BOOL8 == spikeproj.FMTS["bool8"]
+    for name, val in found.items():
+        assert getattr(spikeproj, name) == val, name
+
+
 def test_every_declared_symbol_is_exported(lib):
     names = declared_functions()
     assert names

@@ -40,8 +40,9 @@ def test_batch64(down, correlated, strategy):
     bits = synth.pack_bits(X)
     acc, y = run_batched(plan, to_dev(bits), "bits", 64, bits.shape[1], 1536, strategy)
     assert_parity(acc, y, want_acc, want_y, f"B=64 {strategy} corr={correlated}")
-    acc, y = run_batched(plan, to_dev(X), "u8", 64, X.shape[1], 1536, strategy)
-    assert_parity(acc, y, want_acc, want_y, f"B=64 u8 {strategy} corr={correlated}")
+    for fmt in ("u8", "bool8"):
+        acc, y = run_batched(plan, to_dev(X), fmt, 64, X.shape[1], 1536, strategy)
+        assert_parity(acc, y, want_acc, want_y, f"B=64 {fmt} {strategy} corr={correlated}")
     if strategy == "auto":
         chosen, active = plan.last_dispatch()
         assert chosen in STRATEGIES
@@ -67,6 +68,10 @@ def test_prefill_512_tokens(down):
         plan.prefill(Xd, 512, 6144, acc, y, strategy)
         torch.cuda.synchronize()
         assert_parity(acc, y, want_acc, want_y, f"prefill {strategy}")
+    # the same block as 0/1 bytes (a torch.bool tensor): read in place by the GEMM
+    Xbool = Xd.bool()
+    acc, y = run_batched(plan, Xbool, "bool8", 512, 6144, 1536, "gemm")
+    assert_parity(acc, y, want_acc, want_y, "prefill bool8 in place")
     assert plan.status() == sp.SP_OK
 
 
@@ -85,10 +90,10 @@ def test_gemm_ragged(T, N, K, ldq):
 
 @pytest.mark.parametrize("T,N,K", [(1, 16, 1), (5, 48, 100), (129, 272, 1000), (300, 1552, 777),
                                    (257, 512, 6143)])
-def test_gemm_u8_rows_read_in_kernel(T, N, K):
-    """u8 spike rows with a 16-byte-aligned row stride are read by the
-    tensor-core kernel itself (no bf16 staging copy): any nonzero byte is a
-    spike, bytes past K in each row are ignored, rows and K-blocks ragged."""
+def test_gemm_u8_rows_any_nonzero(T, N, K):
+    """u8 spike rows on the tensor-core path: any nonzero byte is a spike
+    (the 0/1 staging pass maps them), bytes past K in each row are ignored,
+    rows and K-blocks ragged."""
     Qc, s, X = synth.random_case(80 + T, N, K, T=T, p=0.3)
     ldx = (K + 15) // 16 * 16 + 16
     rng = synth.rng_for(81, T, K)
@@ -102,6 +107,27 @@ def test_gemm_u8_rows_read_in_kernel(T, N, K):
     assert plan.status() == sp.SP_OK
 
 
+@pytest.mark.parametrize("T,N,K", [(1, 16, 1), (5, 48, 100), (129, 272, 1000), (300, 1552, 777),
+                                   (257, 512, 6143), (512, 1536, 6144)])
+def test_gemm_bool8_rows(T, N, K):
+    """0/1 byte rows (SP_SPIKES_BOOL8): with a 16-byte-aligned row stride the
+    tensor-core kernel reads them in place (bytes past K ignored, whatever
+    they hold); with an odd stride they go through the staging pass.  Both
+    equal the oracle and the gather path bit for bit."""
+    Qc, s, X = synth.random_case(90 + T, N, K, T=T, p=0.3)
+    want_acc, want_y = oracle.project(Qc, s, N, K, X, "u8")
+    plan = sp.Plan(to_dev(Qc), to_dev(s), N, K, max_batch=T, gemm=True)
+    rng = synth.rng_for(91, T, K)
+    for ldx in ((K + 15) // 16 * 16 + 16, K + 1 if (K + 1) % 16 else K + 2):
+        Xs = rng.integers(2, 256, size=(T, ldx)).astype(np.uint8)    # not 0/1 past K
+        Xs[:, :K] = X != 0
+        Xd = to_dev(Xs)
+        for strategy in ("gemm", "gemm", "gather"):
+            acc, y = run_batched(plan, Xd, "bool8", T, ldx, N, strategy)
+            assert_parity(acc, y, want_acc, want_y, f"T={T} N={N} K={K} ldx={ldx} {strategy}")
+    assert plan.status() == sp.SP_OK
+
+
 def test_gemm_extremes():
     """All-ones spikes against -128 / +127 weights: the largest sums the
     tensor-core path must carry exactly (|acc| = 128 * K)."""
@@ -109,13 +135,14 @@ def test_gemm_extremes():
     X = np.ones((T, K), np.uint8)
     X[1::2, ::3] = 0
     s = np.linspace(-2, 2, N).astype(np.float32)
-    for c in (-128, 127):
+    for c, other in ((-128, 127), (127, -127), (127, 1), (-128, -1)):
         Qc = np.full((K, N), c, np.int8)
-        Qc[::5] = -c if c == 127 else 127
+        Qc[::5] = other                  # (127, 1) and (-128, -1): large odd sums
         want_acc, want_y = oracle.project(Qc, s, N, K, X, "u8")
         plan = sp.Plan(to_dev(Qc), to_dev(s), N, K, max_batch=T, gemm=True)
-        acc, y = run_batched(plan, to_dev(X), "u8", T, K, N, "gemm")
-        assert_parity(acc, y, want_acc, want_y, f"gemm extremes {c}")
+        for fmt in ("u8", "bool8"):
+            acc, y = run_batched(plan, to_dev(X), fmt, T, K, N, "gemm")
+            assert_parity(acc, y, want_acc, want_y, f"gemm extremes {c} {other} {fmt}")
 
 
 def test_auto_dispatch_by_cost(down):

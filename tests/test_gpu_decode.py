@@ -25,7 +25,7 @@ def test_single_projection_1536():
     N, K = c["N"], c["K"]
     want_acc, want_y = oracle.project(c["Q"], c["s"], N, K, c["x"], "u8")
     plan = sp.Plan(to_dev(c["Q"]), to_dev(c["s"]), N, K)
-    for fmt, x in (("u8", c["x"]), ("bits", c["bits"])):
+    for fmt, x in (("u8", c["x"]), ("bool8", c["x"]), ("bits", c["bits"])):
         acc, y = run_decode(plan, to_dev(x), fmt, N)
         assert_parity(acc, y, want_acc[0], want_y[0], f"single {fmt}")
     assert plan.status() == sp.SP_OK

@@ -86,7 +86,7 @@ def test_host_buffer_pageable_and_page_locked(step):
     want_acc, want_y = oracle_step(weights, xs)
     n, ld = len(weights), 1600
     for locked in (False, True):
-        for fmt, rows in (("bits", bits), ("u8", u8)):
+        for fmt, rows in (("bits", bits), ("u8", u8), ("bool8", u8 != 0)):
             h_rows = torch.from_numpy(np.ascontiguousarray(rows))
             h_acc = torch.full((n, ld), -3, dtype=torch.int32)
             h_y = torch.full((n, ld), -3.0, dtype=torch.float32)
