@@ -22,7 +22,7 @@
 // one bf16 MMA, while the spike operand is one byte per element and needs no
 // conversion pass.
 //
-// Kernel structure (192 threads):
+// Kernel structure (320 threads):
 //   warp 0      TMA producer: per 64-column K block, a 128 x 64 spike box
 //               (64-byte swizzle) and a 256 x 128 weight box (both planes,
 //               128-byte swizzle) into a 5-stage shared-memory ring
@@ -30,8 +30,10 @@
 //               and issues tcgen05.mma (M = 128, N = 256, K = 32) from one
 //               thread; tcgen05.commit frees ring slots and publishes
 //               accumulators
-//   warps 2-5   epilogue: warp w reads TMEM lane quarter w % 4 (32 rows),
-//               32 columns per tcgen05.ld
+//   warps 2-9   epilogue: warp w reads TMEM lane quarter w % 4 (32 rows);
+//               with K whole, warps 2-5 write 32-column chunks; with K split,
+//               warps 2-5 and 6-9 take alternate chunks of the partial and
+//               the two 16-column halves of every owned chunk
 // Whole K (enough output tiles for every SM): one CTA per SM, persistent over
 // 128 x 256 tiles; the epilogue of one tile overlaps the next tile's MMAs
 // (double-buffered accumulator) and writes acc / y through a shared-memory
@@ -40,8 +42,10 @@
 // 1536): the S CTAs of a thread-block cluster hold one tile for S K ranges.
 // Each CTA stores the 32-column chunks it does not own (chunk c belongs to
 // cluster rank c % S) into an fp32 workspace that stays in L2, one cluster
-// barrier (release / acquire) publishes them, and each owner adds the S - 1
-// partials of its chunks to its own accumulator and writes acc / y.
+// barrier (release / acquire) publishes them, and each owner pulls the S - 1
+// partials of each of its chunks into shared memory (bulk copies completing on
+// one mbarrier per chunk, so chunk 0 is added while chunk 1 lands), adds them
+// to its own accumulator and writes acc / y.
 //
 // Every mbarrier wait is bounded (2^31 SM cycles, about a second); on
 // timeout the kernel sets the error word, stops issuing work, drains what it
@@ -62,10 +66,12 @@ constexpr int A_BYTES = BM * BK;              // 8 KB: 0/1 spike bytes
 constexpr int B_BYTES = BN * BK * 2;          // 32 KB: the 16h and l planes
 constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
 constexpr int TMEM_COLS = 2 * BN;             // double-buffered accumulator
-constexpr int kGemmThreads = 192;             // TMA, MMA and 4 epilogue warps
+constexpr int kGemmThreads = 320;             // TMA, MMA and 8 epilogue warps
 constexpr int TR_STRIDE = 33;                 // padded transpose rows (words)
 constexpr size_t SMEM_RING = (size_t)STAGES * STAGE_BYTES;
-constexpr size_t SMEM_TR = (size_t)4 * 32 * TR_STRIDE * 4;
+constexpr int TR16_STRIDE = 17;               // padded 16-column transpose rows
+constexpr size_t SMEM_TR = (size_t)8 * 32 * TR16_STRIDE * 4 > (size_t)4 * 32 * TR_STRIDE * 4
+                               ? (size_t)8 * 32 * TR16_STRIDE * 4 : (size_t)4 * 32 * TR_STRIDE * 4;
 constexpr size_t SMEM_BARS = 256;
 constexpr size_t kGemmSmem = 1024 + SMEM_RING + SMEM_TR + SMEM_BARS;
 static_assert(kGemmSmem <= 227 * 1024, "shared memory per CTA");
@@ -160,12 +166,19 @@ __device__ __forceinline__ void store_chunk(const GemmParams& p, uint32_t* tr,
     int32_t* acc = p.acc ? p.acc + (int64_t)row0 * p.N + n : nullptr;
     float* y = p.y ? p.y + (int64_t)row0 * p.N + n : nullptr;
     if (nrows == 32) {
-      // full chunk: unrolled, so the 32 shared-memory reads are in flight together
+      // full chunk: all 32 shared-memory reads into registers before the
+      // first global store, so no store orders a later read
+      int val[32];
 #pragma unroll
-      for (int rr = 0; rr < 32; ++rr) {
-        const int val = __float2int_rn(__uint_as_float(tr[rr * TR_STRIDE + lane]) * kUnitsPerSpike);
-        if (acc) acc[(int64_t)rr * p.N] = val;
-        if (y) y[(int64_t)rr * p.N] = scale_out(sc, val);
+      for (int rr = 0; rr < 32; ++rr)
+        val[rr] = __float2int_rn(__uint_as_float(tr[rr * TR_STRIDE + lane]) * kUnitsPerSpike);
+      if (acc) {
+#pragma unroll
+        for (int rr = 0; rr < 32; ++rr) acc[(int64_t)rr * p.N] = val[rr];
+      }
+      if (y) {
+#pragma unroll
+        for (int rr = 0; rr < 32; ++rr) y[(int64_t)rr * p.N] = scale_out(sc, val[rr]);
       }
     } else {
       for (int rr = 0; rr < nrows; ++rr) {
@@ -176,6 +189,42 @@ __device__ __forceinline__ void store_chunk(const GemmParams& p, uint32_t* tr,
     }
   }
   __syncwarp();
+}
+
+// One warp writes a 32-row x 16-column block of fp32 sums in accumulator
+// units (v[i] = column col0 + i of row row0 + lane) through a shared-memory
+// transpose: lane l then holds column col0 + (l & 15) of rows 2 rr + (l >> 4),
+// so each store instruction covers 64 contiguous bytes of two rows.  sc = the
+// scale of column col0 + (lane & 15).
+__device__ __forceinline__ void store_block16(const GemmParams& p, uint32_t* tr,
+                                              const uint32_t (&v)[16], int row0, int col0,
+                                              float sc) {
+  const int lane = threadIdx.x & 31;
+#pragma unroll
+  for (int i = 0; i < 16; ++i) tr[lane * TR16_STRIDE + i] = v[i];
+  __syncwarp();
+  const int col = lane & 15, sub = lane >> 4;
+  const int n = col0 + col;
+  int val[16];
+#pragma unroll
+  for (int r2 = 0; r2 < 16; ++r2)
+    val[r2] = __float2int_rn(__uint_as_float(tr[(2 * r2 + sub) * TR16_STRIDE + col]) * kUnitsPerSpike);
+  __syncwarp();
+  if (n < p.N) {
+    const int nrows = p.T - row0 < 32 ? p.T - row0 : 32;
+    if (p.acc) {
+      int32_t* acc = p.acc + (int64_t)(row0 + sub) * p.N + n;
+#pragma unroll
+      for (int r2 = 0; r2 < 16; ++r2)
+        if (2 * r2 + sub < nrows) acc[(int64_t)(2 * r2) * p.N] = val[r2];
+    }
+    if (p.y) {
+      float* y = p.y + (int64_t)(row0 + sub) * p.N + n;
+#pragma unroll
+      for (int r2 = 0; r2 < 16; ++r2)
+        if (2 * r2 + sub < nrows) y[(int64_t)(2 * r2) * p.N] = scale_out(sc, val[r2]);
+    }
+  }
 }
 
 __global__ void __launch_bounds__(kGemmThreads, 1)
@@ -193,8 +242,8 @@ gemm_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CU
   uint64_t* tfull = bars + 2 * STAGES;   // [2] MMA -> epilogue
   uint64_t* tempty = tfull + 2;          // [2] epilogue -> MMA
   uint64_t* done = tempty + 2;           // all MMAs retired
-  uint64_t* pfull = done + 1;            // split K: peers' partials landed
-  uint32_t* s_tmem = reinterpret_cast<uint32_t*>(pfull + 1);
+  uint64_t* pfull = done + 1;            // [kMaxOwned] split K: peers' partials of owned chunk j
+  uint32_t* s_tmem = reinterpret_cast<uint32_t*>(pfull + kMaxOwned);
   volatile int* s_abort = reinterpret_cast<volatile int*>(s_tmem + 1);
 
   const int warp = threadIdx.x >> 5;
@@ -210,7 +259,7 @@ gemm_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CU
       mbar_init(&tempty[b], 4);          // one arrive per epilogue warp
     }
     mbar_init(done, 1);
-    mbar_init(pfull, 1);
+    for (int j = 0; j < kMaxOwned; ++j) mbar_init(&pfull[j], 1);
     *s_abort = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     tma_prefetch_desc(&mapA);
@@ -305,33 +354,35 @@ gemm_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CU
       mbar_wait(done, 0);
     }
   } else if (a.splits == 1) {
-    // ------------------------------ epilogue (whole K) ------------------------
-    // Each warp owns one 32-row quarter of the tile (its TMEM lane quarter) and
-    // works alone: no barrier joins the epilogue warps, so a warp that gives up
-    // on a timed-out wait cannot strand the others.
-    const int q = warp & 3;
-    uint32_t* tr = s_tr + (size_t)(warp - 2) * 32 * TR_STRIDE;
-    int ab = 0;
-    uint32_t aph = 0;
-    for (int u = blockIdx.x; u < a.units; u += gridDim.x) {
-      int tile, mb, nb, kb0, kb1;
-      unit_coords(a, u, tile, mb, nb, kb0, kb1);
-      if (!mbar_wait(&tfull[ab], aph)) {
-        *s_abort = 1;
-        if (lane == 0) atomicExch(a.p.err, kErrMbarTimeout);
-        break;
+    if (warp < 6) {                           // the whole-K epilogue uses warps 2-5
+      // ------------------------------ epilogue (whole K) ------------------------
+      // Each warp owns one 32-row quarter of the tile (its TMEM lane quarter) and
+      // works alone: no barrier joins the epilogue warps, so a warp that gives up
+      // on a timed-out wait cannot strand the others.
+      const int q = warp & 3;
+      uint32_t* tr = s_tr + (size_t)(warp - 2) * 32 * TR_STRIDE;
+      int ab = 0;
+      uint32_t aph = 0;
+      for (int u = blockIdx.x; u < a.units; u += gridDim.x) {
+        int tile, mb, nb, kb0, kb1;
+        unit_coords(a, u, tile, mb, nb, kb0, kb1);
+        if (!mbar_wait(&tfull[ab], aph)) {
+          *s_abort = 1;
+          if (lane == 0) atomicExch(a.p.err, kErrMbarTimeout);
+          break;
+        }
+        tc_fence_after();
+        const int row0 = mb * BM + q * 32;
+        for (int c = 0; c < BN; c += 32) {
+          uint32_t v[32];
+          tmem_ld32(tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(ab * BN + c), v);
+          store_chunk(a.p, tr, v, row0, nb * BN + c, column_scale(a.p, nb * BN + c + lane));
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&tempty[ab]);
+        if (++ab == 2) { ab = 0; aph ^= 1u; }
       }
-      tc_fence_after();
-      const int row0 = mb * BM + q * 32;
-      for (int c = 0; c < BN; c += 32) {
-        uint32_t v[32];
-        tmem_ld32(tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(ab * BN + c), v);
-        store_chunk(a.p, tr, v, row0, nb * BN + c, column_scale(a.p, nb * BN + c + lane));
-      }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&tempty[ab]);
-      if (++ab == 2) { ab = 0; aph ^= 1u; }
     }
   } else {
     // ---------------- epilogue (split K): reduce-scatter through L2 -----------
@@ -352,29 +403,36 @@ gemm_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CU
     const int S = a.splits;
     const int rank = (int)cluster_ctarank();
     const bool epi = warp >= 2;
-    const int q = warp & 3;
+    const int q = warp & 3;                  // TMEM lane quarter
+    const int half = (warp - 2) >> 2;        // warps 2-5: 0, warps 6-9: 1
     int tile, mb, nb, kb0, kb1;
     unit_coords(a, blockIdx.x, tile, mb, nb, kb0, kb1);
     const float* tile_part = a.p.part + (size_t)tile * S * (BM * BN);
-    // scales of the owned chunks' columns, in flight while the partials go out
+    // scales of this warp's 16 columns of each owned chunk
     float sc[kMaxOwned];
 #pragma unroll
     for (int j = 0; j < kMaxOwned; ++j)
-      sc[j] = (epi && rank + j * S < BN / 32) ? column_scale(a.p, nb * BN + (rank + j * S) * 32 + lane)
-                                              : 0.f;
+      sc[j] = (epi && rank + j * S < BN / 32)
+                  ? column_scale(a.p, nb * BN + (rank + j * S) * 32 + half * 16 + (lane & 15))
+                  : 0.f;
     if (epi && !*s_abort) {
-      // chunks two at a time: two TMEM loads behind one wait
+      // the chunks of this warp's parity, two at a time behind one wait
       float* mine = a.p.part + ((size_t)tile * S + rank) * (BM * BN) + q * 1024 + lane;
-      for (int c = 0; c < BN / 32; c += 2) {
+      const uint32_t trow = tmem_base + ((uint32_t)(q * 32) << 16);
+      for (int c = half; c < BN / 32; c += 4) {
         uint32_t v0[32], v1[32];
-        tmem_ld32x2(tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)c * 32u, v0, v1);
+        tmem_ld32_issue(trow + (uint32_t)c * 32u, v0);
+        tmem_ld32_issue(trow + (uint32_t)(c + 2) * 32u, v1);
+        asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+        reg_pin(v0);
+        reg_pin(v1);
         if (c % S != rank) {
           float* dst = mine + (size_t)c * 4096;
 #pragma unroll
           for (int i = 0; i < 32; ++i) __stcg(dst + i * 32, __uint_as_float(v0[i]));
         }
-        if ((c + 1) % S != rank) {
-          float* dst = mine + (size_t)(c + 1) * 4096;
+        if ((c + 2) % S != rank) {
+          float* dst = mine + (size_t)(c + 2) * 4096;
 #pragma unroll
           for (int i = 0; i < 32; ++i) __stcg(dst + i * 32, __uint_as_float(v1[i]));
         }
@@ -382,39 +440,40 @@ gemm_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CU
     }
     cluster_sync();                                     // partials published
     // The ring is idle (every MMA of this CTA has completed): one thread pulls
-    // the S - 1 peer partials of every owned chunk into it with bulk copies.
-    const int owned = (BN / 32 - rank + S - 1) / S;
+    // the S - 1 peer partials of each owned chunk j into it with bulk copies
+    // that complete on pfull[j].
     if (warp == 2 && lane == 0 && !*s_abort) {
       asm volatile("fence.proxy.async.global;" ::: "memory");
-      mbar_arrive_expect_tx(pfull, (uint32_t)((S - 1) * owned * kPartChunkBytes));
       int slot = 0;
-      for (int c = rank; c < BN / 32; c += S)
+      for (int j = 0, c = rank; c < BN / 32; ++j, c += S) {
+        mbar_arrive_expect_tx(&pfull[j], (uint32_t)((S - 1) * kPartChunkBytes));
         for (int r = 0; r < S; ++r)
           if (r != rank)
             bulk_load(smem + (size_t)(slot++) * kPartChunkBytes,
-                      tile_part + ((size_t)r * CPT + c) * 4096, kPartChunkBytes, pfull);
+                      tile_part + ((size_t)r * CPT + c) * 4096, kPartChunkBytes, &pfull[j]);
+      }
     }
     if (epi && !*s_abort) {
-      if (!mbar_wait(pfull, 0)) {
-        *s_abort = 1;
-        if (lane == 0) atomicExch(a.p.err, kErrMbarTimeout);
-      } else {
-        uint32_t* tr = s_tr + (size_t)(warp - 2) * 32 * TR_STRIDE;
+      uint32_t* tr = s_tr + (size_t)(warp - 2) * 32 * TR16_STRIDE;
 #pragma unroll
-        for (int j = 0; j < kMaxOwned; ++j) {
-          const int c = rank + j * S;
-          if (c >= BN / 32) break;
-          uint32_t v[32];
-          tmem_ld32(tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)c * 32u, v);
-          for (int r = 0; r < S - 1; ++r) {
-            const float* src = reinterpret_cast<const float*>(
-                                   smem + (size_t)(j * (S - 1) + r) * kPartChunkBytes) +
-                               q * 1024 + lane;
-#pragma unroll
-            for (int i = 0; i < 32; ++i) v[i] = __float_as_uint(__uint_as_float(v[i]) + src[i * 32]);
-          }
-          store_chunk(a.p, tr, v, mb * BM + q * 32, nb * BN + c * 32, sc[j]);
+      for (int j = 0; j < kMaxOwned; ++j) {
+        const int c = rank + j * S;
+        if (c >= BN / 32) break;
+        if (!mbar_wait(&pfull[j], 0)) {
+          *s_abort = 1;
+          if (lane == 0) atomicExch(a.p.err, kErrMbarTimeout);
+          break;
         }
+        uint32_t v[16];
+        tmem_ld16(tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(c * 32 + half * 16), v);
+        for (int r = 0; r < S - 1; ++r) {
+          const float* src = reinterpret_cast<const float*>(
+                                 smem + (size_t)(j * (S - 1) + r) * kPartChunkBytes) +
+                             q * 1024 + half * 16 * 32 + lane;
+#pragma unroll
+          for (int i = 0; i < 16; ++i) v[i] = __float_as_uint(__uint_as_float(v[i]) + src[i * 32]);
+        }
+        store_block16(a.p, tr, v, mb * BM + q * 32, nb * BN + c * 32 + half * 16, sc[j]);
       }
     }
   }
