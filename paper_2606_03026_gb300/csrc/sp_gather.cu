@@ -349,6 +349,9 @@ gather_cluster_kernel(const __grid_constant__ GatherParamsT<NP> p) {
   __shared__ ClusterSmem sm;
   // [sender chunk][owned group]: kch * ceil(128 / kch) < 128 + kch entries
   __shared__ __align__(16) int4 s_recv[kGatherNT / 4 + kGatherCluster];
+  // every CTA of the cluster arrives here and waits (below) before its first
+  // store into a peer's shared memory: the peer is then known to be running
+  asm volatile("barrier.cluster.arrive.relaxed;" ::: "memory");
   pdl_launch_dependents();
   if (blockIdx.y == 0) prefetch_spike_rows(p);   // before the wait: see gather_kernel
   pdl_wait();
@@ -362,7 +365,10 @@ gather_cluster_kernel(const __grid_constant__ GatherParamsT<NP> p) {
     cl = e & 0xff;
   }
   const GatherProblem& P = p.prob[j];
-  if (cl >= P.ncl) return;                  // the whole cluster: no tile of this problem
+  if (cl >= P.ncl) {                        // the whole cluster: no tile of this problem
+    asm volatile("barrier.cluster.wait;" ::: "memory");
+    return;
+  }
   const int kch = P.kch;
   const int per = (kGatherNT / 4 + kch - 1) / kch;   // most groups owned by one CTA
   const int ts = rank / kch;
@@ -372,6 +378,7 @@ gather_cluster_kernel(const __grid_constant__ GatherParamsT<NP> p) {
   if (work) {
     unit_partial<kGatherClusterWarps, kGatherClusterMaxCK, kClusterLoads, kClusterSlots>(
         sm, P, spike_row(p.spikes, p.fmt, j, p.ld_spikes), p.fmt, n0, kc * P.ck, P.ck);
+    asm volatile("barrier.cluster.wait;" ::: "memory");
     const int g = threadIdx.x;              // the 4-channel group of this thread
     if (g < kGatherNT / 4) {
       const int4 v = unit_sum4(sm, 4 * g);
@@ -380,6 +387,7 @@ gather_cluster_kernel(const __grid_constant__ GatherParamsT<NP> p) {
                  (uint32_t)(ts * kch + owner), v);
     }
   }
+  if (!work) asm volatile("barrier.cluster.wait;" ::: "memory");
   cluster_sync_all();                       // every partial is in its owner's shared memory
   const int g_own = kc * per + threadIdx.x; // this thread's owned group (a contiguous run)
   const int n = n0 + 4 * g_own;
