@@ -200,9 +200,9 @@ sp_status spike_proj_plan_status(sp_plan_t plan, sp_stream_t stream);
 
 /* ---------------------------------------------------------------------------
  * Groups: several independent batch-1 projections in ONE kernel launch, e.g.
- * the 44 binary-input projections of one 22-block decode step (per block the
- * sequence-mixer projection and the feed-forward down projection, Section
- * 2.1).  All projections of a group run concurrently, so their combined
+ * the 44 binary-input projections of one 22-block decode step (per block,
+ * the sequence mixer's TCAM projection and the FFN's down projection,
+ * Section 2.1).  All projections of a group run concurrently, so their combined
  * active-column traffic can fill the memory system.
  *
  * spike_proj_group_create: plans[0..count) (1 <= count <= SPIKE_PROJ_MAX_GROUP)

@@ -12,6 +12,10 @@ Functions mirror ``spike_oracle.h``:
   to INT32, ``y_m = s_m * float32(acc_m)`` (Eq. sparse and the sentence after
   it), for T spike rows.
 * :func:`project_entries` -- the same at selected (row, channel) pairs.
+* :func:`dense` -- the continuous-input projection over row-major INT8
+  weights, ``y_m = s_m * sum_k Q[m*ldq + k] * x_k`` evaluated in double, with
+  ``sum_k |Q_mk x_k|`` for error bounds (Section 2.3, the sentence on
+  continuous inputs; Section 2.2 for the row-major layout).
 
 Spike formats: ``"bits"`` = uint32 words, column k is bit k%32 of word k//32
 (LSB first, tail bits ignored); ``"u8"`` = one byte per column, nonzero fires.
@@ -83,6 +87,8 @@ class Oracle:
                                                   ctypes.c_int, i64, i32, i64,
                                                   p, p, p, p]
         lib.sp_oracle_project_entries.restype = ctypes.c_int
+        lib.sp_oracle_dense.argtypes = [p, i64, p, i32, i32, p, i64, i32, p, p]
+        lib.sp_oracle_dense.restype = ctypes.c_int
         self.lib = lib
 
     # -- helpers -----------------------------------------------------------
@@ -168,6 +174,34 @@ class Oracle:
         return acc, y
 
 
+    def dense(self, Q: np.ndarray, scale: np.ndarray, N: int, K: int,
+              x: np.ndarray, ldq: int | None = None):
+        """Continuous-input projection of every row of ``x`` (float32 [T, >=K])
+        through row-major ``Q`` ([N, ldq] int8); returns (y, abs_dot), both
+        float64 [T, N]."""
+        ldq = K if ldq is None else ldq
+        Q = np.ascontiguousarray(Q, dtype=np.int8).reshape(-1)
+        if ldq < K or Q.size < ldq * (N - 1) + K:
+            raise ValueError("Q too small for N, K, ldq")
+        scale = np.ascontiguousarray(scale, dtype=np.float32).reshape(-1)
+        if scale.size < N:
+            raise ValueError("scale shorter than N")
+        x = np.ascontiguousarray(x, dtype=np.float32)
+        if x.ndim == 1:
+            x = x[None, :]
+        if x.shape[1] < K:
+            raise ValueError("x rows shorter than K")
+        T = x.shape[0]
+        y = np.zeros((T, N), dtype=np.float64)
+        mag = np.zeros((T, N), dtype=np.float64)
+        rc = self.lib.sp_oracle_dense(Q.ctypes.data, ldq, scale.ctypes.data, N, K,
+                                      x.ctypes.data, x.shape[1], T, y.ctypes.data,
+                                      mag.ctypes.data)
+        if rc:
+            raise RuntimeError(f"sp_oracle_dense failed: {rc}")
+        return y, mag
+
+
 _DEFAULT: Oracle | None = None
 
 
@@ -190,3 +224,7 @@ def project(Q, scale, N, K, spikes, fmt, ldq=None):
 def project_entries(Q, scale, N, K, spikes, fmt, t_idx, m_idx, ldq=None):
     return default().project_entries(Q, scale, N, K, spikes, fmt, t_idx,
                                      m_idx, ldq)
+
+
+def dense(Q, scale, N, K, x, ldq=None):
+    return default().dense(Q, scale, N, K, x, ldq)

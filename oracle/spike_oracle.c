@@ -147,3 +147,33 @@ int sp_oracle_project_entries(const int8_t *Q, int64_t ldq, const float *s,
     free(A);
     return rc;
 }
+
+/* Continuous-input projection, written out as its definition (Section 2.3):
+ * for each row t and output m, dot = sum_k Q_{m,k} x_k with Q row-major
+ * (Section 2.2), then y = s_m * dot.  See spike_oracle.h for the precision. */
+int sp_oracle_dense(const int8_t *Q, int64_t ldq, const float *s,
+                    int32_t N, int32_t K, const float *x, int64_t ldx,
+                    int32_t T, double *y, double *abs_dot)
+{
+    if (!Q || !x || N < 0 || K < 0 || T < 0 || ldq < K || (y && !s))
+        return -1;
+    if (T > 1 && ldx < K)
+        return -1;
+    for (int32_t t = 0; t < T; ++t) {
+        const float *xt = x + (int64_t)t * ldx;
+        for (int32_t m = 0; m < N; ++m) {
+            const int8_t *q = Q + (int64_t)m * ldq;
+            double dot = 0.0, mag = 0.0;
+            for (int32_t k = 0; k < K; ++k) {
+                double term = (double)q[k] * (double)xt[k];
+                dot += term;
+                mag += term < 0 ? -term : term;
+            }
+            if (y)
+                y[(int64_t)t * N + m] = (double)s[m] * dot;
+            if (abs_dot)
+                abs_dot[(int64_t)t * N + m] = mag;
+        }
+    }
+    return 0;
+}

@@ -16,12 +16,14 @@
  * per-output-channel scale (Section 2.3 quantiser); x a binary spike vector.
  * The sum is held in a 64-bit integer, range-checked and narrowed to INT32
  * (the paper's general accumulator is INT32, Section 2.3), converted to FP32
- * and multiplied by s_m once (Section 2.3: "converted to FP32 and scaled once
- * per output channel").
+ * and multiplied by s_m once per output channel (Section 2.3).
  *
  * Spike formats: SP_ORACLE_U8 -- one byte per column, any nonzero byte is a
  * spike; SP_ORACLE_BITS32 -- uint32 words, column k is bit (k % 32) of word
  * (k / 32), bits at or beyond K are ignored.
+ *
+ * sp_oracle_dense (declared last) is the paper's other kernel: the
+ * continuous-input projection over row-major INT8 weights.
  *
  * All functions are single-threaded, allocate only O(K) scratch, and return
  * 0 on success, a negative code on a bad argument (-1) or an INT32 overflow of
@@ -61,6 +63,25 @@ int sp_oracle_project_entries(const int8_t *Q, int64_t ldq, const float *s,
                               int32_t T, int64_t count,
                               const int32_t *t_idx, const int32_t *m_idx,
                               int32_t *acc, float *y);
+
+/* Continuous-input projection (Section 2.3: for continuous inputs the
+ * weights are converted to FP32, multiplied with the FP32 activations and
+ * accumulated, and the row scale is applied afterwards; Section 2.2: dense
+ * projections keep row-major storage, one contiguous dot product per output):
+ *
+ *     y_m = s_m * sum_k Q_{m,k} x_k
+ *
+ * with Q INT8 ROW-MAJOR, element (m, k) at Q[m * ldq + k] (ldq >= K), and x
+ * FP32 rows, row t at x + t * ldx (ldx >= K when T > 1).  The value is
+ * computed in double: every product (double)Q * (double)x is exact (8 + 24
+ * significant bits), the K products are summed in ascending k (error at most
+ * K * 2^-53 of sum_k |Q_{m,k} x_k|, far below FP32 resolution), and the scale
+ * is one double multiply.  Outputs are dense [T][N]: y[t*N + m] and
+ * abs_dot[t*N + m] = sum_k |Q_{m,k} x_k| (for error bounds); either may be
+ * NULL. */
+int sp_oracle_dense(const int8_t *Q, int64_t ldq, const float *s,
+                    int32_t N, int32_t K, const float *x, int64_t ldx,
+                    int32_t T, double *y, double *abs_dot);
 
 #ifdef __cplusplus
 }

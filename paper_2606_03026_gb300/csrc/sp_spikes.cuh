@@ -1,6 +1,6 @@
 // sp_spikes.cuh -- device helpers shared by the gather and union kernels:
 // reading spike rows as 32-column words, compacting words into the ascending
-// active-column list (Section 2.2: "the runtime gathers these indices"), and
+// active-column list (Section 2.2: the active indices are collected first), and
 // the byte-lane accumulation of INT8 columns.
 #pragma once
 

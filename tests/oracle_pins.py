@@ -18,6 +18,14 @@ What pins what (Section 2.3, Eq. sparse: y_m = s_m * sum_{k in A} Q_{m,k}):
   all-ones row sums, column permutation, format equivalence, tail bits,
   nonzero bytes;
 * closed forms -- constant Q, INT8 extremes, INT32 overflow reported.
+
+The continuous-input projection (Section 2.3, row-major weights of Section
+2.2: y_m = s_m * sum_k Q[m][k] x_k, evaluated in double) is pinned by a
+hand-worked fixture (tests/golden/hand_worked_dense.json), numpy float64
+matmul with padded row strides, closed forms (constant Q and x, one-hot,
+zero, extremes), linearity on dyadic inputs (exact in double), and, for
+0/1 inputs, exact agreement with the spike-gated projection of the same
+matrix.
 """
 from __future__ import annotations
 
@@ -200,6 +208,95 @@ def pin_entries(orc):
     assert np.array_equal(be, ae)
 
 
+# --- continuous-input projection ---------------------------------------------
+
+def dense_case(seed, N, K, T, ldq, ldx):
+    """Row-major Q [N, ldq] with random padding, x float32 [T, ldx] whose
+    columns past K are large (so a read past K shows), scale [N]."""
+    rng = synth.rng_for(300 + seed, N, K, T)
+    Q = rng.integers(-128, 128, size=(N, ldq)).astype(np.int8)
+    x = rng.standard_normal((T, ldx)).astype(np.float32)
+    x[:, K:] = 1.0e6
+    s = rng.uniform(0.25, 2.0, N).astype(np.float32)
+    return Q, x, s
+
+
+def pin_dense_hand_fixture(orc):
+    g = json.loads((GOLDEN / "hand_worked_dense.json").read_text())
+    Q = np.array(g["Q_rows"], np.int8)
+    y, mag = orc.dense(Q, np.array(g["s"], np.float32), g["N"], g["K"],
+                       np.array(g["x"], np.float32), ldq=g["ldq"])
+    assert y[0].tolist() == g["y"], (y, g["y"])
+    assert mag[0].tolist() == g["abs_dot"], (mag, g["abs_dot"])
+
+
+def pin_dense_matmul(orc):
+    # N != K, ldq > K and ldx > K so a transposed operand, a dropped stride
+    # or a read past K shows.
+    for (N, K, T, ldq, ldx, seed) in ((7, 13, 3, 16, 20, 1), (64, 300, 2, 304, 308, 2),
+                                      (1536, 1536, 1, 1536, 1540, 3)):
+        Q, x, s = dense_case(seed, N, K, T, ldq, ldx)
+        y, mag = orc.dense(Q, s, N, K, x, ldq=ldq)
+        Ql = Q[:, :K].astype(np.float64)
+        xl = x[:, :K].astype(np.float64)
+        want = (xl @ Ql.T) * s.astype(np.float64)[None, :]
+        want_mag = np.abs(xl) @ np.abs(Ql).T
+        tol = 4 * K * 2.0 ** -53 * want_mag * s.astype(np.float64)[None, :]
+        assert np.all(np.abs(y - want) <= tol), np.max(np.abs(y - want) - tol)
+        assert np.allclose(mag, want_mag, rtol=4 * K * 2.0 ** -53, atol=0)
+
+
+def pin_dense_closed_forms(orc):
+    N, K = 24, 1000
+    s = np.linspace(0.5, 3.0, N).astype(np.float32)
+    # constant Q = c, constant x = 0.5: every dot is c * K / 2 exactly
+    for c in (1, -128, 127):
+        Q = np.full((N, K), c, np.int8)
+        y, _ = orc.dense(Q, s, N, K, np.full(K, 0.5, np.float32))
+        assert np.array_equal(y[0], s.astype(np.float64) * (c * K / 2)), c
+    Q, x, _ = dense_case(4, N, K, 1, K, K)
+    # zero input, one-hot input (column k of Q times the scale)
+    y, mag = orc.dense(Q, s, N, K, np.zeros(K, np.float32))
+    assert not y.any() and not mag.any()
+    for k in (0, 1, K // 2, K - 1):
+        e = np.zeros(K, np.float32)
+        e[k] = 1.0
+        y, _ = orc.dense(Q, s, N, K, e)
+        assert np.array_equal(y[0], s.astype(np.float64) * Q[:, k]), k
+
+
+def pin_dense_linearity(orc):
+    # dyadic inputs (multiples of 1/4, |x| <= 8): every partial sum is exact
+    # in double, so y(x1 + x2) = y(x1) + y(x2) and y(-x) = -y(x) bit for bit
+    N, K = 40, 257
+    rng = synth.rng_for(305)
+    Q = rng.integers(-128, 128, size=(N, K)).astype(np.int8)
+    s = np.ones(N, np.float32)
+    x1 = (rng.integers(-16, 17, K) / 4).astype(np.float32)
+    x2 = (rng.integers(-16, 17, K) / 4).astype(np.float32)
+    y1, _ = orc.dense(Q, s, N, K, x1)
+    y2, _ = orc.dense(Q, s, N, K, x2)
+    y12, _ = orc.dense(Q, s, N, K, x1 + x2)
+    yn, _ = orc.dense(Q, s, N, K, -x1)
+    assert np.array_equal(y12, y1 + y2)
+    assert np.array_equal(yn, -y1)
+
+
+def pin_dense_binary_is_sparse(orc):
+    # for x in {0, 1}^K the dot product is the integer sum of Eq. (sparse)
+    # over the active columns, and s * dot rounded to FP32 is the sparse y
+    N, K, T = 48, 700, 4
+    Q, _, s = dense_case(6, N, K, T, K, K)
+    xb = synth.bernoulli(synth.rng_for(306), (T, K), 0.3)
+    y, _ = orc.dense(Q, np.ones(N, np.float32), N, K, xb.astype(np.float32))
+    acc, ysp = orc.project(np.ascontiguousarray(Q.T), s, N, K, xb, "u8")
+    assert np.array_equal(y, acc.astype(np.float64))
+    yd, _ = orc.dense(Q, s, N, K, xb.astype(np.float32))
+    assert np.array_equal(yd.astype(np.float32), ysp)
+
+
 ALL_PINS = [pin_hand_fixture, pin_exhaustive_small, pin_full_shapes,
             pin_scale_rounding, pin_invariants, pin_closed_forms,
-            pin_overflow_reported, pin_entries]
+            pin_overflow_reported, pin_entries,
+            pin_dense_hand_fixture, pin_dense_matmul, pin_dense_closed_forms,
+            pin_dense_linearity, pin_dense_binary_is_sparse]

@@ -1,6 +1,8 @@
 """Plant one mistake at a time in a copy of the oracle and check that the
 pins catch it: a dropped term, a wrong sign, a transposed operand, a wrong
-bit index, a lost scale, a wrong spike test, a lost overflow check.  The
+bit index, a lost scale, a wrong spike test, a lost overflow check; for the
+continuous-input projection a dropped row or activation stride, a dropped
+term, a wrong sign, a lost scale, a signed magnitude, a float accumulator.  The
 mutants are compiled on the CPU from the oracle's own source text."""
 from pathlib import Path
 
@@ -24,6 +26,14 @@ MUTANTS = {
     "last_column_skipped": ("for (int32_t k = 0; k < K; ++k)\n        if (spike_at", "for (int32_t k = 0; k < K - 1; ++k)\n        if (spike_at"),
     "overflow_unchecked": ("if (acc > INT32_MAX || acc < INT32_MIN)\n        return -2;", ""),
     "narrow_accumulator": ("int64_t acc = 0;", "int16_t acc = 0;"),
+    # continuous-input projection (every mutant stays inside its buffers)
+    "dense_row_stride_ignored": ("const int8_t *q = Q + (int64_t)m * ldq;", "const int8_t *q = Q + (int64_t)m * K;"),
+    "dense_x_stride_ignored": ("const float *xt = x + (int64_t)t * ldx;", "const float *xt = x + (int64_t)t * K;"),
+    "dense_last_term_dropped": ("for (int32_t k = 0; k < K; ++k) {\n                double term", "for (int32_t k = 0; k + 1 < K; ++k) {\n                double term"),
+    "dense_wrong_sign": ("dot += term;", "dot -= term;"),
+    "dense_scale_dropped": ("y[(int64_t)t * N + m] = (double)s[m] * dot;", "y[(int64_t)t * N + m] = dot;"),
+    "dense_abs_signed": ("mag += term < 0 ? -term : term;", "mag += term;"),
+    "dense_float_accumulator": ("double dot = 0.0, mag = 0.0;", "float dot = 0.0f; double mag = 0.0;"),
 }
 
 
