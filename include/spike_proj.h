@@ -48,6 +48,8 @@ extern "C" {
 #define SPIKE_PROJ_MAX_K 131072        /* 128 * K < 2^24: exact FP32 conversion */
 #define SPIKE_PROJ_MAX_GROUP 64        /* projections per group */
 #define SPIKE_PROJ_NOALLOC_MAX_N 32768 /* largest N of spike_proj_decode_noalloc */
+#define SPIKE_PROJ_DENSE_MAX_B 4       /* activation rows per spike_proj_dense call */
+#define SPIKE_PROJ_DENSE_MAX_GROUP 128 /* problems per spike_proj_dense call */
 
 typedef struct sp_plan_s *sp_plan_t;
 typedef struct sp_group_s *sp_group_t;
@@ -278,6 +280,52 @@ sp_status spike_proj_decode_noalloc(const int8_t *W, int64_t ldw,
                                     const void *spikes, sp_fmt fmt,
                                     int32_t *acc, float *y,
                                     sp_stream_t stream);
+
+/* ---------------------------------------------------------------------------
+ * Continuous-input projections: the paper's other kernel (Section 2.3: for
+ * continuous inputs the INT8 weights are converted to FP32, multiplied with
+ * the FP32 activations and accumulated, and the row scale is applied after;
+ * Section 2.2: these projections keep ROW-MAJOR weights, one contiguous dot
+ * product per output).  For each problem and each activation row b < B:
+ *
+ *     y[b*ldy + m] = s_m * sum_{k<K} float(W[m*ldw + k]) * x[b*ldx + k]
+ *
+ * computed in FP32: each lane of a warp accumulates the products of its
+ * 16-column chunks (columns 16 l .. 16 l + 15 of every 512) with fmaf in
+ * ascending k, the 32 lane sums meet in a 5-level butterfly, and one FP32
+ * multiply applies s_m.  Each y is thus the FP32 value of a fixed summation
+ * tree of depth d <= 16 * ceil(K / 512) + 5, identical on every run, with
+ * |y - s_m * exact| <= |s_m| * gamma(d) * sum_k |W x| + u |y| (u = 2^-24,
+ * gamma(d) = d u / (1 - d u)).  Weights are read once per call for all B rows.
+ *
+ *   problems[j]  one projection (fields below); count in 1 ..
+ *                SPIKE_PROJ_DENSE_MAX_GROUP.  All run in ONE kernel launch.
+ *   B            activation rows, 1 .. SPIKE_PROJ_DENSE_MAX_B.
+ * Fields of sp_dense (device pointers, caller-owned, not retained):
+ *   W      INT8 row-major, element (m, k) at W[m*ldw + k]; 16-byte aligned;
+ *          ldw >= K, ldw % 16 == 0 (bytes past K in a row are never used).
+ *   scale  FP32 [N], one per output row; 4-byte aligned.
+ *   x      FP32, row b at x + b*ldx; 16-byte aligned; ldx >= K, ldx % 4 == 0.
+ *   y      FP32, row b at y + b*ldy; 4-byte aligned; ldy >= N.  Must not
+ *          overlap W, scale, x or another problem's y.
+ *   N, K   1 <= N; 1 <= K <= SPIKE_PROJ_MAX_K.
+ * Errors: SP_EINVAL, SP_EALIGN, SP_ERANGE, SP_EDEVICE, SP_ECUDA (nothing is
+ * enqueued on an error).  The kernel cannot fail once launched.
+ * ------------------------------------------------------------------------- */
+typedef struct sp_dense {
+    const int8_t *W;
+    int64_t ldw;
+    const float *scale;
+    const float *x;
+    int64_t ldx;
+    float *y;
+    int64_t ldy;
+    int32_t N;
+    int32_t K;
+} sp_dense;
+
+sp_status spike_proj_dense(const sp_dense *problems, int32_t count, int32_t B,
+                           sp_stream_t stream);
 
 /* --------------------------------------------------------------------------- */
 const char *spike_proj_strerror(sp_status status);

@@ -635,6 +635,28 @@ sp_status spike_proj_decode_noalloc(const int8_t* W, int64_t ldw, const float* s
   return SP_OK;
 }
 
+sp_status spike_proj_dense(const sp_dense* problems, int32_t count, int32_t B,
+                           sp_stream_t stream) {
+  if (!problems || count < 1 || count > SPIKE_PROJ_DENSE_MAX_GROUP || B < 1 ||
+      B > SPIKE_PROJ_DENSE_MAX_B)
+    return SP_EINVAL;
+  DenseProblem probs[kDenseMaxProblems];
+  for (int j = 0; j < count; ++j) {
+    const sp_dense& d = problems[j];
+    if (!d.W || !d.scale || !d.x || !d.y || d.N < 1 || d.K < 1 || d.ldy < d.N) return SP_EINVAL;
+    if (d.K > SPIKE_PROJ_MAX_K) return SP_ERANGE;
+    if (d.ldw < d.K || d.ldw % 16 != 0 || !aligned(d.W, 16)) return SP_EALIGN;
+    if (d.ldx < d.K || d.ldx % 4 != 0 || !aligned(d.x, 16)) return SP_EALIGN;
+    if (!aligned(d.scale, 4) || !aligned(d.y, 4)) return SP_EALIGN;
+    probs[j] = DenseProblem{d.W, d.ldw, d.scale, d.x, d.ldx, d.y, d.ldy, d.N, d.K};
+  }
+  int dev = 0;
+  const sp_status st = check_device(&dev);
+  if (st != SP_OK) return st;
+  SP_CUDA(launch_dense(probs, count, B, as_stream(stream)));
+  return SP_OK;
+}
+
 const char* spike_proj_strerror(sp_status status) {
   switch (status) {
     case SP_OK: return "success";

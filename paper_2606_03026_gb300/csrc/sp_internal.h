@@ -118,6 +118,21 @@ struct GemmParams {
   int32_t part_units;
 };
 
+// One continuous-input projection as the dense kernel sees it (row-major
+// INT8 weights, FP32 activations; see spike_proj_dense).
+struct DenseProblem {
+  const int8_t* W;
+  int64_t ldw;
+  const float* scale;
+  const float* x;
+  int64_t ldx;
+  float* y;
+  int64_t ldy;
+  int32_t N, K;
+};
+constexpr int kDenseMaxProblems = SPIKE_PROJ_DENSE_MAX_GROUP;
+cudaError_t launch_dense(const DenseProblem* probs, int count, int B, cudaStream_t s);
+
 // Launches `kernel` with programmatic stream serialization: its blocks may
 // become resident while the previous kernel of the stream is still running
 // and wait for it in pdl_wait (see sp_ptx.cuh) before touching memory.

@@ -23,6 +23,8 @@ SP_PLAN_GEMM = 0x1
 SPIKE_PROJ_MAX_K = 131072
 SPIKE_PROJ_MAX_GROUP = 64
 SPIKE_PROJ_NOALLOC_MAX_N = 32768
+SPIKE_PROJ_DENSE_MAX_B = 4
+SPIKE_PROJ_DENSE_MAX_GROUP = 128
 
 FMTS = {"bits": SP_SPIKES_BITS32, "u8": SP_SPIKES_U8, "bool8": SP_SPIKES_BOOL8}
 KERNELS = {"auto": SP_AUTO, "gather": SP_GATHER, "union": SP_UNION, "gemm": SP_GEMM}
@@ -47,6 +49,7 @@ _SIGNATURES = {
     "spike_proj_group_status": ([_P, _P], ctypes.c_int),
     "spike_proj_decode_noalloc": ([_P, _I64, _P, _I32, _I32, _P, ctypes.c_int, _P, _P, _P],
                                   ctypes.c_int),
+    "spike_proj_dense": ([_P, _I32, _I32, _P], ctypes.c_int),
     "spike_proj_strerror": ([ctypes.c_int], ctypes.c_char_p),
     "spike_proj_last_cuda_error": ([], ctypes.c_int),
     "spike_proj_abi_version": ([], ctypes.c_int),
@@ -188,6 +191,34 @@ def spike_proj_group_decode_host(group, h_spikes, fmt, ld_spikes, h_acc=None, h_
 
 def spike_proj_group_status(group, stream=None) -> int:
     return lib().spike_proj_group_status(group, _stream(stream))
+
+
+class SpDense(ctypes.Structure):
+    """struct sp_dense of spike_proj.h (one continuous-input projection)."""
+    _fields_ = [("W", ctypes.c_void_p), ("ldw", ctypes.c_int64), ("scale", ctypes.c_void_p),
+                ("x", ctypes.c_void_p), ("ldx", ctypes.c_int64), ("y", ctypes.c_void_p),
+                ("ldy", ctypes.c_int64), ("N", ctypes.c_int32), ("K", ctypes.c_int32)]
+
+
+def spike_proj_dense(problems, B, stream=None):
+    """problems: sequence of (W, ldw, scale, x, ldx, y, ldy, N, K), the fields
+    of struct sp_dense (tensors or addresses); all run in one launch."""
+    arr = (SpDense * len(problems))()
+    for i, (W, ldw, scale, x, ldx, y, ldy, N, K) in enumerate(problems):
+        arr[i] = SpDense(_addr(W), ldw, _addr(scale), _addr(x), ldx, _addr(y), ldy, N, K)
+    _check(lib().spike_proj_dense(ctypes.addressof(arr), len(problems), B, _stream(stream)),
+           "spike_proj_dense")
+
+
+def dense(W, scale, x, y, K=None, stream=None):
+    """One continuous-input projection: W int8 [N, ldw] row-major, scale
+    float32 [N], x float32 [B, ldx], y float32 [B, ldy] (torch tensors)."""
+    N, ldw = W.shape
+    xs = x if x.dim() == 2 else x.reshape(1, -1)
+    ys = y if y.dim() == 2 else y.reshape(1, -1)
+    K = ldw if K is None else K
+    spike_proj_dense([(W, ldw, scale, xs, xs.stride(0), ys, ys.stride(0), N, K)], xs.shape[0],
+                     stream)
 
 
 def spike_proj_decode_noalloc(W, ldw, scale, N, K, spikes, fmt, acc=None, y=None,

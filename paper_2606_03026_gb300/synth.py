@@ -31,7 +31,7 @@ D_FFN = 4 * D_MODEL       # 6144: down-projection input width, Appendix A.2
 N_BLOCKS = 22             # decoder blocks, Section 2.1
 
 # workload ids used as the first word of every seed sequence
-_W_SINGLE, _W_DOWN, _W_STEP, _W_BATCH, _W_PREFILL, _W_MISC = 1, 2, 3, 4, 5, 9
+_W_SINGLE, _W_DOWN, _W_STEP, _W_BATCH, _W_PREFILL, _W_DENSE, _W_MISC = 1, 2, 3, 4, 5, 6, 9
 
 
 def rng_for(*words: int) -> np.random.Generator:
@@ -215,3 +215,27 @@ def random_case(seed: int, N: int, K: int, T: int = 1, p: float = 0.1,
     s = rng.uniform(-2.0, 2.0, size=N).astype(np.float32)
     x = bernoulli(rng, (T, K), p)
     return np.ascontiguousarray(Q), s, x
+
+
+# --------------------------------------------------------------------------
+# continuous-input projections (row-major INT8 weights, FP32 activations)
+# --------------------------------------------------------------------------
+# Per block, the projections that read the continuous stream (Section 2.1):
+# fused query/key/value (3 x 1536 out), attention output (1536 out) and FFN up
+# (6144 out), all with 1536 inputs.  The paper does not give their exact
+# shapes; these follow the stated residual width and FFN width.
+DENSE_KINDS = {"qkv": 3 * D_MODEL, "out": D_MODEL, "up": D_FFN}
+
+
+def dense_weights(block: int, kind: str, seed: int = 0, K: int = D_MODEL):
+    """Row-major INT8 weights [N, K] and scale [N] of one continuous-input
+    projection of block ``block``: N(0, 1) exported per output channel
+    (the same export as the spike-gated weights, transposed to row-major)."""
+    N = DENSE_KINDS[kind]
+    Qc, s = quantised_normal(rng_for(_W_DENSE, seed, block, list(DENSE_KINDS).index(kind)), N, K)
+    return np.ascontiguousarray(Qc.T), s
+
+
+def hidden_state(step: int, B: int = 1, seed: int = 0, K: int = D_MODEL):
+    """Continuous activations x ~ N(0, 1), float32 [B, K]."""
+    return rng_for(_W_DENSE, seed, 10_000 + step).standard_normal((B, K), dtype=np.float32)

@@ -71,6 +71,13 @@ def test_host_only_calls(lib):
         spikeproj.SP_EINVAL                # unknown flag
     assert lib.spike_proj_decode(None, fake, 0, fake, fake, None) == spikeproj.SP_EINVAL
     assert lib.spike_proj_group_create(None, None, 0, None) == spikeproj.SP_EINVAL
+    assert lib.spike_proj_dense(None, 1, 1, None) == spikeproj.SP_EINVAL
+    d = spikeproj.SpDense(fake, 32, fake, fake, 32, fake, 16, 16, 32)
+    assert lib.spike_proj_dense(ctypes.addressof(d), 1, 0, None) == spikeproj.SP_EINVAL   # B = 0
+    d.ldw = 24
+    assert lib.spike_proj_dense(ctypes.addressof(d), 1, 1, None) == spikeproj.SP_EALIGN   # ldw % 16
+    d.ldw, d.W = 32, fake + 4
+    assert lib.spike_proj_dense(ctypes.addressof(d), 1, 1, None) == spikeproj.SP_EALIGN   # W alignment
     assert lib.spike_proj_plan_destroy(None) == spikeproj.SP_OK
     assert lib.spike_proj_group_destroy(None) == spikeproj.SP_OK
 
