@@ -3,6 +3,7 @@
 // and tensor-core kernels, and status reporting.  See include/spike_proj.h.
 #include <atomic>
 #include <cstdlib>
+#include <algorithm>
 #include <cstring>
 #include <mutex>
 #include <new>
@@ -246,17 +247,19 @@ sp_status run_gemm(sp_plan_s* p, const void* spikes, int fmt, int T, int64_t ld,
 
 // Measured-density dispatch between the per-token gather and the
 // tensor-core GEMM, by a cost model fitted on GB300 (K = 6144, N = 1536,
-// token rates U(0.05, 0.2), B = 2 .. 1024, weights L2-resident):
-//   gather ~ 6 us + active bytes (sum_t |A_t| * N) / 6.3 TB/s
-//   GEMM   ~ 12 us + 2 B N K ops / 1 PFLOP/s            (plans with SP_PLAN_GEMM)
-// The crossover lies between B = 32 and B = 64 at these rates.  The union
-// fetch is never chosen automatically: it was slower than the per-token
-// gather at every batch size measured (its adds are ALU-bound, and the
-// 126 MB L2 serves the per-token re-reads of a 9.4 MB weight matrix).
+// token rates U(0.05, 0.2), B = 1 .. 1024, weights L2-resident, graph-timed):
+//   gather ~ 5 us + active bytes (sum_t |A_t| * N) / 6.7 TB/s
+//   GEMM   ~ max(12.1 us, 11.3 us + 2 B N K ops / 1.4 PFLOP/s)   (SP_PLAN_GEMM plans)
+// (the e4m3 GEMM is flat at 12.1-12.3 us up to B = 128 and takes 25 us at
+// B = 1024).  The crossover lies near 31 k active columns, B ~ 36 at these
+// rates (measured: B = 32 gather 11.3 us / GEMM 12.3 us, B = 48 14.5 / 12.2).
+// The union fetch is never chosen automatically: it was slower than the
+// per-token gather at every batch size measured (its adds are ALU-bound, and
+// the 126 MB L2 serves the per-token re-reads of a 9.4 MB weight matrix).
 sp_kernel choose(const sp_plan_s* p, int B, int32_t total) {
   if (!(p->flags & SP_PLAN_GEMM)) return SP_GATHER;
-  const double gather_us = 6.0 + (double)total * p->N / 6.3e6;
-  const double gemm_us = 12.0 + 2.0 * B * (double)p->N * p->K / 1.0e9;
+  const double gather_us = 5.0 + (double)total * p->N / 6.7e6;
+  const double gemm_us = std::max(12.1, 11.3 + 2.0 * B * (double)p->N * p->K / 1.4e9);
   return gemm_us < gather_us ? SP_GEMM : SP_GATHER;
 }
 
