@@ -145,6 +145,28 @@ def test_gemm_extremes():
             assert_parity(acc, y, want_acc, want_y, f"gemm extremes {c} {other} {fmt}")
 
 
+def test_gemm_largest_k():
+    """K = SPIKE_PROJ_MAX_K on the tensor-core path: all-ones spikes against
+    -128 weights give acc = -2^24 exactly (the exactness boundary), and
+    +127 / +1 mixes give large odd sums; K is split 8 ways here."""
+    T, N, K = 130, 64, sp.SPIKE_PROJ_MAX_K
+    X = np.ones((T, K), np.uint8)
+    X[1::2, ::7] = 0
+    s = np.linspace(-1, 1, N).astype(np.float32)
+    for c, other in ((-128, -128), (127, 1)):
+        Qc = np.full((K, N), c, np.int8)
+        Qc[::3] = other
+        want_acc, want_y = oracle.project(Qc, s, N, K, X, "u8")
+        if c == -128:
+            assert int(want_acc[0, 0]) == -(1 << 24)
+        plan = sp.Plan(to_dev(Qc), to_dev(s), N, K, max_batch=T, gemm=True)
+        for fmt in ("bool8", "u8"):
+            acc, y = run_batched(plan, to_dev(X), fmt, T, K, N, "gemm")
+            assert_parity(acc, y, want_acc, want_y, f"gemm K max {c} {fmt}")
+        assert plan.status() == sp.SP_OK
+        plan.close()
+
+
 def test_auto_dispatch_by_cost(down):
     """SP_AUTO: per-token gather for small batches, the tensor-core GEMM for
     large ones on a plan with SP_PLAN_GEMM, never the GEMM without it; the

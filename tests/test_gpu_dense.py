@@ -70,6 +70,20 @@ def test_dense_vs_oracle(N, K, B):
     check(y, W, x, s, N, K, ldw, f"N={N} K={K} B={B}")
 
 
+def test_dense_largest_k():
+    """K = SPIKE_PROJ_MAX_K (the tree is 16 * 256 + 5 deep) within its bound,
+    and an exact case: constant weights and activations 1/4 (every partial
+    sum a small dyadic multiple, exact in FP32)."""
+    N, K, B = 9, sp.SPIKE_PROJ_MAX_K, 2
+    W, x, s, ldw, ldx = case(77, N, K, B)
+    y, = run([(W, x, s, N, K, ldw, ldx)], B)
+    check(y, W, x, s, N, K, ldw, "K max")
+    W = np.full((N, ldw), -3, np.int8)
+    x = np.full((B, ldx), 0.25, np.float32)
+    y, = run([(W, x, s, N, K, ldw, ldx)], B)
+    assert np.array_equal(y, np.broadcast_to(s * np.float32(-0.75 * K), (B, N)))
+
+
 def test_dense_group_mixed_shapes():
     """Many problems of different shapes in one launch (unit boundaries
     inside and across problems)."""
