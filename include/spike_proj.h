@@ -184,6 +184,9 @@ sp_status spike_proj_batched(sp_plan_t plan, const void *spikes, sp_fmt fmt,
  *   strategy   as for spike_proj_batched; SP_AUTO picks SP_GEMM on a plan
  *              with SP_PLAN_GEMM when the measured density makes the dense
  *              contraction cheaper than the gathers.
+ * On SP_GEMM these rows first go through the 0/1 staging pass (any nonzero
+ * byte fires); rows already holding exactly 0 / 1 (a torch.bool tensor) can
+ * skip it: spike_proj_batched with SP_SPIKES_BOOL8 reads them in place.
  * ------------------------------------------------------------------------- */
 sp_status spike_proj_prefill(sp_plan_t plan, const uint8_t *X, int32_t T,
                              int64_t ldx, int32_t *acc, float *y,
