@@ -12,9 +12,11 @@
 //      the shared-memory segment into biased 16-bit lanes (lane = 8 channels;
 //      at most 256 columns per chunk, so the lanes cannot overflow),
 //   4. single-chunk problems write acc / y directly; otherwise the row sums go
-//      into the INT32 workspace with red.add and the CTA that completes an
-//      output tile (atomic ticket) applies y = s * float(acc) for every row and
-//      re-zeroes the workspace.  Nothing waits on another CTA.
+//      into the workspace as fp32 with 16-byte red.add (exact: integers below
+//      2^24), and the CTA that completes an output tile (atomic ticket) reads
+//      the tile back in 16-byte groups, 16 loads per thread in flight, writes
+//      acc and y = s * float(acc) for every row, and re-zeroes the workspace.
+//      Nothing waits on another CTA.
 #include "sp_spikes.cuh"
 
 namespace sp {
@@ -28,6 +30,11 @@ constexpr size_t kUnionSmem = kUnionSmemTile + kUnionSmemMask;
 __device__ __forceinline__ void cp_async16(void* smem, const void* gmem) {
   const uint32_t s = static_cast<uint32_t>(__cvta_generic_to_shared(smem));
   asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(s), "l"(gmem) : "memory");
+}
+__device__ __forceinline__ void red_add_v4(float* addr, float a, float b, float c, float d) {
+  asm volatile("red.relaxed.gpu.global.add.v4.f32 [%0], {%1, %2, %3, %4};" ::"l"(addr), "f"(a),
+               "f"(b), "f"(c), "f"(d)
+               : "memory");
 }
 __device__ __forceinline__ void cp_async_wait_all() {
   asm volatile("cp.async.wait_all;" ::: "memory");
@@ -117,10 +124,12 @@ union_kernel(const __grid_constant__ UnionParams p) {
             if (p.y) p.y[(int64_t)t * p.N + ch + q] = scale_out(__ldg(p.scale + ch + q), o[q]);
           }
         } else {
-          int32_t* ws = p.ws + (int64_t)t * p.N + ch;
-#pragma unroll
-          for (int q = 0; q < 8; ++q)
-            if (o[q]) atomicAdd(ws + q, o[q]);
+          // integer partials below 2^24 added as fp32 (exact), 16 bytes at a time
+          float* ws = reinterpret_cast<float*>(p.ws) + (int64_t)t * p.N + ch;
+          if (o[0] | o[1] | o[2] | o[3])
+            red_add_v4(ws, (float)o[0], (float)o[1], (float)o[2], (float)o[3]);
+          if (o[4] | o[5] | o[6] | o[7])
+            red_add_v4(ws + 4, (float)o[4], (float)o[5], (float)o[6], (float)o[7]);
         }
       }
     }
@@ -138,15 +147,52 @@ union_kernel(const __grid_constant__ UnionParams p) {
       __syncthreads();
       if (s_last) {
         __threadfence();
-        const int width = min(kUnionNT, p.N - n0);
-        for (int i = threadIdx.x; i < p.B * width; i += kUnionThreads) {
-          const int t = i / width;
-          const int n = n0 + (i - t * width);
-          int32_t* wsp = p.ws + (int64_t)t * p.N + n;
-          const int v = __ldcg(wsp);
-          __stcg(wsp, 0);
-          if (p.acc) p.acc[(int64_t)t * p.N + n] = v;
-          if (p.y) p.y[(int64_t)t * p.N + n] = scale_out(__ldg(p.scale + n), v);
+        // every (row, 4-channel group) of the tile: N % 16 == 0, so groups
+        // never straddle N; 16 loads of each thread in flight before any store
+        const int groups = min(kUnionNT, p.N - n0) / 4;
+        const int total = p.B * groups;
+        constexpr int kBatch = 16;
+        // acc / y may be only 4-byte aligned (rows are 64-byte multiples apart)
+        const bool vec_out = ((reinterpret_cast<uintptr_t>(p.acc) | reinterpret_cast<uintptr_t>(p.y)) & 15u) == 0;
+        for (int i0 = threadIdx.x; i0 < total; i0 += kUnionThreads * kBatch) {
+          float4 v[kBatch];
+#pragma unroll
+          for (int j = 0; j < kBatch; ++j) {
+            const int i = i0 + j * kUnionThreads;
+            if (i < total) {
+              const int t = i / groups;
+              const int n = n0 + 4 * (i - t * groups);
+              v[j] = __ldcg(reinterpret_cast<const float4*>(reinterpret_cast<float*>(p.ws) +
+                                                              (int64_t)t * p.N + n));
+            }
+          }
+#pragma unroll
+          for (int j = 0; j < kBatch; ++j) {
+            const int i = i0 + j * kUnionThreads;
+            if (i < total) {
+              const int t = i / groups;
+              const int n = n0 + 4 * (i - t * groups);
+              __stcg(reinterpret_cast<float4*>(reinterpret_cast<float*>(p.ws) + (int64_t)t * p.N + n),
+                     make_float4(0.f, 0.f, 0.f, 0.f));
+              const int o[4] = {__float2int_rn(v[j].x), __float2int_rn(v[j].y), __float2int_rn(v[j].z),
+                                __float2int_rn(v[j].w)};
+              int32_t* acc_row = p.acc ? p.acc + (int64_t)t * p.N : nullptr;
+              float* y_row = p.y ? p.y + (int64_t)t * p.N : nullptr;
+              if (vec_out) {
+                if (acc_row) *reinterpret_cast<int4*>(acc_row + n) = make_int4(o[0], o[1], o[2], o[3]);
+                if (y_row)
+                  *reinterpret_cast<float4*>(y_row + n) =
+                      make_float4(scale_out(__ldg(p.scale + n), o[0]), scale_out(__ldg(p.scale + n + 1), o[1]),
+                                  scale_out(__ldg(p.scale + n + 2), o[2]), scale_out(__ldg(p.scale + n + 3), o[3]));
+              } else {
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                  if (acc_row) acc_row[n + q] = o[q];
+                  if (y_row) y_row[n + q] = scale_out(__ldg(p.scale + n + q), o[q]);
+                }
+              }
+            }
+          }
         }
       }
     }
