@@ -735,9 +735,8 @@ def bench_dense(torch, sp, synth, dev, stream, peaks, peak_kind, world, blocks=2
                         "kernel": "dense_kernel<1> (66 projections, one launch)",
                         "peak_kind": peak_kind},
            "B_sweep": sweep,
-           "note": "B = 2-4 reuse each weight byte for B FMAs; the registers those take "
-                   "(127-215 per thread) leave 8-16 warps per SM, and the kernel runs below both "
-                   "the HBM rate and the FP32 issue rate (latency-bound)"}
+           "note": "B = 2-4 reuse each converted weight for B FMAs at 2 CTAs per SM; they run "
+                   "below both the HBM rate and the FP32 issue rate (latency-bound)"}
     if with_oracle:
         W, s = srcs["up"]
         N, K = W.shape

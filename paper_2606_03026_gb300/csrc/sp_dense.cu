@@ -14,7 +14,7 @@
 // A unit is 4 consecutive rows of one problem, owned by one warp.  Lane l
 // covers the 16-column chunks l, l + 32, l + 64, ... of the row (16-byte
 // weight loads, 512 contiguous bytes per warp instruction), issuing the loads
-// of 1 (B = 1) or 3 (B > 1) chunks of all 4 rows before any arithmetic.  A weight byte
+// of one chunk of all 4 rows before any arithmetic.  A weight byte
 // becomes a float exactly through its bias (w + 128 in the low byte of 2^23's
 // mantissa, minus 2^23 + 128).  Each lane accumulates with fmaf in ascending
 // k, the 32 lane sums meet in a 5-level butterfly, and one FP32 multiply by s_m
@@ -30,14 +30,14 @@ namespace {
 constexpr int kDenseRows = 4;        // rows per unit (one warp)
 constexpr int kDenseThreads = 256;
 // Per activation count B: 16-column chunks per lane loaded per round, and
-// CTAs per SM the registers must allow.  With one activation row the FMA
-// work per byte is small, and 32 warps per SM with one chunk of 4 rows in
-// flight each (63 registers) stream faster than 16 warps with three chunks
-// (measured on the 22-block step: 5.1 against 3.6 TB/s).  More activation
-// rows need the registers for their partial sums and x values.
-template <int B> struct DenseShape { static constexpr int batch = 3, min_ctas = 1; };
+// CTAs per SM the registers must allow.  One chunk of 4 rows per round: the
+// converted weights stay in registers for the B activation rows, and more
+// warps with less in flight each stream faster than fewer warps with three
+// chunks (measured on the 22-block step: B = 1 at 32 warps per SM 5.1 TB/s
+// against 3.6 with three chunks; B = 2 / 3 / 4 at 16 warps per SM 2.9 / 2.3 /
+// 1.7 TB/s against 2.5 / 1.6 / 1.3).
+template <int B> struct DenseShape { static constexpr int batch = 1, min_ctas = 2; };
 template <> struct DenseShape<1> { static constexpr int batch = 1, min_ctas = 4; };
-template <> struct DenseShape<2> { static constexpr int batch = 3, min_ctas = 2; };
 
 struct DenseParams {
   int32_t count, B;
