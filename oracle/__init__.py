@@ -12,6 +12,8 @@ Functions mirror ``spike_oracle.h``:
   to INT32, ``y_m = s_m * float32(acc_m)`` (Eq. sparse and the sentence after
   it), for T spike rows.
 * :func:`project_entries` -- the same at selected (row, channel) pairs.
+* :func:`lif` -- one leaky integrate-and-fire step producing spike rows in
+  the ``"bits"`` format (a stated reading: the paper names LIF only).
 * :func:`dense` -- the continuous-input projection over row-major INT8
   weights, ``y_m = s_m * sum_k Q[m*ldq + k] * x_k`` evaluated in double, with
   ``sum_k |Q_mk x_k|`` for error bounds (Section 2.3, the sentence on
@@ -89,6 +91,8 @@ class Oracle:
         lib.sp_oracle_project_entries.restype = ctypes.c_int
         lib.sp_oracle_dense.argtypes = [p, i64, p, i32, i32, p, i64, i32, p, p]
         lib.sp_oracle_dense.restype = ctypes.c_int
+        lib.sp_oracle_lif.argtypes = [p, p, i32, i32, i64, ctypes.c_float, ctypes.c_float, p, i64]
+        lib.sp_oracle_lif.restype = ctypes.c_int
         self.lib = lib
 
     # -- helpers -----------------------------------------------------------
@@ -202,6 +206,25 @@ class Oracle:
         return y, mag
 
 
+    def lif(self, v: np.ndarray, I: np.ndarray, K: int, beta: float, theta: float):
+        """One LIF step of every row of ``v`` / ``I`` (float32 [T, >=K]);
+        returns (v_new float32 [T, ld], bits uint32 [T, ceil(K/32)])."""
+        v = np.array(v, dtype=np.float32, copy=True, ndmin=2, order="C")
+        I = np.ascontiguousarray(I, dtype=np.float32)
+        if I.ndim == 1:
+            I = I[None, :]
+        if v.shape != I.shape or v.shape[1] < K:
+            raise ValueError("v and I must have the same shape, rows >= K")
+        T, ld = v.shape
+        words = (K + 31) // 32
+        bits = np.full((T, max(words, 1)), 0xA5A5A5A5, dtype=np.uint32)
+        rc = self.lib.sp_oracle_lif(v.ctypes.data, I.ctypes.data, K, T, ld, beta, theta,
+                                    bits.ctypes.data, bits.shape[1])
+        if rc:
+            raise RuntimeError(f"sp_oracle_lif failed: {rc}")
+        return v, bits[:, :words]
+
+
 _DEFAULT: Oracle | None = None
 
 
@@ -228,3 +251,7 @@ def project_entries(Q, scale, N, K, spikes, fmt, t_idx, m_idx, ldq=None):
 
 def dense(Q, scale, N, K, x, ldq=None):
     return default().dense(Q, scale, N, K, x, ldq)
+
+
+def lif(v, I, K, beta, theta):
+    return default().lif(v, I, K, beta, theta)

@@ -25,6 +25,7 @@
  */
 #include "spike_oracle.h"
 
+#include <math.h>
 #include <stdlib.h>
 
 /* Spike x_k of one row: 1 if column k fires, else 0 (Section 1: x in {0,1}^K;
@@ -173,6 +174,32 @@ int sp_oracle_dense(const int8_t *Q, int64_t ldq, const float *s,
                 y[(int64_t)t * N + m] = (double)s[m] * dot;
             if (abs_dot)
                 abs_dot[(int64_t)t * N + m] = mag;
+        }
+    }
+    return 0;
+}
+
+/* One LIF step and the spike bits, as stated in spike_oracle.h (a reading:
+ * the paper does not give the update). */
+int sp_oracle_lif(float *v, const float *I, int32_t K, int32_t T, int64_t ld,
+                  float beta, float theta, uint32_t *bits, int64_t ld_bits)
+{
+    const int64_t words = ((int64_t)K + 31) / 32;
+    if (!v || !I || !bits || K < 0 || T < 0 || (T > 1 && (ld < K || ld_bits < words)))
+        return -1;
+    for (int32_t t = 0; t < T; ++t) {
+        float *vt = v + (int64_t)t * ld;
+        const float *it = I + (int64_t)t * ld;
+        uint32_t *bt = bits + (int64_t)t * ld_bits;
+        for (int64_t w = 0; w < words; ++w)
+            bt[w] = 0u;
+        for (int32_t k = 0; k < K; ++k) {
+            float u = fmaf(beta, vt[k], it[k]);
+            if (u >= theta) {
+                bt[k / 32] |= 1u << (k % 32);
+                u = u - theta;
+            }
+            vt[k] = u;
         }
     }
     return 0;

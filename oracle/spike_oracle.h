@@ -22,8 +22,9 @@
  * spike; SP_ORACLE_BITS32 -- uint32 words, column k is bit (k % 32) of word
  * (k / 32), bits at or beyond K are ignored.
  *
- * sp_oracle_dense (declared last) is the paper's other kernel: the
- * continuous-input projection over row-major INT8 weights.
+ * sp_oracle_dense is the paper's other kernel: the continuous-input
+ * projection over row-major INT8 weights.  sp_oracle_lif (declared last)
+ * produces spike rows in the BITS32 format from a LIF state.
  *
  * All functions are single-threaded, allocate only O(K) scratch, and return
  * 0 on success, a negative code on a bad argument (-1) or an INT32 overflow of
@@ -82,6 +83,20 @@ int sp_oracle_project_entries(const int8_t *Q, int64_t ldq, const float *s,
 int sp_oracle_dense(const int8_t *Q, int64_t ldq, const float *s,
                     int32_t N, int32_t K, const float *x, int64_t ldx,
                     int32_t T, double *y, double *abs_dot);
+
+/* Spike producer: one leaky integrate-and-fire step for T rows of K neurons,
+ * written straight into the SP_ORACLE_BITS32 format.  The paper names LIF
+ * dynamics (Section 1) without stating the update, so this is a reading:
+ *
+ *     v  <- fmaf(beta, v, I)            one FP32 fused multiply-add
+ *     x  =  (v >= theta)                the spike
+ *     v  <- v - theta   where x = 1     soft reset, one FP32 subtract
+ *
+ * Row t of v and I starts at element t * ld; row t of the bits at word
+ * t * ld_bits (ceil(K/32) words: bit k % 32 of word k / 32, LSB first, bits at
+ * or past K written as 0).  v is updated in place. */
+int sp_oracle_lif(float *v, const float *I, int32_t K, int32_t T, int64_t ld,
+                  float beta, float theta, uint32_t *bits, int64_t ld_bits);
 
 #ifdef __cplusplus
 }

@@ -26,6 +26,13 @@ matmul with padded row strides, closed forms (constant Q and x, one-hot,
 zero, extremes), linearity on dyadic inputs (exact in double), and, for
 0/1 inputs, exact agreement with the spike-gated projection of the same
 matrix.
+
+The spike producer (one LIF step of the stated reading, written as BITS32
+rows) is pinned by a hand-worked fixture (tests/golden/hand_worked_lif.json),
+an exactly periodic closed form, cases where a fused multiply-add and a
+separate multiply then add round differently (exact rational arithmetic
+rounded to FP32), the bit format and cleared tail bits via the spike
+oracle's own unpacking, row strides, and an infinite threshold.
 """
 from __future__ import annotations
 
@@ -295,8 +302,89 @@ def pin_dense_binary_is_sparse(orc):
     assert np.array_equal(yd.astype(np.float32), ysp)
 
 
+# --- spike producer (LIF step) -------------------------------------------------
+
+def rn32(q):
+    """A rational rounded to the nearest float32, ties to even (exact)."""
+    from fractions import Fraction
+    f = np.float32(float(q))
+    best = None
+    for c in (np.nextafter(f, np.float32(-np.inf)), f, np.nextafter(f, np.float32(np.inf))):
+        d = abs(Fraction(float(c)) - q)
+        key = (d, int(np.array(c, np.float32).view(np.uint32)) & 1)
+        if best is None or key < best[0]:
+            best = (key, c)
+    return np.float32(best[1])
+
+
+def pin_lif_hand_fixture(orc):
+    g = json.loads((GOLDEN / "hand_worked_lif.json").read_text())
+    v, bits = orc.lif(np.array(g["v"], np.float32), np.array(g["I"], np.float32), g["K"],
+                      g["beta"], g["theta"])
+    assert v[0].tolist() == g["v_new"], v
+    assert bits[0].tolist() == g["bits"], bits
+
+
+def pin_lif_periodic(orc):
+    # beta = 1/2, I = 1, theta = 7/4: v = 1, 3/2, 7/4 -> spike, 0, ... (all exact),
+    # so every neuron fires on steps 2, 5, 8, ... and ends a step at v = 0 there
+    K, T = 70, 3
+    v = np.zeros((T, 72), np.float32)
+    I = np.ones((T, 72), np.float32)
+    v[:, K:] = 123.0                       # row padding: never touched
+    for step in range(30):
+        v, bits = orc.lif(v, I, K, 0.5, 1.75)
+        fire = step % 3 == 2
+        want = np.zeros(3, np.uint32)
+        if fire:
+            want[:] = [0xFFFFFFFF, 0xFFFFFFFF, (1 << 6) - 1]
+        assert np.array_equal(bits, np.broadcast_to(want, (T, 3))), step
+        assert np.all(v[:, :K] == [1.0, 1.5, 0.0][step % 3]), step
+        assert np.all(v[:, K:] == 123.0)
+
+
+def pin_lif_fma_rounding(orc):
+    # beta * v + I with one rounding: exact rationals rounded once to FP32;
+    # the inputs are chosen so that rounding the product first would differ
+    from fractions import Fraction
+    rng = synth.rng_for(310)
+    cases = []
+    while len(cases) < 16:
+        b, v0, i0 = (np.float32(rng.uniform(0.5, 1.0)), np.float32(rng.normal()),
+                     np.float32(rng.normal()))
+        exact = Fraction(float(b)) * Fraction(float(v0)) + Fraction(float(i0))
+        if rn32(exact) != np.float32(np.float32(b * v0) + i0):
+            cases.append((b, v0, i0, rn32(exact)))
+    for b, v0, i0, want in cases:
+        v, bits = orc.lif(np.array([v0], np.float32), np.array([i0], np.float32), 1, float(b),
+                          float("inf"))
+        assert v[0, 0] == want and bits[0, 0] == 0, (b, v0, i0, v[0, 0], want)
+
+
+def pin_lif_bits_format(orc):
+    # dyadic inputs: beta * v + I is exact, so the spikes are known; the bits
+    # must unpack (through the spike oracle) to exactly those columns, and the
+    # words past K must be zero
+    K = 83
+    rng = synth.rng_for(311)
+    v = (rng.integers(-64, 64, (4, K)) / 32).astype(np.float32)
+    I = (rng.integers(-64, 64, (4, K)) / 32).astype(np.float32)
+    pre = 0.75 * v.astype(np.float64) + I.astype(np.float64)
+    vn, bits = orc.lif(v, I, K, 0.75, 0.5)
+    for t in range(4):
+        fired = np.flatnonzero(pre[t] >= 0.5)
+        assert np.array_equal(orc.active_set(bits[t], "bits", K), fired), t
+        assert (int(bits[t, -1]) >> (K % 32)) == 0, "tail bits set"
+        want_v = np.where(pre[t] >= 0.5, pre[t] - 0.5, pre[t]).astype(np.float32)
+        assert np.array_equal(vn[t], want_v), t
+    # an infinite threshold never fires
+    _, bits = orc.lif(v, I, K, 0.75, float("inf"))
+    assert not bits.any()
+
+
 ALL_PINS = [pin_hand_fixture, pin_exhaustive_small, pin_full_shapes,
             pin_scale_rounding, pin_invariants, pin_closed_forms,
             pin_overflow_reported, pin_entries,
             pin_dense_hand_fixture, pin_dense_matmul, pin_dense_closed_forms,
-            pin_dense_linearity, pin_dense_binary_is_sparse]
+            pin_dense_linearity, pin_dense_binary_is_sparse,
+            pin_lif_hand_fixture, pin_lif_periodic, pin_lif_fma_rounding, pin_lif_bits_format]

@@ -34,6 +34,14 @@ MUTANTS = {
     "dense_scale_dropped": ("y[(int64_t)t * N + m] = (double)s[m] * dot;", "y[(int64_t)t * N + m] = dot;"),
     "dense_abs_signed": ("mag += term < 0 ? -term : term;", "mag += term;"),
     "dense_float_accumulator": ("double dot = 0.0, mag = 0.0;", "float dot = 0.0f; double mag = 0.0;"),
+    # spike producer (LIF step)
+    "lif_multiply_then_add": ("float u = fmaf(beta, vt[k], it[k]);", "float u = beta * vt[k] + it[k];"),
+    "lif_strict_threshold": ("if (u >= theta) {", "if (u > theta) {"),
+    "lif_hard_reset": ("u = u - theta;", "u = 0.0f;"),
+    "lif_no_reset": ("u = u - theta;", ""),
+    "lif_msb_first": ("bt[k / 32] |= 1u << (k % 32);", "bt[k / 32] |= 1u << (31 - k % 32);"),
+    "lif_tail_kept": ("for (int64_t w = 0; w < words; ++w)\n            bt[w] = 0u;", ""),
+    "lif_row_stride_ignored": ("float *vt = v + (int64_t)t * ld;", "float *vt = v + (int64_t)t * K;"),
 }
 
 
