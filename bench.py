@@ -71,6 +71,8 @@ def parse():
     ap.add_argument("--no-prefill", action="store_true")
     ap.add_argument("--no-dense", action="store_true",
                     help="skip the continuous-input projections section")
+    ap.add_argument("--no-lif", action="store_true",
+                    help="skip the spike-producer section")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
     ap.add_argument("--e2e-steps", type=int, default=6400)
@@ -457,6 +459,10 @@ def run_ours(args):
                                           args.prefill_blocks)
         result["gpu_launches"] = steps   # prefill is timed outside the headline region
 
+    if not args.no_lif:
+        result["lif"] = bench_lif(torch, sp, synth, dev, stream, copies, weights, acc, y, peaks,
+                                  peak_kind)
+
     if not args.no_dense:
         result["dense"] = bench_dense(torch, sp, synth, dev, stream, peaks, peak_kind, world,
                                       with_oracle=rank == 0 and not args.no_cpu_baseline)
@@ -655,6 +661,105 @@ def measured_traffic(kernel, source):
         return float(rec["dram_bytes_per_launch"])
     except (OSError, KeyError, ValueError):
         return None
+
+
+def bench_lif(torch, sp, synth, dev, stream, copies, weights, acc, y, peaks, peak_kind):
+    """Spike producer: the decode step with its 44 spike rows made on the
+    GPU by one LIF step per layer (spike_proj_lif for the 22 TCAM inputs of
+    1536 neurons and the 22 down-projection inputs of 6144 neurons, written
+    into the rows the group reads), then the grouped decode, graph-replayed.
+    Currents are drawn fresh for every step (64 rotating sets of
+    N(0.135, 0.3), a stationary rate near 10% with beta = 0.9, theta = 1);
+    the warm-up replays reach that rate before timing.  Also the producer
+    alone on the step, and on a 400 MB state (its HBM roofline)."""
+    import oracle
+    n = len(weights)
+    words = 6144 // 32
+    beta, theta = 0.9, 1.0
+    sets = 64
+    rng = synth.rng_for(9100)
+    v_t = torch.zeros((n // 2, 1536), dtype=torch.float32, device=dev)
+    v_d = torch.zeros((n // 2, 6144), dtype=torch.float32, device=dev)
+    i_t = torch.from_numpy(rng.normal(0.135, 0.3, (sets, n // 2, 1536)).astype(np.float32)).to(dev)
+    i_d = torch.from_numpy(rng.normal(0.135, 0.3, (sets, n // 2, 6144)).astype(np.float32)).to(dev)
+    bits = torch.zeros((n, words), dtype=torch.int32, device=dev)
+    # rows of the group's spike input: projection j = 2b (TCAM) or 2b + 1 (down)
+    bits_t, bits_d = bits[0::2], bits[1::2]
+
+    def produce(i, s):
+        sp.spike_proj_lif(v_t, i_t[i % sets], 1536, n // 2, 1536, beta, theta, bits_t, 2 * words, s)
+        sp.spike_proj_lif(v_d, i_d[i % sets], 6144, n // 2, 6144, beta, theta, bits_d, 2 * words, s)
+
+    # spot check of one producer step against the oracle
+    v0 = v_d.cpu().numpy()
+    with torch.cuda.stream(stream):
+        produce(0, stream)
+    stream.synchronize()
+    want_v, want_bits = oracle.lif(v0, i_d[0].cpu().numpy(), 6144, beta, theta)
+    assert np.array_equal(bits_d.cpu().numpy().view(np.uint32), want_bits), "lif spot check failed"
+    assert np.array_equal(v_d.cpu().numpy(), want_v), "lif spot check failed"
+
+    n_copies = len(copies)
+
+    def graph_us(decode, steps=64):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            cs = torch.cuda.current_stream()
+            for i in range(steps):
+                produce(i, cs)
+                if decode:
+                    copies[i % n_copies].decode(bits, "bits", words, acc, y, 1536, stream=cs)
+        with torch.cuda.stream(stream):
+            for _ in range(4):
+                g.replay()
+        stream.synchronize()
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        with torch.cuda.stream(stream):
+            e0.record(stream)
+            for _ in range(5):
+                g.replay()
+            e1.record(stream)
+        stream.synchronize()
+        return e0.elapsed_time(e1) * 1e3 / (5 * steps)
+
+    with_p = graph_us(True)
+    bn = bits.cpu().numpy().view(np.uint32)
+    Ks = [w[3] for w in weights]
+    active = sum(int(np.unpackbits(bn[j, : Ks[j] // 32].view(np.uint8)).sum()) for j in range(n))
+    rate = active / float(sum(Ks))
+    producer_only = graph_us(False)
+    # the producer alone on a large state: 512 rows of 65536 neurons
+    R, K = 512, 65536
+    vb = torch.zeros((R, K), dtype=torch.float32, device=dev)
+    ib = torch.full((R, K), 0.05, dtype=torch.float32, device=dev)
+    bb = torch.zeros((R, K // 32), dtype=torch.int32, device=dev)
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        for _ in range(10):
+            sp.spike_proj_lif(vb, ib, K, R, K, beta, theta, bb, K // 32, torch.cuda.current_stream())
+    with torch.cuda.stream(stream):
+        g.replay()
+    stream.synchronize()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        e0.record(stream)
+        for _ in range(3):
+            g.replay()
+        e1.record(stream)
+    stream.synchronize()
+    us = e0.elapsed_time(e1) * 1e3 / 30
+    nbytes = R * K * 12 + R * K // 8          # v read + written, I read, bits written
+    gbs = nbytes / (us * 1e-6) / 1e9
+    hbm = float(peaks["hbm_gbs"])
+    return {"decode_step_with_producer_us": with_p, "producer_only_us_per_step": producer_only,
+            "spike_rate_after_warmup": rate, "active_bytes_last_step": active * 1536,
+            "lif": {"beta": beta, "theta": theta, "current": "N(0.135, 0.3) per neuron per step",
+                    "reading": "v <- fmaf(beta, v, I); spike v >= theta; v -= theta"},
+            "stream": {"rows": R, "K": K, "us": us, "gbs": gbs, "bytes": nbytes,
+                       "roofline": {"bound": "hbm", "achieved": gbs, "peak": hbm, "unit": "GB/s",
+                                    "frac": gbs / hbm, "peak_kind": peak_kind}}}
 
 
 def bench_dense(torch, sp, synth, dev, stream, peaks, peak_kind, world, blocks=22,

@@ -315,6 +315,31 @@ sp_status spike_proj_decode_noalloc(const int8_t *W, int64_t ldw,
  * Errors: SP_EINVAL, SP_EALIGN, SP_ERANGE, SP_EDEVICE, SP_ECUDA (nothing is
  * enqueued on an error).  The kernel cannot fail once launched.
  * ------------------------------------------------------------------------- */
+/* ---------------------------------------------------------------------------
+ * spike_proj_lif -- spike producer: one leaky integrate-and-fire step for
+ * `rows` layers of K neurons, written straight into SP_SPIKES_BITS32 rows
+ * (what spike_proj_decode, _group_decode and _batched read).  The paper names
+ * LIF dynamics (Section 1) without giving the update; this is the reading:
+ *
+ *     v <- fmaf(beta, v, I);   x = (v >= theta);   v <- v - theta where x
+ *
+ * FP32 IEEE operations throughout (no flush of subnormals), so v and the bits
+ * equal the definition's exactly, on every run (a NaN state stays NaN and
+ * never fires; its payload is not preserved).
+ *
+ *   v        device FP32, row r at v + r*ld, updated in place; 4-byte aligned.
+ *   I        device FP32 input current, row r at I + r*ld; 4-byte aligned.
+ *   K        neurons per row, 1 <= K <= SPIKE_PROJ_MAX_K; ld >= K.
+ *   rows     1 <= rows.
+ *   bits     device uint32, row r at bits + r*ld_bits, ld_bits >= ceil(K/32);
+ *            4-byte aligned; bits at or past K are written 0.  Must not
+ *            overlap v or I.
+ * Errors: SP_EINVAL, SP_EALIGN, SP_ERANGE, SP_EDEVICE, SP_ECUDA.
+ * ------------------------------------------------------------------------- */
+sp_status spike_proj_lif(float *v, const float *I, int32_t K, int32_t rows,
+                         int64_t ld, float beta, float theta, uint32_t *bits,
+                         int64_t ld_bits, sp_stream_t stream);
+
 typedef struct sp_dense {
     const int8_t *W;
     int64_t ldw;

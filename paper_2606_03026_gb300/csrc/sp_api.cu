@@ -638,6 +638,20 @@ sp_status spike_proj_decode_noalloc(const int8_t* W, int64_t ldw, const float* s
   return SP_OK;
 }
 
+sp_status spike_proj_lif(float* v, const float* I, int32_t K, int32_t rows, int64_t ld,
+                         float beta, float theta, uint32_t* bits, int64_t ld_bits,
+                         sp_stream_t stream) {
+  if (!v || !I || !bits || rows < 1 || K < 1) return SP_EINVAL;
+  if (K > SPIKE_PROJ_MAX_K) return SP_ERANGE;
+  if (ld < K || ld_bits < words_for(K)) return SP_EINVAL;
+  if (!aligned(v, 4) || !aligned(I, 4) || !aligned(bits, 4)) return SP_EALIGN;
+  int dev = 0;
+  const sp_status st = check_device(&dev);
+  if (st != SP_OK) return st;
+  SP_CUDA(launch_lif(v, I, K, rows, ld, beta, theta, bits, ld_bits, as_stream(stream)));
+  return SP_OK;
+}
+
 sp_status spike_proj_dense(const sp_dense* problems, int32_t count, int32_t B,
                            sp_stream_t stream) {
   if (!problems || count < 1 || count > SPIKE_PROJ_DENSE_MAX_GROUP || B < 1 ||

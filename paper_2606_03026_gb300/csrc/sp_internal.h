@@ -133,6 +133,11 @@ struct DenseProblem {
 constexpr int kDenseMaxProblems = SPIKE_PROJ_DENSE_MAX_GROUP;
 cudaError_t launch_dense(const DenseProblem* probs, int count, int B, cudaStream_t s);
 
+// One LIF step of `rows` layers of K neurons into BITS32 spike rows (see
+// spike_proj_lif).
+cudaError_t launch_lif(float* v, const float* I, int K, int rows, int64_t ld, float beta,
+                       float theta, uint32_t* bits, int64_t ld_bits, cudaStream_t s);
+
 // Launches `kernel` with programmatic stream serialization: its blocks may
 // become resident while the previous kernel of the stream is still running
 // and wait for it in pdl_wait (see sp_ptx.cuh) before touching memory.

@@ -50,6 +50,8 @@ _SIGNATURES = {
     "spike_proj_decode_noalloc": ([_P, _I64, _P, _I32, _I32, _P, ctypes.c_int, _P, _P, _P],
                                   ctypes.c_int),
     "spike_proj_dense": ([_P, _I32, _I32, _P], ctypes.c_int),
+    "spike_proj_lif": ([_P, _P, _I32, _I32, _I64, ctypes.c_float, ctypes.c_float, _P, _I64, _P],
+                       ctypes.c_int),
     "spike_proj_strerror": ([ctypes.c_int], ctypes.c_char_p),
     "spike_proj_last_cuda_error": ([], ctypes.c_int),
     "spike_proj_abi_version": ([], ctypes.c_int),
@@ -191,6 +193,19 @@ def spike_proj_group_decode_host(group, h_spikes, fmt, ld_spikes, h_acc=None, h_
 
 def spike_proj_group_status(group, stream=None) -> int:
     return lib().spike_proj_group_status(group, _stream(stream))
+
+
+def spike_proj_lif(v, I, K, rows, ld, beta, theta, bits, ld_bits, stream=None):
+    _check(lib().spike_proj_lif(_addr(v), _addr(I), K, rows, ld, beta, theta, _addr(bits), ld_bits,
+                                _stream(stream)), "spike_proj_lif")
+
+
+def lif(v, I, beta, theta, bits, K=None, stream=None):
+    """One LIF step of every row of v / I (float32 [rows, ld] tensors),
+    spikes into bits (uint32 [rows, >= ceil(K/32)])."""
+    rows, ld = v.shape
+    spike_proj_lif(v, I, ld if K is None else K, rows, v.stride(0), beta, theta, bits,
+                   bits.stride(0), stream)
 
 
 class SpDense(ctypes.Structure):

@@ -78,6 +78,11 @@ def test_host_only_calls(lib):
     assert lib.spike_proj_dense(ctypes.addressof(d), 1, 1, None) == spikeproj.SP_EALIGN   # ldw % 16
     d.ldw, d.W = 32, fake + 4
     assert lib.spike_proj_dense(ctypes.addressof(d), 1, 1, None) == spikeproj.SP_EALIGN   # W alignment
+    assert lib.spike_proj_lif(None, fake, 64, 1, 64, 0.5, 1.0, fake, 2, None) == spikeproj.SP_EINVAL
+    assert lib.spike_proj_lif(fake, fake, 64, 1, 64, 0.5, 1.0, fake, 1, None) == spikeproj.SP_EINVAL  # ld_bits
+    assert lib.spike_proj_lif(fake + 2, fake, 64, 1, 64, 0.5, 1.0, fake, 2, None) == spikeproj.SP_EALIGN
+    assert lib.spike_proj_lif(fake, fake, 131073, 1, 131073, 0.5, 1.0, fake, 4097, None) == \
+        spikeproj.SP_ERANGE
     assert lib.spike_proj_plan_destroy(None) == spikeproj.SP_OK
     assert lib.spike_proj_group_destroy(None) == spikeproj.SP_OK
 
