@@ -729,6 +729,53 @@ def bench_lif(torch, sp, synth, dev, stream, copies, weights, acc, y, peaks, pea
     active = sum(int(np.unpackbits(bn[j, : Ks[j] // 32].view(np.uint8)).sum()) for j in range(n))
     rate = active / float(sum(Ks))
     producer_only = graph_us(False)
+
+    # the producer fused into the decode launch: state row j = 2b (TCAM, 1536
+    # neurons) or 2b + 1 (down, 6144), two state buffers swapped every step
+    ld = 6144
+    cur = torch.zeros((sets, n, ld), dtype=torch.float32, device=dev)
+    cur[:, 0::2, :1536] = i_t
+    cur[:, 1::2, :] = i_d
+    vs = [torch.zeros((n, ld), dtype=torch.float32, device=dev) for _ in range(2)]
+
+    def fused_us(steps=64):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            cs = torch.cuda.current_stream()
+            for i in range(steps):
+                copies[i % n_copies].decode_lif(vs[i % 2], vs[(i + 1) % 2], cur[i % sets], beta,
+                                                theta, acc=acc, y=y, ld_out=1536, stream=cs)
+        with torch.cuda.stream(stream):
+            for _ in range(4):
+                g.replay()
+        stream.synchronize()
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        with torch.cuda.stream(stream):
+            e0.record(stream)
+            for _ in range(5):
+                g.replay()
+            e1.record(stream)
+        stream.synchronize()
+        return e0.elapsed_time(e1) * 1e3 / (5 * steps)
+
+    fused = fused_us()
+    # one more fused step, spike words written, checked against the oracle
+    fb = torch.zeros((n, words), dtype=torch.int32, device=dev)
+    v0, i0 = vs[0].cpu().numpy(), cur[0].cpu().numpy()
+    with torch.cuda.stream(stream):
+        copies[0].decode_lif(vs[0], vs[1], cur[0], beta, theta, bits=fb, acc=acc, y=y,
+                             ld_out=1536, stream=stream)
+    stream.synchronize()
+    fbn = fb.cpu().numpy().view(np.uint32)
+    v1 = vs[1].cpu().numpy()
+    f_active = 0
+    for j in range(n):
+        wv, wb = oracle.lif(v0[j:j + 1], i0[j:j + 1], Ks[j], beta, theta)
+        assert np.array_equal(fbn[j, : Ks[j] // 32], wb[0]), "fused lif spot check failed"
+        assert np.array_equal(v1[j, : Ks[j]], wv[0, : Ks[j]]), "fused lif spot check failed"
+        f_active += int(np.unpackbits(wb[0].view(np.uint8)).sum())
+    f_rate = f_active / float(sum(Ks))
     # the producer alone on a large state: 512 rows of 65536 neurons
     R, K = 512, 65536
     vb = torch.zeros((R, K), dtype=torch.float32, device=dev)
@@ -755,6 +802,7 @@ def bench_lif(torch, sp, synth, dev, stream, copies, weights, acc, y, peaks, pea
     hbm = float(peaks["hbm_gbs"])
     return {"decode_step_with_producer_us": with_p, "producer_only_us_per_step": producer_only,
             "spike_rate_after_warmup": rate, "active_bytes_last_step": active * 1536,
+            "decode_step_fused_producer_us": fused, "fused_spike_rate_after_warmup": f_rate,
             "lif": {"beta": beta, "theta": theta, "current": "N(0.135, 0.3) per neuron per step",
                     "reading": "v <- fmaf(beta, v, I); spike v >= theta; v -= theta"},
             "stream": {"rows": R, "K": K, "us": us, "gbs": gbs, "bytes": nbytes,

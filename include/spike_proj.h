@@ -240,6 +240,35 @@ sp_status spike_proj_group_decode_host(sp_group_t group, const void *h_spikes,
                                        int32_t *h_acc, float *h_y,
                                        int64_t ld_out, sp_stream_t stream);
 
+/* spike_proj_group_decode_lif: the decode step with its spike producer
+ * fused in.  Projection j's spike row is made by one LIF step (the reading
+ * spike_proj_lif states) of row j of the state and current, inside the same
+ * launch that projects it:
+ *
+ *     u = fmaf(beta, v_in[j][k], I[j][k]);  x_k = (u >= theta);
+ *     v_out[j][k] = x_k ? u - theta : u;    y_j = s ⊙ (Q_j x)     (k < K_j)
+ *
+ * so the step needs one launch instead of producer + decode.  Results equal
+ * spike_proj_lif on a copy of v_in followed by spike_proj_group_decode on its
+ * bits, bit for bit.
+ *
+ *   v_in, I  device FP32, row j at + j*ld (ld >= the largest K); read only.
+ *   v_out    device FP32, same layout; elements k < K_j of row j are written,
+ *            the rest untouched.  Must not overlap v_in or I (swap two state
+ *            buffers from step to step).
+ *   bits     NULL, or device uint32 rows at bits + j*ld_bits (ld_bits >=
+ *            ceil(largest K / 32)) that receive row j's ceil(K_j/32) spike
+ *            words (bits past K_j zero); must not overlap the other buffers.
+ *   acc, y, ld_out  as spike_proj_group_decode.
+ * All of v_in, v_out, I, bits 4-byte aligned (SP_EALIGN).  The fused form
+ * needs every K_j <= 6144 and the group's tiles resident at once; otherwise
+ * the call runs the producer and the decode as two launches, same results. */
+sp_status spike_proj_group_decode_lif(sp_group_t group, const float *v_in,
+                                      float *v_out, const float *I, int64_t ld,
+                                      float beta, float theta, uint32_t *bits,
+                                      int64_t ld_bits, int32_t *acc, float *y,
+                                      int64_t ld_out, sp_stream_t stream);
+
 /* Reads and clears the group's device error word (synchronises `stream`). */
 sp_status spike_proj_group_status(sp_group_t group, sp_stream_t stream);
 

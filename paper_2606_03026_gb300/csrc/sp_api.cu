@@ -586,6 +586,69 @@ sp_status spike_proj_group_decode_host(sp_group_t g, const void* h_spikes, sp_fm
   return SP_OK;
 }
 
+namespace {
+// true when the byte ranges [a, a + na) and [b, b + nb) share a byte
+bool overlaps(const void* a, int64_t na, const void* b, int64_t nb) {
+  const uintptr_t x = (uintptr_t)a, y = (uintptr_t)b;
+  return x < y + (uintptr_t)nb && y < x + (uintptr_t)na;
+}
+}  // namespace
+
+sp_status spike_proj_group_decode_lif(sp_group_t g, const float* v_in, float* v_out,
+                                      const float* I, int64_t ld, float beta, float theta,
+                                      uint32_t* bits, int64_t ld_bits, int32_t* acc, float* y,
+                                      int64_t ld_out, sp_stream_t stream) {
+  if (!g || !v_in || !v_out || !I || (!acc && !y)) return SP_EINVAL;
+  if (ld < g->maxK || ld_out < g->maxN || (bits && ld_bits < words_for(g->maxK))) return SP_EINVAL;
+  if (!aligned(v_in, 4) || !aligned(v_out, 4) || !aligned(I, 4) || (bits && !aligned(bits, 4)) ||
+      (acc && !aligned(acc, 4)) || (y && !aligned(y, 4)))
+    return SP_EALIGN;
+  const int64_t state_bytes = ((int64_t)(g->count - 1) * ld + g->maxK) * 4;
+  const int64_t bits_bytes = bits ? ((int64_t)(g->count - 1) * ld_bits + words_for(g->maxK)) * 4 : 0;
+  if (overlaps(v_out, state_bytes, v_in, state_bytes) || overlaps(v_out, state_bytes, I, state_bytes))
+    return SP_EINVAL;
+  if (bits && (overlaps(bits, bits_bytes, v_in, state_bytes) ||
+               overlaps(bits, bits_bytes, v_out, state_bytes) ||
+               overlaps(bits, bits_bytes, I, state_bytes)))
+    return SP_EINVAL;
+  cudaStream_t s = as_stream(stream);
+  GatherParamsG q = g->params;
+  q.acc = acc;
+  q.y = y;
+  q.ld_out = ld_out;
+  q.fmt = SP_SPIKES_BITS32;
+  q.lif_vin = v_in;
+  q.lif_vout = v_out;
+  q.lif_I = I;
+  q.lif_ld = ld;
+  q.lif_beta = beta;
+  q.lif_theta = theta;
+  q.lif_bits = bits;
+  q.lif_ld_bits = ld_bits;
+  q.spikes = nullptr;
+  q.ld_spikes = 0;
+  const cudaError_t e = launch_gather(q, s);
+  if (e != cudaErrorNotSupported) {
+    SP_CUDA(e);
+    return SP_OK;
+  }
+  // the fused form does not apply: the producer into bits (or the group's
+  // staging rows), then the decode of those rows
+  uint32_t* b = bits ? bits : static_cast<uint32_t*>(g->d_spikes);
+  const int64_t ldb = bits ? ld_bits : (int64_t)(g->spike_row_bytes / 4);
+  int32_t Ks[kMaxProblems];
+  for (int j = 0; j < g->count; ++j) Ks[j] = q.prob[j].K;
+  SP_CUDA(launch_lif_rows(v_in, v_out, I, Ks, g->count, ld, beta, theta, b, ldb, s));
+  q.lif_vin = nullptr;
+  q.lif_vout = nullptr;
+  q.lif_I = nullptr;
+  q.lif_bits = nullptr;
+  q.spikes = b;
+  q.ld_spikes = ldb;
+  SP_CUDA(launch_gather(q, s));
+  return SP_OK;
+}
+
 sp_status spike_proj_group_status(sp_group_t g, sp_stream_t stream) {
   if (!g) return SP_EINVAL;
   cudaStream_t s = as_stream(stream);

@@ -79,6 +79,18 @@ __device__ __forceinline__ void st_peer_v4(uint32_t local, uint32_t rank, int4 v
 template <int NP>
 __device__ __forceinline__ void prefetch_spike_rows(const GatherParamsT<NP>& p) {
   const int rows = p.nprob * p.B;
+  if (p.lif_I) {                            // LIF mode: the state and current rows
+    for (int r = blockIdx.x; r < rows; r += gridDim.x) {
+      const int64_t bytes = (int64_t)p.prob[r].K * 4;
+      const char* vr = reinterpret_cast<const char*>(p.lif_vin + (int64_t)r * p.lif_ld);
+      const char* ir = reinterpret_cast<const char*>(p.lif_I + (int64_t)r * p.lif_ld);
+      for (int64_t off = (int64_t)threadIdx.x * 128; off < bytes; off += (int64_t)blockDim.x * 128) {
+        asm volatile("prefetch.global.L2 [%0];" ::"l"(vr + off));
+        asm volatile("prefetch.global.L2 [%0];" ::"l"(ir + off));
+      }
+    }
+    return;
+  }
   for (int r = blockIdx.x; r < rows; r += gridDim.x) {
     const int j = r / p.B;
     const int K = p.prob[j].K;
@@ -116,14 +128,19 @@ struct UnitSmem {
 // warp w's partial sums in sm.area[w].red and ends with a CTA barrier.
 template <int W, int MAXCK, int L, int S>
 __device__ __forceinline__ void unit_partial(UnitSmem<W, MAXCK, S>& sm, const GatherProblem& P,
-                                             const void* srow, int fmt, int n0, int k0, int ck) {
+                                             const void* srow, int fmt, int n0, int k0, int ck,
+                                             const uint32_t* s_words = nullptr) {
   static_assert(MAXCK % 32 == 0 && MAXCK / 32 <= 32, "one spike word per lane");
   static_assert(MAXCK / W <= 256, "biased 16-bit lanes hold at most 257 columns");
   const int lane = threadIdx.x & 31;
   const int warp = threadIdx.x >> 5;
 
   // ---- 1. this warp's share of the chunk's active columns ---------------------
-  const uint32_t word = lane < ck / 32 ? spike_word(srow, fmt, P.K, k0 + 32 * lane) : 0u;
+  // the chunk's spike words: from the spike row, or already in shared memory
+  // (s_words[i] = columns k0 + 32 i .. k0 + 32 i + 31, bits past K clear)
+  const uint32_t word = lane < ck / 32
+                            ? (s_words ? s_words[lane] : spike_word(srow, fmt, P.K, k0 + 32 * lane))
+                            : 0u;
   const int c = __popc(word);
   int incl = c;
 #pragma unroll
@@ -349,6 +366,7 @@ gather_cluster_kernel(const __grid_constant__ GatherParamsT<NP> p) {
   __shared__ ClusterSmem sm;
   // [sender chunk][owned group]: kch * ceil(128 / kch) < 128 + kch entries
   __shared__ __align__(16) int4 s_recv[kGatherNT / 4 + kGatherCluster];
+  __shared__ uint32_t s_lif[kGatherClusterMaxCK / 32];   // LIF mode: this chunk's spike words
   // every CTA of the cluster arrives here and waits (below) before its first
   // store into a peer's shared memory: the peer is then known to be running
   asm volatile("barrier.cluster.arrive.relaxed;" ::: "memory");
@@ -376,8 +394,35 @@ gather_cluster_kernel(const __grid_constant__ GatherParamsT<NP> p) {
   const int n0 = (cl * P.tpc + ts) * kGatherNT;
   const bool work = n0 < P.N;               // tile slots past the last tile idle
   if (work) {
+    const bool lif = p.lif_I != nullptr;
+    if (lif) {
+      // fused spike producer: one LIF step of this chunk's neurons (every CTA
+      // of the chunk computes the same words from the old state; the CTA of
+      // tile slot 0 in cluster 0 writes the new state and the bits)
+      const int k0 = kc * P.ck;
+      const float* vr = p.lif_vin + (int64_t)j * p.lif_ld;
+      const float* ir = p.lif_I + (int64_t)j * p.lif_ld;
+      const bool writer = cl == 0 && ts == 0;
+      for (int i = threadIdx.x; i < P.ck; i += kGatherClusterThreads) {   // warp-uniform: ck % 32 == 0
+        const int k = k0 + i;
+        bool fire = false;
+        if (k < P.K) {
+          float u = fmaf(p.lif_beta, vr[k], ir[k]);
+          fire = u >= p.lif_theta;
+          if (fire) u = __fsub_rn(u, p.lif_theta);
+          if (writer) p.lif_vout[(int64_t)j * p.lif_ld + k] = u;
+        }
+        const uint32_t w = __ballot_sync(0xffffffffu, fire);
+        if ((threadIdx.x & 31) == 0) {
+          s_lif[i >> 5] = w;
+          if (writer && p.lif_bits && k < P.K) p.lif_bits[(int64_t)j * p.lif_ld_bits + (k >> 5)] = w;
+        }
+      }
+      __syncthreads();
+    }
     unit_partial<kGatherClusterWarps, kGatherClusterMaxCK, kClusterLoads, kClusterSlots>(
-        sm, P, spike_row(p.spikes, p.fmt, j, p.ld_spikes), p.fmt, n0, kc * P.ck, P.ck);
+        sm, P, lif ? nullptr : spike_row(p.spikes, p.fmt, j, p.ld_spikes), p.fmt, n0, kc * P.ck,
+        P.ck, lif ? s_lif : nullptr);
     asm volatile("barrier.cluster.wait;" ::: "memory");
     const int g = threadIdx.x;              // the 4-channel group of this thread
     if (g < kGatherNT / 4) {
@@ -498,7 +543,9 @@ cudaError_t launch_gather_t(const GatherParamsT<NP>& p, cudaStream_t s) {
   if (e != cudaSuccess) return e;
   GatherParamsT<NP> q = p;
   int gx = 0, gy = 0;
-  if (cluster_form(q, &gx, &gy)) {
+  const bool cluster = cluster_form(q, &gx, &gy);
+  if (p.lif_I && !cluster) return cudaErrorNotSupported;   // the fused producer needs the cluster form
+  if (cluster) {
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3((unsigned)gx, (unsigned)gy, 1);
     cfg.blockDim = dim3(kGatherClusterThreads, 1, 1);

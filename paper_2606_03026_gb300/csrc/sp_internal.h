@@ -81,6 +81,17 @@ struct GatherParamsT {
   // problem (cl_list[c] >> 8); ncl_list == 0: grid (clusters x 6, problems)
   int32_t ncl_list;
   uint16_t cl_list[kGatherMaxClusterList];
+  // fused spike producer (cluster form only): when lif_I is set, problem j's
+  // spike row is made inside the kernel by one LIF step of row j of
+  // (lif_vin, lif_I); the new state goes to lif_vout (and the spike words to
+  // lif_bits when set), each element by exactly one CTA
+  const float* lif_vin = nullptr;
+  float* lif_vout = nullptr;
+  const float* lif_I = nullptr;
+  int64_t lif_ld = 0;
+  float lif_beta = 0.f, lif_theta = 0.f;
+  uint32_t* lif_bits = nullptr;
+  int64_t lif_ld_bits = 0;
 };
 using GatherParams1 = GatherParamsT<1>;
 using GatherParamsG = GatherParamsT<kMaxProblems>;
@@ -137,6 +148,11 @@ cudaError_t launch_dense(const DenseProblem* probs, int count, int B, cudaStream
 // spike_proj_lif).
 cudaError_t launch_lif(float* v, const float* I, int K, int rows, int64_t ld, float beta,
                        float theta, uint32_t* bits, int64_t ld_bits, cudaStream_t s);
+// The same for rows <= kMaxProblems rows of Ks[r] neurons each, the state read
+// from vin and written to vout (which may equal vin).
+cudaError_t launch_lif_rows(const float* vin, float* vout, const float* I, const int32_t* Ks,
+                            int rows, int64_t ld, float beta, float theta, uint32_t* bits,
+                            int64_t ld_bits, cudaStream_t s);
 
 // Launches `kernel` with programmatic stream serialization: its blocks may
 // become resident while the previous kernel of the stream is still running

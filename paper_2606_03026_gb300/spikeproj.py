@@ -46,6 +46,8 @@ _SIGNATURES = {
     "spike_proj_group_decode": ([_P, _P, ctypes.c_int, _I64, _P, _P, _I64, _P], ctypes.c_int),
     "spike_proj_group_decode_host": ([_P, _P, ctypes.c_int, _I64, _P, _P, _I64, _P],
                                      ctypes.c_int),
+    "spike_proj_group_decode_lif": ([_P, _P, _P, _P, _I64, ctypes.c_float, ctypes.c_float, _P,
+                                     _I64, _P, _P, _I64, _P], ctypes.c_int),
     "spike_proj_group_status": ([_P, _P], ctypes.c_int),
     "spike_proj_decode_noalloc": ([_P, _I64, _P, _I32, _I32, _P, ctypes.c_int, _P, _P, _P],
                                   ctypes.c_int),
@@ -191,6 +193,14 @@ def spike_proj_group_decode_host(group, h_spikes, fmt, ld_spikes, h_acc=None, h_
            "spike_proj_group_decode_host")
 
 
+def spike_proj_group_decode_lif(group, v_in, v_out, I, ld, beta, theta, bits=None, ld_bits=0,
+                                acc=None, y=None, ld_out=0, stream=None):
+    _check(lib().spike_proj_group_decode_lif(group, _addr(v_in), _addr(v_out), _addr(I), ld, beta,
+                                             theta, _addr(bits), ld_bits, _addr(acc), _addr(y),
+                                             ld_out, _stream(stream)),
+           "spike_proj_group_decode_lif")
+
+
 def spike_proj_group_status(group, stream=None) -> int:
     return lib().spike_proj_group_status(group, _stream(stream))
 
@@ -310,6 +320,14 @@ class Group:
                     stream=None):
         spike_proj_group_decode_host(self.handle, h_spikes, fmt, ld_spikes, h_acc, h_y,
                                      ld_out, stream)
+
+    def decode_lif(self, v_in, v_out, I, beta, theta, bits=None, acc=None, y=None, ld_out=0,
+                   stream=None):
+        """One LIF step of row j of v_in / I (float32 [count, ld] tensors) into
+        v_out, its spikes projected by plan j, in one launch; bits (uint32
+        [count, >= ceil(maxK/32)]) optionally receives the spike words."""
+        spike_proj_group_decode_lif(self.handle, v_in, v_out, I, v_in.stride(0), beta, theta, bits,
+                                    0 if bits is None else bits.stride(0), acc, y, ld_out, stream)
 
     def status(self, stream=None) -> int:
         return spike_proj_group_status(self.handle, stream)

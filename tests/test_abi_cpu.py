@@ -83,6 +83,8 @@ def test_host_only_calls(lib):
     assert lib.spike_proj_lif(fake + 2, fake, 64, 1, 64, 0.5, 1.0, fake, 2, None) == spikeproj.SP_EALIGN
     assert lib.spike_proj_lif(fake, fake, 131073, 1, 131073, 0.5, 1.0, fake, 4097, None) == \
         spikeproj.SP_ERANGE
+    assert lib.spike_proj_group_decode_lif(None, fake, fake, fake, 64, 0.5, 1.0, None, 0, None,
+                                           fake, 64, None) == spikeproj.SP_EINVAL
     assert lib.spike_proj_plan_destroy(None) == spikeproj.SP_OK
     assert lib.spike_proj_group_destroy(None) == spikeproj.SP_OK
 

@@ -1,7 +1,8 @@
 """Spike producer (spike_proj_lif) against the CPU oracle, bit for bit
 (GPU): the membrane state and the BITS32 spike rows over many steps, ragged
-K, padded rows, IEEE special values, and the produced rows fed straight into
-the grouped decode step."""
+K, padded rows, IEEE special values, the produced rows fed straight into
+the grouped decode step, and the producer fused into that step
+(spike_proj_group_decode_lif, both of its forms)."""
 import numpy as np
 import pytest
 import torch
@@ -90,3 +91,122 @@ def test_lif_feeds_group_decode():
         for j, (Q, s, N, K) in enumerate(weights):
             wa, wy = oracle.project(Q, s, N, K, want_bits[j], "bits")
             assert_parity(acc[j], y[j], wa[0], wy[0], f"step {step} projection {j}")
+
+
+# ---------------------------------------------------------------------------
+# the producer fused into the grouped decode (spike_proj_group_decode_lif)
+
+def _fused_steps(weights, steps, with_bits, seed):
+    """Runs `steps` fused decode steps, swapping the two state buffers, and
+    checks every step against the oracle: the new state (bit for bit, rows
+    past K_j untouched, the old state unchanged), the spike words and the
+    projections."""
+    plans = [sp.Plan(to_dev(Q), to_dev(s), N, K) for (Q, s, N, K) in weights]
+    group = sp.Group(plans)
+    n = len(weights)
+    Ks = [w[3] for w in weights]
+    maxK, maxN = max(Ks), max(w[2] for w in weights)
+    ld = maxK + 3
+    words = (maxK + 31) // 32
+    rng = synth.rng_for(830, seed)
+    v = rng.normal(0.0, 0.5, (n, ld)).astype(np.float32)
+    for j, K in enumerate(Ks):
+        v[j, K:] = 7.0
+    bufs = [to_dev(v), torch.full((n, ld), 9.0, dtype=torch.float32, device=DEV)]
+    pads = [v.copy(), np.full((n, ld), 9.0, np.float32)]
+    bits_d = (torch.full((n, words + 1), 0x5A5A5A5A, dtype=torch.int32, device=DEV)
+              if with_bits else None)
+    acc = torch.empty((n, maxN), dtype=torch.int32, device=DEV)
+    y = torch.empty((n, maxN), dtype=torch.float32, device=DEV)
+    for step in range(steps):
+        beta, theta = (0.9, 1.0) if step % 2 == 0 else (0.7, 0.6)
+        I = rng.normal(0.15, 0.6, (n, ld)).astype(np.float32)
+        vin, vout = bufs[step % 2], bufs[(step + 1) % 2]
+        group.decode_lif(vin, vout, to_dev(I), beta, theta, bits=bits_d, acc=acc, y=y,
+                         ld_out=maxN)
+        torch.cuda.synchronize()
+        got_in = vin.cpu().numpy()
+        got_out = vout.cpu().numpy()
+        assert np.array_equal(got_in.view(np.uint32), v.view(np.uint32)), f"v_in written, step {step}"
+        new_v = v.copy()
+        for j, (Q, s, N, K) in enumerate(weights):
+            vj, bj = oracle.lif(v[j:j + 1], I[j:j + 1], K, beta, theta)
+            new_v[j, :K] = vj[0, :K]
+            assert np.array_equal(got_out[j, :K].view(np.uint32), vj[0, :K].view(np.uint32)), \
+                f"step {step} state row {j}"
+            pad = pads[(step + 1) % 2]
+            assert np.array_equal(got_out[j, K:].view(np.uint32), pad[j, K:].view(np.uint32)), \
+                f"step {step} row {j}: wrote past K"
+            if with_bits:
+                wj = (K + 31) // 32
+                gb = bits_d[j].cpu().numpy().view(np.uint32)
+                assert np.array_equal(gb[:wj], bj[0]), f"step {step} bits row {j}"
+                assert np.all(gb[words:] == 0x5A5A5A5A), f"step {step} bits row {j} past ld"
+            wa, wy = oracle.project(Q, s, N, K, bj[0], "bits", ldq=Q.shape[1])
+            assert_parity(acc[j, :N], y[j, :N], wa[0], wy[0], f"step {step} projection {j}")
+        # the buffer just written is the next step's input: its rows past K_j
+        # keep their earlier contents
+        v = new_v.copy()
+        for j, K in enumerate(Ks):
+            v[j, K:] = pads[(step + 1) % 2][j, K:]
+    return group
+
+
+def test_group_decode_lif_decode_step():
+    """The 22-block decode step (44 projections, K = 1536 / 6144) with its
+    spike producer fused in, three steps, spike words written out."""
+    _fused_steps(synth.decode_step_weights(0), steps=3, with_bits=True, seed=1)
+
+
+@pytest.mark.parametrize("with_bits", [True, False])
+def test_group_decode_lif_ragged(with_bits):
+    """Ragged N and K (chunk tails, a K below one word, partial tiles; N a
+    multiple of 16 as plans require)."""
+    shapes = [(16, 33), (496, 1000), (1536, 4097), (4000, 6144), (2096, 1536), (64, 32),
+              (704, 6000), (16, 1)]
+    weights = []
+    for i, (N, K) in enumerate(shapes):
+        Q, s, _ = synth.random_case(840 + i, N, K, ldq=(N + 15) // 16 * 16)
+        weights.append((Q, s, N, K))
+    _fused_steps(weights, steps=4, with_bits=with_bits, seed=2 + with_bits)
+
+
+@pytest.mark.parametrize("with_bits", [True, False])
+def test_group_decode_lif_two_launch_form(with_bits):
+    """A K above the fused form's 6144 columns takes the two-launch route
+    (producer into the spike words or the group's staging, then the decode):
+    the same results."""
+    shapes = [(304, 8192), (1536, 1536), (48, 7000)]
+    weights = []
+    for i, (N, K) in enumerate(shapes):
+        Q, s, _ = synth.random_case(850 + i, N, K, ldq=(N + 15) // 16 * 16)
+        weights.append((Q, s, N, K))
+    _fused_steps(weights, steps=3, with_bits=with_bits, seed=4 + with_bits)
+
+
+def test_group_decode_lif_rejects_overlap_and_alignment():
+    weights = synth.decode_step_weights(0, blocks=1)
+    plans = [sp.Plan(to_dev(Q), to_dev(s), N, K) for (Q, s, N, K) in weights]
+    group = sp.Group(plans)
+    n, ld = len(weights), 6144
+    a = torch.zeros((n, ld), dtype=torch.float32, device=DEV)
+    b = torch.zeros((n, ld), dtype=torch.float32, device=DEV)
+    I = torch.zeros((n, ld), dtype=torch.float32, device=DEV)
+    bits = torch.zeros((n, ld // 32), dtype=torch.int32, device=DEV)
+    y = torch.zeros((n, 1536), dtype=torch.float32, device=DEV)
+    lib = sp.lib()
+    h, s = group.handle, None
+
+    def call(vin, vout, cur, bt, ldb=ld // 32, ld_=ld):
+        return lib.spike_proj_group_decode_lif(h, vin, vout, cur, ld_, 0.9, 1.0, bt, ldb, None,
+                                               y.data_ptr(), 1536, s)
+
+    assert call(a.data_ptr(), a.data_ptr(), I.data_ptr(), None) == sp.SP_EINVAL       # in place
+    assert call(a.data_ptr(), b.data_ptr() - 64, b.data_ptr(), None) == sp.SP_EINVAL  # v_out over I
+    assert call(a.data_ptr(), b.data_ptr(), I.data_ptr(), a.data_ptr() + 4096) == sp.SP_EINVAL
+    assert call(a.data_ptr(), b.data_ptr(), I.data_ptr(), bits.data_ptr(), ldb=191) == sp.SP_EINVAL
+    assert call(a.data_ptr(), b.data_ptr(), I.data_ptr(), None, ld_=6143) == sp.SP_EINVAL
+    assert call(a.data_ptr() + 2, b.data_ptr(), I.data_ptr(), None) == sp.SP_EALIGN
+    assert call(a.data_ptr(), b.data_ptr(), I.data_ptr(), bits.data_ptr()) == sp.SP_OK
+    torch.cuda.synchronize()
+    assert group.status() == sp.SP_OK
