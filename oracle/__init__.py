@@ -18,6 +18,10 @@ Functions mirror ``spike_oracle.h``:
   weights, ``y_m = s_m * sum_k Q[m*ldq + k] * x_k`` evaluated in double, with
   ``sum_k |Q_mk x_k|`` for error bounds (Section 2.3, the sentence on
   continuous inputs; Section 2.2 for the row-major layout).
+* :func:`head` -- the vocabulary head with INT8 activations, the top-two
+  gap gate and FP32-activation recomputation of the top candidates
+  (Section 5, trace configuration; Appendix D; the activation quantiser is a
+  stated reading).
 
 Spike formats: ``"bits"`` = uint32 words, column k is bit k%32 of word k//32
 (LSB first, tail bits ignored); ``"u8"`` = one byte per column, nonzero fires.
@@ -93,6 +97,9 @@ class Oracle:
         lib.sp_oracle_dense.restype = ctypes.c_int
         lib.sp_oracle_lif.argtypes = [p, p, i32, i32, i64, ctypes.c_float, ctypes.c_float, p, i64]
         lib.sp_oracle_lif.restype = ctypes.c_int
+        lib.sp_oracle_head.argtypes = [p, i64, p, i32, i32, p, i64, i32, ctypes.c_float, i32,
+                                       p, p, p, p, p, p, p, p, p]
+        lib.sp_oracle_head.restype = ctypes.c_int
         self.lib = lib
 
     # -- helpers -----------------------------------------------------------
@@ -225,6 +232,43 @@ class Oracle:
         return v, bits[:, :words]
 
 
+    def head(self, Q: np.ndarray, scale: np.ndarray, V: int, K: int, h: np.ndarray,
+             tau: float, k_sel: int, ldq: int | None = None) -> dict:
+        """Vocabulary head for every row of ``h`` (float32 [B, >=K]) through
+        row-major ``Q`` ([V, ldq] int8).  Returns a dict of numpy arrays:
+        codes int8 [B, K], s_x float32 [B], z float32 [B, V], gap float32 [B],
+        verified int32 [B], cand int32 [B, k_sel], r / r_abs float64
+        [B, k_sel], token int32 [B]."""
+        ldq = K if ldq is None else ldq
+        Q = np.ascontiguousarray(Q, dtype=np.int8).reshape(-1)
+        if ldq < K or Q.size < ldq * (V - 1) + K:
+            raise ValueError("Q too small for V, K, ldq")
+        scale = np.ascontiguousarray(scale, dtype=np.float32).reshape(-1)
+        if scale.size < V:
+            raise ValueError("scale shorter than V")
+        h = np.ascontiguousarray(h, dtype=np.float32)
+        if h.ndim == 1:
+            h = h[None, :]
+        if h.shape[1] < K:
+            raise ValueError("h rows shorter than K")
+        B = h.shape[0]
+        out = {"codes": np.zeros((B, K), np.int8), "s_x": np.zeros(B, np.float32),
+               "z": np.zeros((B, V), np.float32), "gap": np.zeros(B, np.float32),
+               "verified": np.zeros(B, np.int32), "cand": np.zeros((B, k_sel), np.int32),
+               "r": np.zeros((B, k_sel), np.float64), "r_abs": np.zeros((B, k_sel), np.float64),
+               "token": np.zeros(B, np.int32)}
+        o = out
+        rc = self.lib.sp_oracle_head(Q.ctypes.data, ldq, scale.ctypes.data, V, K, h.ctypes.data,
+                                     h.shape[1], B, tau, k_sel, o["codes"].ctypes.data,
+                                     o["s_x"].ctypes.data, o["z"].ctypes.data,
+                                     o["gap"].ctypes.data, o["verified"].ctypes.data,
+                                     o["cand"].ctypes.data, o["r"].ctypes.data,
+                                     o["r_abs"].ctypes.data, o["token"].ctypes.data)
+        if rc:
+            raise RuntimeError(f"sp_oracle_head failed: {rc}")
+        return out
+
+
 _DEFAULT: Oracle | None = None
 
 
@@ -255,3 +299,7 @@ def dense(Q, scale, N, K, x, ldq=None):
 
 def lif(v, I, K, beta, theta):
     return default().lif(v, I, K, beta, theta)
+
+
+def head(Q, scale, V, K, h, tau, k_sel, ldq=None):
+    return default().head(Q, scale, V, K, h, tau, k_sel, ldq)

@@ -204,3 +204,118 @@ int sp_oracle_lif(float *v, const float *I, int32_t K, int32_t T, int64_t ld,
     }
     return 0;
 }
+
+/* Vocabulary head with INT8 activations and candidate-row verification, as
+ * stated in spike_oracle.h (Section 5 and Appendix D; the activation quantiser
+ * is a reading).  Steps are numbered as there. */
+typedef struct {
+    float z;
+    int32_t m;
+} head_entry;
+
+/* z descending, then index ascending */
+static int head_order(const void *pa, const void *pb)
+{
+    const head_entry *a = (const head_entry *)pa, *b = (const head_entry *)pb;
+    if (a->z > b->z)
+        return -1;
+    if (a->z < b->z)
+        return 1;
+    return a->m < b->m ? -1 : (a->m > b->m ? 1 : 0);
+}
+
+int sp_oracle_head(const int8_t *Q, int64_t ldq, const float *s, int32_t V,
+                   int32_t K, const float *h, int64_t ldh, int32_t B, float tau,
+                   int32_t k_sel, int8_t *codes, float *s_x, float *z,
+                   float *gap, int32_t *verified, int32_t *cand, double *r,
+                   double *r_abs, int32_t *token)
+{
+    if (!Q || !s || !h || V < 2 || K < 1 || B < 0 || k_sel < 1 || k_sel > V || ldq < K ||
+        (B > 1 && ldh < K))
+        return -1;
+    int8_t *q = (int8_t *)malloc((size_t)K);
+    head_entry *order = (head_entry *)malloc((size_t)V * sizeof(head_entry));
+    double *rc = (double *)malloc((size_t)k_sel * sizeof(double));
+    if (!q || !order || !rc) {
+        free(q);
+        free(order);
+        free(rc);
+        return -3;
+    }
+    for (int32_t b = 0; b < B; ++b) {
+        const float *hb = h + (int64_t)b * ldh;
+        /* 1. activation scale and codes */
+        float amax = 0.0f;
+        for (int32_t k = 0; k < K; ++k)
+            if (fabsf(hb[k]) > amax)
+                amax = fabsf(hb[k]);
+        const float sx = fmaxf(amax, 1e-8f) / 127.0f;
+        for (int32_t k = 0; k < K; ++k) {
+            float c = rintf(hb[k] / sx);
+            if (c > 127.0f)
+                c = 127.0f;
+            if (c < -127.0f)
+                c = -127.0f;
+            q[k] = (int8_t)c;
+        }
+        /* 2. approximate logits */
+        for (int32_t m = 0; m < V; ++m) {
+            const int8_t *row = Q + (int64_t)m * ldq;
+            int64_t a = 0;
+            for (int32_t k = 0; k < K; ++k)
+                a += (int64_t)row[k] * (int64_t)q[k];
+            if (a > INT32_MAX || a < INT32_MIN) {
+                free(q);
+                free(order);
+                free(rc);
+                return -2;
+            }
+            const float t = sx * (float)(int32_t)a;
+            order[m].z = s[m] * t;
+            order[m].m = m;
+            if (z)
+                z[(int64_t)b * V + m] = order[m].z;
+        }
+        /* 3. order and top-two gap; 4. the gate */
+        qsort(order, (size_t)V, sizeof(head_entry), head_order);
+        const float g = order[0].z - order[1].z;
+        const int open = g < tau;
+        /* 5. candidates, recomputed with the FP32 activations */
+        int32_t best = 0;
+        for (int32_t i = 0; i < k_sel; ++i) {
+            const int32_t m = order[i].m;
+            const int8_t *row = Q + (int64_t)m * ldq;
+            double sum = 0.0, abs_sum = 0.0;
+            for (int32_t k = 0; k < K; ++k) {
+                const double term = (double)row[k] * (double)hb[k];
+                sum += term;
+                abs_sum += fabs(term);
+            }
+            rc[i] = (double)s[m] * sum;
+            if (rc[i] > rc[best] || (rc[i] == rc[best] && m < order[best].m))
+                best = i;
+            if (cand)
+                cand[(int64_t)b * k_sel + i] = m;
+            if (r)
+                r[(int64_t)b * k_sel + i] = rc[i];
+            if (r_abs)
+                r_abs[(int64_t)b * k_sel + i] = abs_sum;
+        }
+        /* 6. the token */
+        if (codes)
+            for (int32_t k = 0; k < K; ++k)
+                codes[(int64_t)b * K + k] = q[k];
+        if (s_x)
+            s_x[b] = sx;
+        if (gap)
+            gap[b] = g;
+        if (verified)
+            verified[b] = open;
+        if (token)
+            token[b] = open ? order[best].m : order[0].m;
+    }
+    free(q);
+    free(order);
+    free(rc);
+    return 0;
+}

@@ -23,8 +23,9 @@
  * (k / 32), bits at or beyond K are ignored.
  *
  * sp_oracle_dense is the paper's other kernel: the continuous-input
- * projection over row-major INT8 weights.  sp_oracle_lif (declared last)
- * produces spike rows in the BITS32 format from a LIF state.
+ * projection over row-major INT8 weights.  sp_oracle_lif produces spike rows
+ * in the BITS32 format from a LIF state.  sp_oracle_head (declared last) is
+ * the vocabulary head with INT8 activations and candidate-row verification.
  *
  * All functions are single-threaded, allocate only O(K) scratch, and return
  * 0 on success, a negative code on a bad argument (-1) or an INT32 overflow of
@@ -97,6 +98,43 @@ int sp_oracle_dense(const int8_t *Q, int64_t ldq, const float *s,
  * or past K written as 0).  v is updated in place. */
 int sp_oracle_lif(float *v, const float *I, int32_t K, int32_t T, int64_t ld,
                   float beta, float theta, uint32_t *bits, int64_t ld_bits);
+
+/* Vocabulary head with INT8 activations and candidate-row verification
+ * (Section 5, trace configuration; Appendix D).  The head is a continuous-
+ * input projection with row-major INT8 weights Q (element (m, k) at
+ * Q[m * ldq + k], V rows of K) and row scales s.  For each hidden state h
+ * (row b at h + b * ldh), in the paper's order:
+ *
+ *   1. INT8 activations.  The paper does not state the activation quantiser;
+ *      this reads it as the weight rule of Section 2.3 applied to the vector,
+ *      in FP32: s_x = max(max_k |h_k|, 1e-8) / 127,
+ *      q_k = clip(round_half_even(h_k / s_x), -127, 127).
+ *   2. Approximate logits over the full vocabulary: the integer dot product
+ *      a_m = sum_k Q_{m,k} q_k (exact, INT32), then
+ *      z_m = s_m * (s_x * float(a_m)), two FP32 multiplies.
+ *   3. Order the rows by z descending, equal z by ascending index; the top-two
+ *      gap is gap = z_(1) - z_(2) (one FP32 subtraction).
+ *   4. The gate: verification runs when gap < tau (0.5 in the trace
+ *      configuration, 4.0 in the power configuration).
+ *   5. Candidates: the first k_sel rows of that order (K = 16, 32, 64 in the
+ *      paper).  Each is recomputed with FP32 activations, the continuous-input
+ *      rule of Section 2.3: r_m = s_m * sum_k float(Q_{m,k}) h_k.  Here in
+ *      double, as sp_oracle_dense: every product exact, the sum within
+ *      K * 2^-53 of sum_k |Q_{m,k} h_k| (returned in r_abs for error bounds).
+ *   6. The token: with verification, the candidate with the largest r (equal r
+ *      by ascending index); without, the first row of the order.
+ *
+ * Outputs per row b (any pointer may be NULL): codes[b*K + k] = q_k, s_x[b],
+ * z[b*V + m], gap[b], verified[b] (0 / 1), cand[b*k_sel + i] (the order's
+ * first k_sel rows), r[b*k_sel + i], r_abs[b*k_sel + i] (for every candidate,
+ * whether or not the gate opened), token[b].
+ * Requires V >= 2, 1 <= k_sel <= V, ldq >= K, ldh >= K when B > 1; -1 on a bad
+ * argument, -3 when scratch allocation fails. */
+int sp_oracle_head(const int8_t *Q, int64_t ldq, const float *s, int32_t V,
+                   int32_t K, const float *h, int64_t ldh, int32_t B, float tau,
+                   int32_t k_sel, int8_t *codes, float *s_x, float *z,
+                   float *gap, int32_t *verified, int32_t *cand, double *r,
+                   double *r_abs, int32_t *token);
 
 #ifdef __cplusplus
 }

@@ -33,6 +33,16 @@ an exactly periodic closed form, cases where a fused multiply-add and a
 separate multiply then add round differently (exact rational arithmetic
 rounded to FP32), the bit format and cleared tail bits via the spike
 oracle's own unpacking, row strides, and an infinite threshold.
+
+The vocabulary head (INT8 activations, top-two gap gate, FP32-activation
+recompute of the top candidates) is pinned by a hand-worked fixture
+(tests/golden/hand_worked_head.json) in which verification changes the
+token and an exact tie picks the lower index; activations that are exact
+INT8 codes times a power of two (the recompute must then equal the
+approximate logit and the numpy integer product); round-half-even codes and
+the 1e-8 floor; numpy's lexsort of the logits with duplicate rows and the
+strict gate at tau = gap; row and column permutations; the dense oracle's
+projection and argmax when every row is a candidate; and the zero state.
 """
 from __future__ import annotations
 
@@ -382,9 +392,136 @@ def pin_lif_bits_format(orc):
     assert not bits.any()
 
 
+def _head_case(seed, V, K, B=1, ldq_pad=0, ldh_pad=0):
+    rng = synth.rng_for(7700, seed, V, K, B)
+    Q = rng.integers(-127, 128, size=(V, K + ldq_pad)).astype(np.int8)
+    s = rng.uniform(0.01, 0.05, size=V).astype(np.float32)
+    h = rng.standard_normal((B, K + ldh_pad)).astype(np.float32)
+    return Q, s, h
+
+
+def pin_head_hand_fixture(orc):
+    g = json.loads((GOLDEN / "hand_worked_head.json").read_text())
+    Q = np.array(g["Q_rows"], np.int8)
+    s = np.array(g["s"], np.float32)
+    h = np.array(g["h"], np.float32)
+    for case in g["cases"]:
+        o = orc.head(Q, s, g["V"], g["K"], h, case["tau"], case["k_sel"])
+        assert o["codes"][0].tolist() == g["codes"]
+        assert np.allclose(o["z"][0] / o["s_x"][0], g["z_over_s_x"], rtol=1e-6)
+        assert np.isclose(o["s_x"][0], 2.0 / 127.0, rtol=1e-6)
+        assert np.isclose(o["gap"][0], g["gap"], rtol=1e-5)
+        assert int(o["verified"][0]) == case["verified"]
+        assert o["cand"][0].tolist() == case["cand"]
+        if "r" in case:
+            assert np.allclose(o["r"][0], case["r"], rtol=1e-7)
+        assert int(o["token"][0]) == case["token"]
+
+
+def pin_head_integer_activations(orc):
+    # h = q * 2^-4 with max |q| = 127: the scale is exactly 2^-4, the codes are
+    # q, and the FP32-activation recompute (a separate loop over h) must equal
+    # the approximate logit of the same row (both exact before one rounding)
+    V, K, B = 40, 50, 2
+    Q, s, _ = _head_case(1, V, K, B, ldq_pad=3)
+    rng = synth.rng_for(7701)
+    q = rng.integers(-127, 128, size=(B, K + 2)).astype(np.int64)
+    q[:, 7] = 127
+    q[1, 7] = -127
+    h = (q * 2.0 ** -4).astype(np.float32)
+    o = orc.head(Q, s, V, K, h, np.inf, V, ldq=K + 3)
+    assert np.array_equal(o["codes"], q[:, :K].astype(np.int8))
+    assert np.all(o["s_x"] == np.float32(2.0 ** -4))
+    for b in range(B):
+        assert np.array_equal(o["r"][b].astype(np.float32), o["z"][b][o["cand"][b]])
+        # and both equal the integer product Q q (numpy int64) scaled
+        a = Q[:, :K].astype(np.int64) @ q[b, :K]
+        assert np.array_equal(o["r"][b], s[o["cand"][b]].astype(np.float64) * (a[o["cand"][b]] * 2.0 ** -4))
+
+
+def pin_head_quantiser_rounding(orc):
+    # with amax = 127 * 2^-3 the scale is exactly 2^-3: halves round to even
+    K = 8
+    h = (np.array([127, 2.5, -2.5, 3.5, 0.5, -0.5, 1.5, 126.5]) * 2.0 ** -3).astype(np.float32)
+    Q = np.ones((2, K), np.int8)
+    o = orc.head(Q, np.ones(2, np.float32), 2, K, h, 0.0, 1)
+    assert o["codes"][0].tolist() == [127, 2, -2, 4, 0, 0, 2, 126]
+    assert o["s_x"][0] == np.float32(0.125)
+    # below the 1e-8 floor the scale stays 1e-8 / 127 (about 7.874e-11)
+    h = np.array([1e-10, -3e-9, 0.0], np.float32)
+    o = orc.head(np.ones((2, 3), np.int8), np.ones(2, np.float32), 2, 3, h, 0.0, 1)
+    assert o["codes"][0].tolist() == [1, -38, 0]
+    assert np.isclose(o["s_x"][0], 1e-8 / 127, rtol=1e-6)
+
+
+def pin_head_order_and_gate(orc):
+    # duplicate rows give equal z: they must come in ascending index; the
+    # order must be numpy's lexsort of (index, -z); the gate is strict
+    V, K = 64, 33
+    Q, s, h = _head_case(2, V, K)
+    for dst, src in ((40, 3), (9, 3), (50, 61), (12, 61)):
+        Q[dst], s[dst] = Q[src], s[src]
+    o = orc.head(Q, s, V, K, h, 0.5, V)
+    z = o["z"][0]
+    assert z[9] == z[3] == z[40] and z[12] == z[50] == z[61]
+    want = np.lexsort((np.arange(V), -z.astype(np.float64)))
+    assert o["cand"][0].tolist() == want.tolist()
+    g = np.float32(z[want[0]]) - np.float32(z[want[1]])
+    assert o["gap"][0] == g
+    for tau, want_v in ((0.0, 0), (float(g), 0), (float(np.nextafter(g, np.float32(np.inf))), 1),
+                        (np.inf, 1)):
+        assert int(orc.head(Q, s, V, K, h, tau, 4)["verified"][0]) == want_v, tau
+
+
+def pin_head_permutation(orc):
+    # renaming the rows renames the candidates and the token; permuting the
+    # columns of Q and h together changes no decision
+    V, K = 50, 40
+    Q, s, h = _head_case(3, V, K)
+    o = orc.head(Q, s, V, K, h, np.inf, 8)
+    perm = synth.rng_for(7703).permutation(V)
+    inv = np.argsort(perm)
+    op = orc.head(Q[perm], s[perm], V, K, h, np.inf, 8)
+    assert op["cand"][0].tolist() == inv[o["cand"][0]].tolist()
+    assert int(op["token"][0]) == int(inv[o["token"][0]])
+    cp = synth.rng_for(7704).permutation(K)
+    oc = orc.head(Q[:, cp], s, V, K, h[:, cp], np.inf, 8)
+    assert np.array_equal(oc["z"], o["z"]) and oc["cand"].tolist() == o["cand"].tolist()
+    assert int(oc["token"][0]) == int(o["token"][0])
+    assert np.allclose(oc["r"], o["r"], rtol=1e-12)
+
+
+def pin_head_full_verification_is_dense_argmax(orc):
+    # every row a candidate and the gate always open: the verified logits are
+    # the continuous-input projection of h (the dense oracle), the token its
+    # argmax; strides padded on both operands
+    V, K, B = 45, 70, 2
+    Q, s, h = _head_case(4, V, K, B, ldq_pad=5, ldh_pad=3)
+    o = orc.head(Q, s, V, K, h, np.inf, V, ldq=K + 5)
+    y, _ = orc.dense(Q, s, V, K, h, ldq=K + 5)
+    for b in range(B):
+        assert np.array_equal(o["r"][b], y[b][o["cand"][b]])
+        assert int(o["token"][b]) == int(np.argmax(y[b]))
+
+
+def pin_head_zero_state(orc):
+    V, K = 10, 6
+    Q, s, _ = _head_case(5, V, K)
+    h = np.zeros(K, np.float32)
+    o = orc.head(Q, s, V, K, h, 0.5, 4)
+    assert np.all(o["codes"] == 0) and np.all(o["z"] == 0) and o["gap"][0] == 0
+    assert int(o["verified"][0]) == 1 and o["cand"][0].tolist() == [0, 1, 2, 3]
+    assert np.all(o["r"] == 0) and int(o["token"][0]) == 0
+    o = orc.head(Q, s, V, K, h, 0.0, 4)
+    assert int(o["verified"][0]) == 0 and int(o["token"][0]) == 0
+
+
 ALL_PINS = [pin_hand_fixture, pin_exhaustive_small, pin_full_shapes,
             pin_scale_rounding, pin_invariants, pin_closed_forms,
             pin_overflow_reported, pin_entries,
             pin_dense_hand_fixture, pin_dense_matmul, pin_dense_closed_forms,
             pin_dense_linearity, pin_dense_binary_is_sparse,
-            pin_lif_hand_fixture, pin_lif_periodic, pin_lif_fma_rounding, pin_lif_bits_format]
+            pin_lif_hand_fixture, pin_lif_periodic, pin_lif_fma_rounding, pin_lif_bits_format,
+            pin_head_hand_fixture, pin_head_integer_activations, pin_head_quantiser_rounding,
+            pin_head_order_and_gate, pin_head_permutation,
+            pin_head_full_verification_is_dense_argmax, pin_head_zero_state]

@@ -2,7 +2,8 @@
 pins catch it: a dropped term, a wrong sign, a transposed operand, a wrong
 bit index, a lost scale, a wrong spike test, a lost overflow check; for the
 continuous-input projection a dropped row or activation stride, a dropped
-term, a wrong sign, a lost scale, a signed magnitude, a float accumulator.  The
+term, a wrong sign, a lost scale, a signed magnitude, a float accumulator;
+for the LIF step and the vocabulary head the mistakes listed by name.  The
 mutants are compiled on the CPU from the oracle's own source text."""
 from pathlib import Path
 
@@ -42,6 +43,25 @@ MUTANTS = {
     "lif_msb_first": ("bt[k / 32] |= 1u << (k % 32);", "bt[k / 32] |= 1u << (31 - k % 32);"),
     "lif_tail_kept": ("for (int64_t w = 0; w < words; ++w)\n            bt[w] = 0u;", ""),
     "lif_row_stride_ignored": ("float *vt = v + (int64_t)t * ld;", "float *vt = v + (int64_t)t * K;"),
+    # vocabulary head (every mutant stays inside its buffers; the comparator
+    # mutants stay consistent orders)
+    "head_scale_without_127": ("fmaxf(amax, 1e-8f) / 127.0f", "fmaxf(amax, 1e-8f) / 128.0f"),
+    "head_no_floor": ("const float sx = fmaxf(amax, 1e-8f)", "const float sx = fmaxf(amax, 1e-12f)"),
+    "head_truncating_round": ("float c = rintf(hb[k] / sx);", "float c = truncf(hb[k] / sx);"),
+    "head_round_half_away": ("float c = rintf(hb[k] / sx);", "float c = roundf(hb[k] / sx);"),
+    "head_clip_126": ("if (c > 127.0f)\n                c = 127.0f;", "if (c > 126.0f)\n                c = 126.0f;"),
+    "head_last_column_dropped": ("for (int32_t k = 0; k < K; ++k)\n                a += ", "for (int32_t k = 0; k + 1 < K; ++k)\n                a += "),
+    "head_row_stride_ignored": ("const int8_t *row = Q + (int64_t)m * ldq;\n            int64_t a = 0;", "const int8_t *row = Q + (int64_t)m * K;\n            int64_t a = 0;"),
+    "head_h_stride_ignored": ("const float *hb = h + (int64_t)b * ldh;", "const float *hb = h + (int64_t)b * K;"),
+    "head_scale_of_wrong_row": ("order[m].z = s[m] * t;", "order[m].z = s[0] * t;"),
+    "head_ascending_order": ("if (a->z > b->z)\n        return -1;\n    if (a->z < b->z)\n        return 1;", "if (a->z < b->z)\n        return -1;\n    if (a->z > b->z)\n        return 1;"),
+    "head_ties_by_higher_index": ("return a->m < b->m ? -1 : (a->m > b->m ? 1 : 0);", "return a->m > b->m ? -1 : (a->m < b->m ? 1 : 0);"),
+    "head_gap_to_third": ("const float g = order[0].z - order[1].z;", "const float g = order[0].z - order[2].z;"),
+    "head_gate_inclusive": ("const int open = g < tau;", "const int open = g <= tau;"),
+    "head_verify_from_codes": ("const double term = (double)row[k] * (double)hb[k];", "const double term = (double)row[k] * (double)q[k] * (double)sx;"),
+    "head_verify_scale_dropped": ("rc[i] = (double)s[m] * sum;", "rc[i] = sum;"),
+    "head_token_never_verified": ("token[b] = open ? order[best].m : order[0].m;", "token[b] = order[0].m;"),
+    "head_token_tie_higher": ("(rc[i] == rc[best] && m < order[best].m)", "(rc[i] == rc[best] && m > order[best].m)"),
 }
 
 
