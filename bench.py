@@ -73,6 +73,10 @@ def parse():
                     help="skip the continuous-input projections section")
     ap.add_argument("--no-lif", action="store_true",
                     help="skip the spike-producer section")
+    ap.add_argument("--no-head", action="store_true",
+                    help="skip the vocabulary-head section")
+    ap.add_argument("--head-only", action="store_true",
+                    help="run only the vocabulary-head section")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
     ap.add_argument("--e2e-steps", type=int, default=6400)
@@ -293,6 +297,12 @@ def run_ours(args):
         if rank == 0:
             print(json.dumps({"prefill": res}))
         return
+    if args.head_only:
+        res = bench_head(torch, sp, synth, dev, torch.cuda.Stream(device=dev), peaks, peak_kind,
+                         with_oracle=rank == 0 and not args.no_cpu_baseline)
+        if rank == 0:
+            print(json.dumps({"head": res}))
+        return
     if args.dense_only:
         res = bench_dense(torch, sp, synth, dev, torch.cuda.Stream(device=dev), peaks, peak_kind,
                           world, with_oracle=rank == 0 and not args.no_cpu_baseline)
@@ -466,6 +476,10 @@ def run_ours(args):
     if not args.no_dense:
         result["dense"] = bench_dense(torch, sp, synth, dev, stream, peaks, peak_kind, world,
                                       with_oracle=rank == 0 and not args.no_cpu_baseline)
+
+    if not args.no_head:
+        result["head"] = bench_head(torch, sp, synth, dev, stream, peaks, peak_kind,
+                                    with_oracle=rank == 0 and not args.no_cpu_baseline)
 
     if not args.no_configs:
         result["configs"] = bench_configs(torch, sp, synth, dev, stream, float(peaks["hbm_gbs"]),
@@ -808,6 +822,96 @@ def bench_lif(torch, sp, synth, dev, stream, copies, weights, acc, y, peaks, pea
             "stream": {"rows": R, "K": K, "us": us, "gbs": gbs, "bytes": nbytes,
                        "roofline": {"bound": "hbm", "achieved": gbs, "peak": hbm, "unit": "GB/s",
                                     "frac": gbs / hbm, "peak_kind": peak_kind}}}
+
+
+def bench_head(torch, sp, synth, dev, stream, peaks, peak_kind, with_oracle=True, copies=3):
+    """Vocabulary head (Section 5, trace configuration): 57,344 x 1536 INT8
+    weights, INT8 activations, the top-two gap gate and FP32 recomputation of
+    the k_sel best rows, one spike_proj_head launch per call, graph-replayed
+    over 64 rotating hidden states.  Three weight copies (264 MB, above L2)
+    rotate so that every call streams its weights from HBM.  Timed with the
+    gate closed (tau = 0), at the trace gate (0.5), the power gate (4.0) and
+    always open (inf), for k_sel = 16, 32, 64 and 1 or 4 hidden states."""
+    import oracle
+    Q, s = synth.head_weights()
+    V, K = Q.shape
+    Qd0, sd0 = torch.from_numpy(Q).to(dev), torch.from_numpy(s).to(dev)
+    heads = []
+    for c in range(copies):
+        Qc = Qd0.clone() if c else Qd0
+        heads.append(sp.Head(Qc, sd0, K=K))
+    steps = GRAPH_STEPS
+    hs = {B: torch.from_numpy(np.stack([synth.head_hidden(i, B=B) for i in range(steps)])).to(dev)
+          for B in (1, 4)}
+    tok = torch.zeros((steps, 4), dtype=torch.int32, device=dev)
+    ver = torch.zeros((steps, 4), dtype=torch.int32, device=dev)
+    gap = torch.zeros((steps, 4), dtype=torch.float32, device=dev)
+    cand = torch.zeros((steps, 4, 64), dtype=torch.int32, device=dev)
+    rr = torch.zeros((steps, 4, 64), dtype=torch.float32, device=dev)
+
+    def timed(B, tau, k_sel, reps=5):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            cs = torch.cuda.current_stream()
+            for i in range(steps):
+                heads[i % copies](hs[B][i], tau, k_sel, tok[i], ver[i], gap[i], cand[i], rr[i],
+                                  stream=cs)
+        with torch.cuda.stream(stream):
+            for _ in range(3):
+                g.replay()
+        stream.synchronize()
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        with torch.cuda.stream(stream):
+            e0.record(stream)
+            for _ in range(reps):
+                g.replay()
+            e1.record(stream)
+        stream.synchronize()
+        return e0.elapsed_time(e1) * 1e3 / (reps * steps)
+
+    res = {"V": V, "K": K, "weight_bytes": V * K, "copies": copies, "calls_per_graph": steps}
+    table = {}
+    for B in (1, 4):
+        for tau in (0.0, 0.5, 4.0, float("inf")):
+            for k_sel in (16, 32, 64):
+                if B == 4 and k_sel != 64:
+                    continue
+                us = timed(B, tau, k_sel)
+                vr = ver[:, :B].cpu().numpy()
+                table[f"B{B}_tau{tau}_k{k_sel}"] = {"us": us, "verified_share": float(vr.mean())}
+    res["calls"] = table
+    base = table["B1_tau0.5_k64"]
+    us = base["us"]
+    gbs = V * K / (us * 1e-6) / 1e9
+    hbm = float(peaks["hbm_gbs"])
+    res["headline"] = {"config": "B=1, tau=0.5, k_sel=64", "us_per_token": us, "gbs": gbs,
+                       "tokens_per_s": 1e6 / us}
+    res["roofline"] = {"bound": "hbm", "achieved": gbs, "peak": hbm, "unit": "GB/s",
+                       "frac": gbs / hbm, "peak_kind": peak_kind,
+                       "bytes_per_call": V * K, "note": "algorithmic bytes = V*K weight bytes"}
+    res["verification_cost_us"] = table["B1_tauinf_k64"]["us"] - table["B1_tau0.0_k64"]["us"]
+    # spot check of the last graph's calls (B = 4, tau = inf, k_sel = 64) against the oracle
+    bad = 0
+    for i in (0, steps - 1):
+        h = hs[4][i].cpu().numpy()
+        want = oracle.head(Q, s, V, K, h, float("inf"), 64)
+        bad += int(not np.array_equal(cand[i].cpu().numpy(), want["cand"]))
+        bad += int(not np.array_equal(gap[i].cpu().numpy(), want["gap"]))
+    assert bad == 0, "head spot check failed"
+    if with_oracle:
+        t0 = time.perf_counter()
+        n = 0
+        while time.perf_counter() - t0 < 3.0:
+            oracle.head(Q, s, V, K, synth.head_hidden(n), 0.5, 64)
+            n += 1
+        dt = time.perf_counter() - t0
+        res["cpu_baseline"] = {"value": n / dt, "unit": "tokens/s", "cores": 1, "kind": "oracle",
+                               "sample": f"{n} single-state head calls (V={V}, K={K}, tau 0.5, "
+                                         f"k_sel 64) in {dt:.1f} s"}
+    for hd in heads:
+        hd.close()
+    return res
 
 
 def bench_dense(torch, sp, synth, dev, stream, peaks, peak_kind, world, blocks=22,

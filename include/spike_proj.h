@@ -50,9 +50,14 @@ extern "C" {
 #define SPIKE_PROJ_NOALLOC_MAX_N 32768 /* largest N of spike_proj_decode_noalloc */
 #define SPIKE_PROJ_DENSE_MAX_B 4       /* activation rows per spike_proj_dense call */
 #define SPIKE_PROJ_DENSE_MAX_GROUP 128 /* problems per spike_proj_dense call */
+#define SPIKE_PROJ_HEAD_MAX_B 4        /* hidden states per spike_proj_head call */
+#define SPIKE_PROJ_HEAD_MAX_CAND 64    /* largest k_sel of spike_proj_head */
+#define SPIKE_PROJ_HEAD_MAX_K 8192     /* largest hidden width of a head */
+#define SPIKE_PROJ_HEAD_MAX_V (1 << 26) /* largest vocabulary of a head */
 
 typedef struct sp_plan_s *sp_plan_t;
 typedef struct sp_group_s *sp_group_t;
+typedef struct sp_head_s *sp_head_t;
 typedef void *sp_stream_t;             /* a cudaStream_t */
 
 typedef enum sp_status {
@@ -383,6 +388,62 @@ typedef struct sp_dense {
 
 sp_status spike_proj_dense(const sp_dense *problems, int32_t count, int32_t B,
                            sp_stream_t stream);
+
+/* ---------------------------------------------------------------------------
+ * Vocabulary head with INT8 activations and candidate-row verification
+ * (Section 5, trace configuration; Appendix D).  The head's weights are a
+ * continuous-input projection: W ROW-MAJOR INT8, row m (one vocabulary slot)
+ * at W + m*ldw, K bytes used, with one FP32 scale per row.  For each hidden
+ * state h, in ONE kernel launch:
+ *
+ *   1. INT8 activations (the paper does not state the activation quantiser;
+ *      this reads it as the weight rule of Section 2.3 applied to h):
+ *        s_x = max(max_k |h_k|, 1e-8) / 127,  q_k = clip(rint(h_k / s_x), +-127)
+ *   2. approximate logits z_m = s_m * (s_x * float(sum_k W[m][k] q_k))
+ *      (exact integer sum, two FP32 multiplies)
+ *   3. rows ordered by z descending, equal z by lower row;
+ *      gap = z_(1) - z_(2) (FP32)
+ *   4. the gate: verification when gap < tau (0.5 in the paper's trace
+ *      configuration, 4.0 in its power configuration)
+ *   5. the first k_sel rows of the order (the candidates) recomputed with the
+ *      FP32 activations: r_m = s_m * sum_k float(W[m][k]) h_k
+ *   6. token = the candidate with the largest r (equal r: lower row) when
+ *      verified, else the first row of the order.
+ *
+ * z, the gap, the gate decision and the candidates equal the definition's
+ * bit for bit; r is an FP32 sum of K products of depth <= 16*ceil(K/512) + 5
+ * (the bound of spike_proj_dense).  The weights are read once per call (the
+ * call is HBM-bound on V*K bytes).
+ *
+ * spike_proj_head_create: W device, 16-byte aligned, ldw >= K with
+ *   ldw % 16 == 0 (SP_EALIGN); scale device FP32 [V], 4-byte aligned;
+ *   2 <= V <= SPIKE_PROJ_HEAD_MAX_V, 1 <= K <= SPIKE_PROJ_HEAD_MAX_K
+ *   (SP_ERANGE).  W and scale are borrowed and must outlive the head, which
+ *   owns a 3 MiB workspace.  A head serves one stream at a time.
+ * ------------------------------------------------------------------------- */
+sp_status spike_proj_head_create(sp_head_t *head, const int8_t *W, int64_t ldw,
+                                 const float *scale, int32_t V, int32_t K,
+                                 sp_stream_t stream);
+sp_status spike_proj_head_destroy(sp_head_t head);
+
+/* spike_proj_head: B hidden states (1 .. SPIKE_PROJ_HEAD_MAX_B), row b at
+ * h + b*ldh (device FP32, h 16-byte aligned, ldh >= K with ldh % 4 == 0,
+ * else SP_EALIGN / SP_EINVAL); 1 <= k_sel <= min(V, SPIKE_PROJ_HEAD_MAX_CAND).
+ * Outputs, device, 4-byte aligned, row b of each:
+ *   token     int32 [B] (required)
+ *   verified  int32 [B]: 1 when the gate opened (may be NULL)
+ *   gap       FP32 [B] (may be NULL)
+ *   cand      int32 [B][k_sel]: the candidate rows in order (may be NULL)
+ *   r         FP32 [B][k_sel]: their recomputed logits, written only for
+ *             the rows whose gate opened (may be NULL)
+ *   z         FP32 rows at z + b*ld_z, ld_z >= V: the approximate logits
+ *             (may be NULL)
+ * A tau of +inf always verifies, 0 or NaN never does.  Non-finite h gives
+ * unspecified (but in-range) results. */
+sp_status spike_proj_head(sp_head_t head, const float *h, int64_t ldh, int32_t B,
+                          float tau, int32_t k_sel, int32_t *token,
+                          int32_t *verified, float *gap, int32_t *cand, float *r,
+                          float *z, int64_t ld_z, sp_stream_t stream);
 
 /* --------------------------------------------------------------------------- */
 const char *spike_proj_strerror(sp_status status);

@@ -50,6 +50,15 @@ struct sp_plan_s {
   int32_t last_active = -1;
 };
 
+struct sp_head_s {
+  int device = 0;
+  const int8_t* W = nullptr;
+  int64_t ldw = 0;
+  const float* scale = nullptr;
+  int32_t V = 0, K = 0;
+  uint8_t* ws = nullptr;          // head_workspace_bytes()
+};
+
 struct sp_group_s {
   int32_t count = 0;
   int32_t maxN = 0, maxK = 0;
@@ -734,6 +743,79 @@ sp_status spike_proj_dense(const sp_dense* problems, int32_t count, int32_t B,
   const sp_status st = check_device(&dev);
   if (st != SP_OK) return st;
   SP_CUDA(launch_dense(probs, count, B, as_stream(stream)));
+  return SP_OK;
+}
+
+// ---------------------------------------------------------------------------
+sp_status spike_proj_head_create(sp_head_t* head, const int8_t* W, int64_t ldw, const float* scale,
+                                 int32_t V, int32_t K, sp_stream_t stream) {
+  if (!head || !W || !scale) return SP_EINVAL;
+  if (V < 2 || V > SPIKE_PROJ_HEAD_MAX_V || K < 1 || K > SPIKE_PROJ_HEAD_MAX_K) return SP_ERANGE;
+  if (ldw < K || ldw % 16 != 0 || !aligned(W, 16) || !aligned(scale, 4)) return SP_EALIGN;
+  int dev = 0;
+  sp_status st = check_device(&dev);
+  if (st != SP_OK) return st;
+  cudaStream_t s = as_stream(stream);
+  sp_head_s* hd = new (std::nothrow) sp_head_s();
+  if (!hd) return SP_ENOMEM;
+  hd->device = dev;
+  hd->W = W;
+  hd->ldw = ldw;
+  hd->scale = scale;
+  hd->V = V;
+  hd->K = K;
+  if ((st = dev_alloc_zero(&hd->ws, head_workspace_bytes(), s)) != SP_OK) {
+    delete hd;
+    return st;
+  }
+  cudaError_t e = cudaStreamSynchronize(s);
+  if (e != cudaSuccess) {
+    cudaFree(hd->ws);
+    delete hd;
+    return cuda_fail(e);
+  }
+  *head = hd;
+  return SP_OK;
+}
+
+sp_status spike_proj_head_destroy(sp_head_t head) {
+  if (!head) return SP_OK;
+  cudaError_t e = cudaDeviceSynchronize();
+  cudaFree(head->ws);
+  delete head;
+  return e == cudaSuccess ? SP_OK : cuda_fail(e);
+}
+
+sp_status spike_proj_head(sp_head_t hd, const float* h, int64_t ldh, int32_t B, float tau,
+                          int32_t k_sel, int32_t* token, int32_t* verified, float* gap,
+                          int32_t* cand, float* r, float* z, int64_t ld_z, sp_stream_t stream) {
+  if (!hd || !h || !token || B < 1 || B > SPIKE_PROJ_HEAD_MAX_B) return SP_EINVAL;
+  if (k_sel < 1 || k_sel > SPIKE_PROJ_HEAD_MAX_CAND || k_sel > hd->V) return SP_EINVAL;
+  if (ldh < hd->K || (z && ld_z < hd->V)) return SP_EINVAL;
+  if (!aligned(h, 16) || ldh % 4 != 0) return SP_EALIGN;
+  if (!aligned(token, 4) || (verified && !aligned(verified, 4)) || (gap && !aligned(gap, 4)) ||
+      (cand && !aligned(cand, 4)) || (r && !aligned(r, 4)) || (z && !aligned(z, 4)))
+    return SP_EALIGN;
+  HeadArgs a;
+  a.W = hd->W;
+  a.ldw = hd->ldw;
+  a.scale = hd->scale;
+  a.V = hd->V;
+  a.K = hd->K;
+  a.h = h;
+  a.ldh = ldh;
+  a.B = B;
+  a.tau = tau;
+  a.k_sel = k_sel;
+  a.token = token;
+  a.verified = verified;
+  a.gap = gap;
+  a.cand = cand;
+  a.r = r;
+  a.z = z;
+  a.ld_z = ld_z;
+  a.ws = hd->ws;
+  SP_CUDA(launch_head(a, as_stream(stream)));
   return SP_OK;
 }
 

@@ -22,6 +22,7 @@
 // most 16 * ceil(K / 512) + 5, whatever the grid, so the error bound and the
 // result are the same on every run.
 #include "sp_ptx.cuh"
+#include "sp_rows.cuh"
 #include "sp_spikes.cuh"
 
 namespace sp {
@@ -45,29 +46,6 @@ struct DenseParams {
   DenseProblem prob[kDenseMaxProblems];
   int32_t unit_end[kDenseMaxProblems]; // prefix sums of each problem's units
 };
-
-// float(int8 byte e of w), exact: byte + 128 placed in the mantissa of 2^23
-__device__ __forceinline__ float byte_to_float(uint32_t w_biased, uint32_t e_sel) {
-  return __int_as_float((int)__byte_perm(w_biased, 0x4B000000u, 0x7650u | e_sel)) - 8388736.0f;
-}
-
-// x[k .. k+15] of one activation row, zero at and past K.
-__device__ __forceinline__ void load_x16(const float* __restrict__ xr, int k, int K, float (&v)[16]) {
-  if (k + 16 <= K) {
-    const float4* p = reinterpret_cast<const float4*>(xr + k);
-#pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      const float4 f = __ldg(p + q);
-      v[4 * q] = f.x;
-      v[4 * q + 1] = f.y;
-      v[4 * q + 2] = f.z;
-      v[4 * q + 3] = f.w;
-    }
-  } else {
-#pragma unroll
-    for (int e = 0; e < 16; ++e) v[e] = (k + e < K) ? __ldg(xr + k + e) : 0.f;
-  }
-}
 
 template <int B>
 __global__ void __launch_bounds__(kDenseThreads, DenseShape<B>::min_ctas)

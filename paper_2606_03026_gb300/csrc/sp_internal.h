@@ -154,6 +154,30 @@ cudaError_t launch_lif_rows(const float* vin, float* vout, const float* I, const
                             int rows, int64_t ld, float beta, float theta, uint32_t* bits,
                             int64_t ld_bits, cudaStream_t s);
 
+// One vocabulary-head call (see spike_proj_head); ws is the head's workspace
+// of head_workspace_bytes(), zero when created (the kernels leave it so).
+struct HeadArgs {
+  const int8_t* W;
+  int64_t ldw;
+  const float* scale;
+  int32_t V, K;
+  const float* h;
+  int64_t ldh;
+  int32_t B;
+  float tau;
+  int32_t k_sel;
+  int32_t* token;
+  int32_t* verified;
+  float* gap;
+  int32_t* cand;
+  float* r;
+  float* z;
+  int64_t ld_z;
+  void* ws;
+};
+size_t head_workspace_bytes();
+cudaError_t launch_head(const HeadArgs& a, cudaStream_t s);
+
 // Launches `kernel` with programmatic stream serialization: its blocks may
 // become resident while the previous kernel of the stream is still running
 // and wait for it in pdl_wait (see sp_ptx.cuh) before touching memory.

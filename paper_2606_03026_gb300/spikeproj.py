@@ -54,6 +54,10 @@ _SIGNATURES = {
     "spike_proj_dense": ([_P, _I32, _I32, _P], ctypes.c_int),
     "spike_proj_lif": ([_P, _P, _I32, _I32, _I64, ctypes.c_float, ctypes.c_float, _P, _I64, _P],
                        ctypes.c_int),
+    "spike_proj_head_create": ([_P, _P, _I64, _P, _I32, _I32, _P], ctypes.c_int),
+    "spike_proj_head_destroy": ([_P], ctypes.c_int),
+    "spike_proj_head": ([_P, _P, _I64, _I32, ctypes.c_float, _I32, _P, _P, _P, _P, _P, _P, _I64,
+                         _P], ctypes.c_int),
     "spike_proj_strerror": ([ctypes.c_int], ctypes.c_char_p),
     "spike_proj_last_cuda_error": ([], ctypes.c_int),
     "spike_proj_abi_version": ([], ctypes.c_int),
@@ -335,6 +339,53 @@ class Group:
     def close(self):
         if self.handle:
             spike_proj_group_destroy(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+def spike_proj_head_create(W, ldw, scale, V, K, stream=None) -> int:
+    h = ctypes.c_void_p()
+    _check(lib().spike_proj_head_create(ctypes.byref(h), _addr(W), ldw, _addr(scale), V, K,
+                                        _stream(stream)), "spike_proj_head_create")
+    return h.value
+
+
+def spike_proj_head_destroy(head):
+    _check(lib().spike_proj_head_destroy(head), "spike_proj_head_destroy")
+
+
+def spike_proj_head(head, h, ldh, B, tau, k_sel, token, verified=None, gap=None, cand=None, r=None,
+                    z=None, ld_z=0, stream=None):
+    _check(lib().spike_proj_head(head, _addr(h), ldh, B, tau, k_sel, _addr(token), _addr(verified),
+                                 _addr(gap), _addr(cand), _addr(r), _addr(z), ld_z,
+                                 _stream(stream)), "spike_proj_head")
+
+
+class Head:
+    """Vocabulary head with INT8 activations and candidate-row verification
+    over row-major INT8 weights W [V, ldw] and row scales [V] (borrowed)."""
+
+    def __init__(self, W, scale, K=None, stream=None):
+        self.W, self.scale = W, scale
+        self.V, self.ldw = W.shape
+        self.K = self.ldw if K is None else K
+        self.handle = spike_proj_head_create(W, self.ldw, scale, self.V, self.K, stream)
+
+    def __call__(self, h, tau, k_sel, token, verified=None, gap=None, cand=None, r=None, z=None,
+                 stream=None):
+        """h float32 [B, ldh]; outputs as spike_proj_head (tensors)."""
+        hs = h if h.dim() == 2 else h.reshape(1, -1)
+        spike_proj_head(self.handle, hs, hs.stride(0), hs.shape[0], tau, k_sel, token, verified,
+                        gap, cand, r, z, 0 if z is None else z.stride(0), stream)
+
+    def close(self):
+        if self.handle:
+            spike_proj_head_destroy(self.handle)
             self.handle = None
 
     def __del__(self):

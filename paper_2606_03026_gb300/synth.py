@@ -32,6 +32,8 @@ N_BLOCKS = 22             # decoder blocks, Section 2.1
 
 # workload ids used as the first word of every seed sequence
 _W_SINGLE, _W_DOWN, _W_STEP, _W_BATCH, _W_PREFILL, _W_DENSE, _W_MISC = 1, 2, 3, 4, 5, 6, 9
+_W_HEAD = 10
+VOCAB = 57344             # output vocabulary slots of the deployed configuration (Section 2.1)
 
 
 def rng_for(*words: int) -> np.random.Generator:
@@ -239,3 +241,36 @@ def dense_weights(block: int, kind: str, seed: int = 0, K: int = D_MODEL):
 def hidden_state(step: int, B: int = 1, seed: int = 0, K: int = D_MODEL):
     """Continuous activations x ~ N(0, 1), float32 [B, K]."""
     return rng_for(_W_DENSE, seed, 10_000 + step).standard_normal((B, K), dtype=np.float32)
+
+
+# --------------------------------------------------------------------------
+# vocabulary head (Section 5, trace configuration)
+# --------------------------------------------------------------------------
+HEAD_LOGIT_STD = 2.5
+
+
+def head_weights(seed: int = 0, V: int = VOCAB, K: int = D_MODEL,
+                 logit_std: float = HEAD_LOGIT_STD):
+    """Row-major INT8 head weights [V, K] and scale [V]: W ~ N(0, sigma^2)
+    with sigma = logit_std / sqrt(K), exported per output row (Section 2.3).
+    With N(0, 1) hidden states the logits then have standard deviation near
+    logit_std, and the top-two gap of 57,344 of them falls below 0.5 in
+    roughly the share of steps the paper's trace reports (54 of 80)."""
+    rng = rng_for(_W_HEAD, seed, V, K)
+    sigma = np.float32(logit_std / np.sqrt(K))
+    Qc = np.empty((K, V), dtype=np.int8)
+    s = np.empty(V, dtype=np.float32)
+    step = 8192
+    for m0 in range(0, V, step):            # row blocks: bounded float32 scratch
+        W = rng.standard_normal((min(step, V - m0), K), dtype=np.float32) * sigma
+        q, sb = quantise_per_channel(W)
+        Qc[:, m0:m0 + W.shape[0]] = q
+        s[m0:m0 + W.shape[0]] = sb
+    return np.ascontiguousarray(Qc.T), s
+
+
+def head_hidden(step: int, B: int = 1, seed: int = 0, K: int = D_MODEL):
+    """Final hidden states h ~ N(0, 1), float32 [B, K] (post-normalisation
+    scale)."""
+    return rng_for(_W_HEAD, seed, 20_000 + step).standard_normal((B, K), dtype=np.float32)
+

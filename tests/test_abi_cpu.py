@@ -85,6 +85,15 @@ def test_host_only_calls(lib):
         spikeproj.SP_ERANGE
     assert lib.spike_proj_group_decode_lif(None, fake, fake, fake, 64, 0.5, 1.0, None, 0, None,
                                            fake, 64, None) == spikeproj.SP_EINVAL
+    assert lib.spike_proj_head(None, fake, 64, 1, 0.5, 16, fake, None, None, None, None, None, 0,
+                               None) == spikeproj.SP_EINVAL
+    h = ctypes.c_void_p()
+    assert lib.spike_proj_head_create(None, fake, 64, fake, 100, 64, None) == spikeproj.SP_EINVAL
+    assert lib.spike_proj_head_create(ctypes.byref(h), fake, 64, fake, 1, 64, None) == \
+        spikeproj.SP_ERANGE
+    assert lib.spike_proj_head_create(ctypes.byref(h), fake, 72, fake, 100, 64, None) == \
+        spikeproj.SP_EALIGN
+    assert lib.spike_proj_head_destroy(None) == spikeproj.SP_OK
     assert lib.spike_proj_plan_destroy(None) == spikeproj.SP_OK
     assert lib.spike_proj_group_destroy(None) == spikeproj.SP_OK
 
