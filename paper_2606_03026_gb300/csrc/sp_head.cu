@@ -57,17 +57,20 @@ constexpr int kHeadCluster = 8;               // CTAs of the selection kernel
 constexpr int kSelThreads = 512;              // threads of a selection CTA
 constexpr int kSelWarps = kSelThreads / 32;
 constexpr int kHeadGatherLists = 128;         // most lists one gather_ge call takes
-constexpr int kHistWords = 256 + 65536;       // coarse and fine histograms of one hidden state
+constexpr int kHistBits = 12;                 // histogram bins: the keys' leading order bits
+constexpr int kHistWords = 1 << kHistBits;    // bins of one hidden state
 constexpr int kHeadMaxGrid = 1024;            // projection CTAs (lists) of one call
 static_assert(kHeadList == 64, "a list is two keys per lane");
+static_assert(SPIKE_PROJ_HEAD_MAX_K % (4 * 256) == 0, "the codes phase covers K in float4 per thread");
+static_assert(kSelThreads * 8 == kHistWords, "hist_bound: 8 bins per selection thread");
 static_assert(kHeadList == kHeadCluster * kHeadWarps, "one candidate per warp of a cluster");
 
 typedef unsigned long long hkey;
 
 // Workspace: the CTA lists (projection CTA c's list of hidden state b is
 // list (b * 8 + c % 8) * ceil(nlists / 8) + c / 8), then per hidden state
-// the histograms of the listed keys' order bits: 256 coarse bins (bits
-// 31-24) and 65536 fine bins (bits 31-16), zero between calls.
+// the histogram of the listed keys' 12 leading order bits (4096 bins, an
+// eighth of an octave of z each), zero between calls.
 constexpr size_t kListBytes = (size_t)SPIKE_PROJ_HEAD_MAX_B * kHeadMaxGrid * kHeadList * 8;
 constexpr size_t kHistBytes = (size_t)SPIKE_PROJ_HEAD_MAX_B * kHistWords * 4;
 
@@ -176,19 +179,16 @@ struct GatherScratch {
 };
 
 // Copies the keys >= T of the n sorted lists s[0 .. n) (64 keys each, in
-// shared memory; a prefix of each, found by binary search) into buf and
+// shared memory; a prefix of each) into buf and
 // returns their number, or -1 (nothing copied) when more than cap pass.
 // n <= kHeadGatherLists; every thread of the CTA calls it.
 __device__ int gather_ge(const hkey* s, int n, hkey T, hkey* buf, int cap, GatherScratch& sc) {
   const int t = threadIdx.x, nt = blockDim.x;
-  for (int l = t; l < n; l += nt) {
+  for (int l = t >> 5; l < n; l += nt >> 5) {    // a warp per list: its keys >= T, counted
     const hkey* L = s + (size_t)l * kHeadList;
-    int lo = 0, hi = kHeadList;                  // first index with key < T
-    while (lo < hi) {
-      const int mid = (lo + hi) >> 1;
-      if (L[mid] >= T) lo = mid + 1; else hi = mid;
-    }
-    sc.off[l] = lo;
+    const uint32_t b0 = __ballot_sync(0xffffffffu, L[t & 31] >= T);
+    const uint32_t b1 = __ballot_sync(0xffffffffu, L[32 + (t & 31)] >= T);
+    if ((t & 31) == 0) sc.off[l] = __popc(b0) + __popc(b1);
   }
   __syncthreads();
   if (t < 32) {                                  // exclusive scan, 4 lists per lane
@@ -248,17 +248,17 @@ __device__ void rank_place(const hkey* buf, int C, hkey* out) {
   __syncthreads();
 }
 
-// Over a 256-bin histogram h in global memory (bin i counts the keys whose
-// leading bits are i, so higher bins hold larger keys): the bin holding the
-// need-th largest key and the number of keys in the bins above it; false
-// when h holds fewer than need keys.  The 8 counts of lane l's bins
-// 8l .. 8l + 7 are left in c.  One full warp calls it.
-__device__ bool find_bin(const uint32_t* h, uint32_t need, int lane, uint32_t (&c)[8],
-                         uint32_t& bin, uint32_t& above) {
-  const uint4 q0 = __ldcg(reinterpret_cast<const uint4*>(h) + 2 * lane);
-  const uint4 q1 = __ldcg(reinterpret_cast<const uint4*>(h) + 2 * lane + 1);
-  c[0] = q0.x; c[1] = q0.y; c[2] = q0.z; c[3] = q0.w;
-  c[4] = q1.x; c[5] = q1.y; c[6] = q1.z; c[7] = q1.w;
+// The lower bound of the leading order bits of the histogram bin that holds
+// the need-th largest key, from a kHistWords-bin histogram in global memory
+// (bin i counts the keys whose leading bits are i): thread t of a
+// kSelThreads-thread CTA reads bins 8t .. 8t + 7, and the suffix sums meet in
+// two barriers.  0 when the histogram holds fewer than need keys.  Every
+// thread calls it.
+__device__ uint32_t hist_bound(const uint32_t* h, uint32_t need, uint32_t* s_wtot, uint32_t& s_bin) {
+  const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
+  const uint4 q0 = __ldcg(reinterpret_cast<const uint4*>(h) + 2 * t);
+  const uint4 q1 = __ldcg(reinterpret_cast<const uint4*>(h) + 2 * t + 1);
+  const uint32_t c[8] = {q0.x, q0.y, q0.z, q0.w, q1.x, q1.y, q1.z, q1.w};
   uint32_t sum = 0;
 #pragma unroll
   for (int i = 0; i < 8; ++i) sum += c[i];
@@ -268,22 +268,23 @@ __device__ bool find_bin(const uint32_t* h, uint32_t need, int lane, uint32_t (&
     const uint32_t o = __shfl_down_sync(0xffffffffu, S, d);
     if (lane + d < 32) S += o;
   }
-  const uint32_t hit = __ballot_sync(0xffffffffu, S >= need);
-  if (hit == 0u) return false;
-  const int L = 31 - __clz(hit);                 // the highest lane reaching need
-  uint32_t cum = __shfl_sync(0xffffffffu, S - sum, L);
-  bool found = false;
+  if (lane == 0) s_wtot[warp] = S;
+  if (t == 0) s_bin = 0u;
+  __syncthreads();
+  for (int w = warp + 1; w < (int)(blockDim.x >> 5); ++w) S += s_wtot[w];
+  if (S >= need && S - sum < need) {             // this thread's bins hold the need-th key
+    uint32_t cum = S - sum;
 #pragma unroll
-  for (int i = 7; i >= 0; --i) {
-    const uint32_t ci = __shfl_sync(0xffffffffu, c[i], L);
-    if (!found && cum + ci >= need) {
-      bin = (uint32_t)(8 * L + i);
-      above = cum;
-      found = true;
+    for (int i = 7; i >= 0; --i) {
+      if (cum + c[i] >= need) {
+        s_bin = (uint32_t)(8 * t + i) << (32 - kHistBits);
+        break;
+      }
+      cum += c[i];
     }
-    cum += ci;
   }
-  return true;
+  __syncthreads();
+  return s_bin;
 }
 
 __device__ __forceinline__ uint32_t peer_addr(const void* local, uint32_t rank) {
@@ -370,30 +371,54 @@ head_kernel(const __grid_constant__ HeadParams p) {
   }
   pdl_wait();
 
-  // 1. activation scale and INT8 codes of each hidden state (zero past K)
-#pragma unroll
+  // 1. activation scale and INT8 codes of each hidden state (zero past K):
+  // thread t holds h[4t + 1024 i .. +3] in registers (one read of h), the
+  // CTA's maximum |h| meets in one barrier, every thread derives s_x
+#pragma unroll 1
   for (int b = 0; b < B; ++b) {
     const float* hb = p.h + (int64_t)b * p.ldh;
+    constexpr int kHv = SPIKE_PROJ_HEAD_MAX_K / (4 * kHeadThreads);
+    float4 hv[kHv];
     float mx = 0.f;
-    for (int k = threadIdx.x; k < p.K; k += kHeadThreads) mx = fmaxf(mx, fabsf(hb[k]));
+#pragma unroll
+    for (int i = 0; i < kHv; ++i) {
+      const int k = 4 * (int)threadIdx.x + 4 * kHeadThreads * i;
+      hv[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (k + 4 <= p.K) {
+        hv[i] = __ldg(reinterpret_cast<const float4*>(hb + k));   // h 16-byte aligned, ldh % 4 == 0
+      } else if (k < p.K) {
+        hv[i].x = hb[k];
+        if (k + 1 < p.K) hv[i].y = hb[k + 1];
+        if (k + 2 < p.K) hv[i].z = hb[k + 2];
+      }
+      mx = fmaxf(mx, fmaxf(fmaxf(fabsf(hv[i].x), fabsf(hv[i].y)), fmaxf(fabsf(hv[i].z), fabsf(hv[i].w))));
+    }
 #pragma unroll
     for (int d = 16; d >= 1; d >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, d));
     if (lane == 0) s_red[warp] = mx;
     __syncthreads();
-    if (threadIdx.x == 0) {
-      float a = s_red[0];
-      for (int w = 1; w < kHeadWarps; ++w) a = fmaxf(a, s_red[w]);
-      s_sx[b] = __fdiv_rn(fmaxf(a, 1e-8f), 127.0f);
+    float a = s_red[0];
+#pragma unroll
+    for (int w = 1; w < kHeadWarps; ++w) a = fmaxf(a, s_red[w]);
+    const float sx = __fdiv_rn(fmaxf(a, 1e-8f), 127.0f);
+    if (threadIdx.x == 0) s_sx[b] = sx;
+#pragma unroll
+    for (int i = 0; i < kHv; ++i) {
+      const int k = 4 * (int)threadIdx.x + 4 * kHeadThreads * i;
+      if (k < p.Kpad) {
+        const float e[4] = {hv[i].x, hv[i].y, hv[i].z, hv[i].w};
+        uint32_t packed = 0;
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          int c = 0;
+          if (k + j < p.K) c = (int)fminf(fmaxf(rintf(__fdiv_rn(e[j], sx)), -127.0f), 127.0f);
+          packed |= ((uint32_t)c & 0xffu) << (8 * j);
+        }
+        *reinterpret_cast<uint32_t*>(s_codes + b * p.Kpad + k) = packed;
+      }
     }
-    __syncthreads();
-    const float sx = s_sx[b];
-    for (int k = threadIdx.x; k < p.Kpad; k += kHeadThreads) {
-      int c = 0;
-      if (k < p.K) c = (int)fminf(fmaxf(rintf(__fdiv_rn(hb[k], sx)), -127.0f), 127.0f);
-      s_codes[b * p.Kpad + k] = (int8_t)c;
-    }
+    __syncthreads();                             // s_red is rewritten by the next hidden state
   }
-  __syncthreads();
 
   // 2. approximate logits; each warp keeps its best 64 keys per hidden state
   hkey la[B], lb[B], pend[B];
@@ -480,16 +505,13 @@ head_kernel(const __grid_constant__ HeadParams p) {
     if (threadIdx.x < kHeadList) {
       const hkey k = s_all[threadIdx.x];
       __stcg(p.lists + slot * kHeadList + threadIdx.x, k);
-      // the listed keys into the histograms (equal bins of a warp summed
+      // the listed keys into the histogram (equal bins of a warp summed
       // first): every key of the final selection is a listed key
       const uint32_t real = __ballot_sync(0xffffffffu, k != 0ull);
       if (k != 0ull) {
-        uint32_t* hc = p.hist + (int64_t)b * kHistWords;
-        const uint32_t ob = (uint32_t)(k >> 32);
-        const uint32_t mf = __match_any_sync(real, ob >> 16);
-        if (lane == __ffs(mf) - 1) atomicAdd(hc + 256 + (ob >> 16), (uint32_t)__popc(mf));
-        const uint32_t mc = __match_any_sync(real, ob >> 24);
-        if (lane == __ffs(mc) - 1) atomicAdd(hc + (ob >> 24), (uint32_t)__popc(mc));
+        const uint32_t bin = (uint32_t)(k >> (64 - kHistBits));
+        const uint32_t mb = __match_any_sync(real, bin);
+        if (lane == __ffs(mb) - 1) atomicAdd(p.hist + (int64_t)b * kHistWords + bin, (uint32_t)__popc(mb));
       }
     }
     __syncthreads();
@@ -511,11 +533,12 @@ head_select_kernel(const __grid_constant__ HeadParams p) {
   __shared__ hkey s_best[kHeadList];
   __shared__ hkey s_buf[kSelThreads];
   __shared__ GatherScratch s_gs;
-  __shared__ uint32_t s_coarse[256];
-  __shared__ hkey s_T;
+  __shared__ uint32_t s_wtot[kSelWarps];
+  __shared__ uint32_t s_bin;
   __shared__ hkey s_final[kHeadList];
   __shared__ float s_r[kHeadList];
-  __shared__ uint32_t s_open, s_bad, s_dirty;
+  __shared__ uint32_t s_open, s_bad, s_ok;
+  __shared__ float s_gap;
   __shared__ __align__(8) uint64_t s_bar;
 
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -534,20 +557,6 @@ head_select_kernel(const __grid_constant__ HeadParams p) {
   pdl_wait();                                    // every CTA list is written
   for (int b = 0; b < p.B; ++b) {
     uint32_t* hc = p.hist + (int64_t)b * kHistWords;
-    if (warp == 1) {
-      // the bound T: the fine bin holding the 64th best listed key (every
-      // CTA finds it; no key of the final 64 lies below T)
-      uint32_t c[8], cb = 0, above = 0;
-      hkey T = 1ull;                             // fewer than 64 keys: all pass
-      if (find_bin(hc, kHeadList, lane, c, cb, above)) {
-        uint32_t cf[8], fb = 0, above2 = 0;
-        if (find_bin(hc + 256 + cb * 256, kHeadList - above, lane, cf, fb, above2))
-          T = (hkey)((cb << 24) | (fb << 16)) << 32;
-      }
-#pragma unroll
-      for (int i = 0; i < 8; ++i) s_coarse[8 * lane + i] = c[i];
-      if (lane == 0) s_T = T;
-    }
     if (threadIdx.x == 0 && mine > 0) {
       // the previous hidden state's reads and writes of s_mine (generic
       // proxy) come before this copy's writes (async proxy)
@@ -555,13 +564,18 @@ head_select_kernel(const __grid_constant__ HeadParams p) {
       const uint32_t bytes = (uint32_t)mine * kHeadList * 8;
       mbar_arrive_expect_tx(&s_bar, bytes);
       bulk_load(s_mine, p.lists + (int64_t)(b * csize + (int)rank) * n8 * kHeadList, bytes, &s_bar);
-      if (!mbar_wait(&s_bar, (uint32_t)(b & 1))) s_bad = 1;
     }
+    // while the lists arrive, the bound T: the histogram bin holding the
+    // 64th best listed key (every CTA finds it; no key of the final 64 lies
+    // below T)
+    const uint32_t tb = hist_bound(hc, kHeadList, s_wtot, s_bin);
+    const hkey T = tb ? (hkey)tb << 32 : 1ull;   // no bound: every key passes
+    if (threadIdx.x == 0 && mine > 0 && !mbar_wait(&s_bar, (uint32_t)(b & 1))) s_bad = 1;
     __syncthreads();
     const int have = s_bad ? 0 : mine;
     // this CTA's best 64 of its keys >= T (all of them, more than
     // kSelThreads only for adversarial spreads: then the merge tree)
-    const int C = gather_ge(s_mine, have, s_T, s_buf, kSelThreads, s_gs);
+    const int C = gather_ge(s_mine, have, T, s_buf, kSelThreads, s_gs);
     if (C >= 0) {
       rank_place(s_buf, C, s_best);
     } else {
@@ -577,10 +591,10 @@ head_select_kernel(const __grid_constant__ HeadParams p) {
       rank_place(s_buf, C0, s_best);             // C0 <= 8 * 64 = kSelThreads
       const hkey* fin = s_best;
       // The 64 best keys >= T are the 64 best keys when at least min(V, 64)
-      // keys pass T, which holds whenever the histograms counted exactly
-      // this call's listed keys; fewer (histograms left dirty by a call that
-      // never reached this kernel) or a failed copy: token -1, and every bin
-      // is cleared below.
+      // keys pass T, which holds whenever the histogram counted exactly this
+      // call's listed keys; fewer (a histogram left dirty by a call that
+      // never reached this kernel) or a failed copy: token -1 (the histogram
+      // is cleared at the end either way).
       const bool ok = s_bad == 0 && C0 >= min(p.V, kHeadList);
       const float g = __fsub_rn(key_z(fin[0]), key_z(fin[1]));
       const uint32_t open = ok && g < p.tau ? 1u : 0u;
@@ -589,25 +603,14 @@ head_select_kernel(const __grid_constant__ HeadParams p) {
         for (int r = 0; r < csize; ++r) st_peer_key(peer_addr(&s_final[threadIdx.x], (uint32_t)r), k);
       }
       if (threadIdx.x == 0) {
-        for (int r = 0; r < csize; ++r) {
-          st_peer_u32(peer_addr(&s_open, (uint32_t)r), open);
-          st_peer_u32(peer_addr(&s_dirty, (uint32_t)r), ok ? 0u : 1u);
-        }
-        p.token[b] = ok ? key_row(fin[0]) : -1;  // replaced below when verified
-        if (p.verified) p.verified[b] = (int)open;
-        if (p.gap) p.gap[b] = g;
+        for (int r = 0; r < csize; ++r) st_peer_u32(peer_addr(&s_open, (uint32_t)r), open);
+        s_ok = ok ? 1u : 0u;
+        s_gap = g;
       }
-      if (p.cand && (int)threadIdx.x < ks) p.cand[(int64_t)b * ks + threadIdx.x] = key_row(fin[threadIdx.x]);
     }
-    cluster_sync();                              // s_final, s_open and s_dirty everywhere
-    // every CTA has read the histograms: clear the fine bins of the coarse
-    // bins r, r + 8, ... that counted keys (all of them after a failed
-    // check), and CTA 0 the coarse bins, for the next call
-    for (int i = threadIdx.x; i < (256 / kHeadCluster) * 256; i += kSelThreads) {
-      const int cbin = (int)rank + kHeadCluster * (i >> 8);
-      if (s_coarse[cbin] || s_dirty) hc[256 + cbin * 256 + (i & 255)] = 0u;
-    }
-    if (rank == 0 && threadIdx.x < 256) hc[threadIdx.x] = 0u;
+    // (global stores come after the cluster barriers: a barrier's release
+    // would wait for them)
+    cluster_sync();                              // s_final and s_open everywhere
     if (s_open && warp < kHeadWarps) {
       const float* hb = p.h + (int64_t)b * p.ldh;
       for (int i = (int)rank + csize * warp; i < ks; i += csize * kHeadWarps) {
@@ -616,6 +619,14 @@ head_select_kernel(const __grid_constant__ HeadParams p) {
       }
     }
     cluster_sync();                              // every r in CTA 0
+    if (rank == 0) {
+      if (threadIdx.x == 0) {
+        if (!s_open) p.token[b] = s_ok ? key_row(s_final[0]) : -1;
+        if (p.verified) p.verified[b] = (int)s_open;
+        if (p.gap) p.gap[b] = s_gap;
+      }
+      if (p.cand && (int)threadIdx.x < ks) p.cand[(int64_t)b * ks + threadIdx.x] = key_row(s_final[threadIdx.x]);
+    }
     if (rank == 0 && s_open && warp == 0) {
       // largest r, equal r: lower row (starting from candidate 0, so the
       // token is always a candidate)
@@ -650,6 +661,11 @@ head_select_kernel(const __grid_constant__ HeadParams p) {
     // one more barrier.
     if (b + 1 < p.B) cluster_sync();
   }
+  // every CTA has read the histograms: CTA r clears bins 512 r .. 512 r + 511
+  // of each hidden state's for the next call
+  for (int b = 0; b < p.B; ++b)
+    for (int i = threadIdx.x; i < kHistWords / kHeadCluster; i += kSelThreads)
+      p.hist[(int64_t)b * kHistWords + (int)rank * (kHistWords / kHeadCluster) + i] = 0u;
 }
 
 int g_head_sms = 0;
