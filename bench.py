@@ -888,8 +888,11 @@ def bench_head(torch, sp, synth, dev, stream, peaks, peak_kind, with_oracle=True
     res["headline"] = {"config": "B=1, tau=0.5, k_sel=64", "us_per_token": us, "gbs": gbs,
                        "tokens_per_s": 1e6 / us}
     res["roofline"] = {"bound": "hbm", "achieved": gbs, "peak": hbm, "unit": "GB/s",
-                       "frac": gbs / hbm, "peak_kind": peak_kind,
-                       "bytes_per_call": V * K, "note": "algorithmic bytes = V*K weight bytes"}
+                       "frac": gbs / hbm, "peak_kind": peak_kind, "bytes_per_call": V * K,
+                       "traffic": measured_traffic("head_kernel", "sp_head.cu"),
+                       "note": "algorithmic bytes = V*K weight bytes; achieved over the whole "
+                               "call (projection and selection launches); traffic = ncu DRAM "
+                               "bytes of one projection launch (B = 1)"}
     res["verification_cost_us"] = table["B1_tauinf_k64"]["us"] - table["B1_tau0.0_k64"]["us"]
     # spot check of the last graph's calls (B = 4, tau = inf, k_sel = 64) against the oracle
     bad = 0
