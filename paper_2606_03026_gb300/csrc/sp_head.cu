@@ -29,18 +29,19 @@
 // keys are distinct) and the warp keeps its best 64 keys in a sorted list
 // (bitonic sort of 32 new keys, then a bitonic merge with the list).
 //
-// The selection is a tree of pairwise bitonic merges of 64-key lists.  The
-// CTA merges its 8 warp lists in shared memory and writes one list to the
-// workspace.  A second kernel, one cluster of 8 CTAs of 512 threads
-// launched as the programmatic dependent of the first, merges those lists:
-// CTA r the lists of projection CTAs r, r + 8, ... (stored contiguously, so
-// one bulk copy brings them into shared memory), CTA 0 the eight results.  CTA 0 applies the gate, the
-// cluster's 64 warps recompute one candidate each, and CTA 0 picks the token.
-// Results move between the CTAs of the cluster by stores into the receiver's
-// shared memory, each followed by a cluster barrier before the receiver
-// reads.  The projection kernel is launched without clusters and with little
-// shared memory: a cluster launch or a larger shared-memory carve-out slows
-// its weight stream (fewer resident CTAs, less L1 for loads in flight).
+// Every key of the final 64 is in some CTA's list, so the CTA lists are all
+// that the selection reads.  Each projection CTA merges its 8 warp lists in
+// shared memory (a tree of pairwise bitonic merges), writes one list to the
+// workspace, and counts the list's keys in a 4096-bin histogram of their 12
+// leading order bits.  A second kernel, one CTA launched as the programmatic
+// dependent of the first, takes as a lower bound T the histogram bin that
+// holds the 64th best listed key, and in the same round of loads the first
+// 4 keys of every list.  The keys >= T (about seventy) are gathered (the
+// rest of a list is fetched only when all 4 of its leading keys pass),
+// ordered by counting, gated, and the candidates recomputed, 4 rows per warp
+// with all their loads in flight.  The projection kernel has little shared
+// memory and no clusters: a larger shared-memory carve-out or a cluster
+// launch slowed its weight stream.
 #include "sp_internal.h"
 #include "sp_ptx.cuh"
 #include "sp_rows.cuh"
@@ -53,24 +54,23 @@ constexpr int kHeadThreads = 256;
 constexpr int kHeadWarps = kHeadThreads / 32;
 constexpr int kHeadRows = 4;                  // rows per unit (one warp)
 constexpr int kHeadList = SPIKE_PROJ_HEAD_MAX_CAND;   // keys per sorted list
-constexpr int kHeadCluster = 8;               // CTAs of the selection kernel
-constexpr int kSelThreads = 512;              // threads of a selection CTA
+constexpr int kSelThreads = 512;              // threads of the selection CTA
 constexpr int kSelWarps = kSelThreads / 32;
-constexpr int kHeadGatherLists = 128;         // most lists one gather_ge call takes
+constexpr int kLead = 4;                      // leading keys of each list read first
 constexpr int kHistBits = 12;                 // histogram bins: the keys' leading order bits
 constexpr int kHistWords = 1 << kHistBits;    // bins of one hidden state
 constexpr int kHeadMaxGrid = 1024;            // projection CTAs (lists) of one call
 static_assert(kHeadList == 64, "a list is two keys per lane");
 static_assert(SPIKE_PROJ_HEAD_MAX_K % (4 * 256) == 0, "the codes phase covers K in float4 per thread");
 static_assert(kSelThreads * 8 == kHistWords, "hist_bound: 8 bins per selection thread");
-static_assert(kHeadList == kHeadCluster * kHeadWarps, "one candidate per warp of a cluster");
+static_assert(kHeadList == 4 * kSelWarps, "four candidates per selection warp");
 
 typedef unsigned long long hkey;
 
 // Workspace: the CTA lists (projection CTA c's list of hidden state b is
-// list (b * 8 + c % 8) * ceil(nlists / 8) + c / 8), then per hidden state
-// the histogram of the listed keys' 12 leading order bits (4096 bins, an
-// eighth of an octave of z each), zero between calls.
+// list b * nlists + c), then per hidden state the histogram of the listed
+// keys' 12 leading order bits (4096 bins, an eighth of an octave of z
+// each), zero between calls.
 constexpr size_t kListBytes = (size_t)SPIKE_PROJ_HEAD_MAX_B * kHeadMaxGrid * kHeadList * 8;
 constexpr size_t kHistBytes = (size_t)SPIKE_PROJ_HEAD_MAX_B * kHistWords * 4;
 
@@ -172,60 +172,6 @@ __device__ void tree_merge(hkey* s, int n, int nw) {
   }
 }
 
-// Scratch of gather_ge (shared memory).
-struct GatherScratch {
-  int off[kHeadGatherLists];       // keys per list that pass the bound, then offsets
-  int total;
-};
-
-// Copies the keys >= T of the n sorted lists s[0 .. n) (64 keys each, in
-// shared memory; a prefix of each) into buf and
-// returns their number, or -1 (nothing copied) when more than cap pass.
-// n <= kHeadGatherLists; every thread of the CTA calls it.
-__device__ int gather_ge(const hkey* s, int n, hkey T, hkey* buf, int cap, GatherScratch& sc) {
-  const int t = threadIdx.x, nt = blockDim.x;
-  for (int l = t >> 5; l < n; l += nt >> 5) {    // a warp per list: its keys >= T, counted
-    const hkey* L = s + (size_t)l * kHeadList;
-    const uint32_t b0 = __ballot_sync(0xffffffffu, L[t & 31] >= T);
-    const uint32_t b1 = __ballot_sync(0xffffffffu, L[32 + (t & 31)] >= T);
-    if ((t & 31) == 0) sc.off[l] = __popc(b0) + __popc(b1);
-  }
-  __syncthreads();
-  if (t < 32) {                                  // exclusive scan, 4 lists per lane
-    int v[4], sum = 0;
-#pragma unroll
-    for (int e = 0; e < 4; ++e) {
-      const int l = 4 * t + e;
-      v[e] = l < n ? sc.off[l] : 0;
-      sum += v[e];
-    }
-    int inc = sum;
-#pragma unroll
-    for (int d = 1; d < 32; d <<= 1) {
-      const int o = __shfl_up_sync(0xffffffffu, inc, d);
-      if (t >= d) inc += o;
-    }
-    int o = inc - sum;
-#pragma unroll
-    for (int e = 0; e < 4; ++e) {
-      const int l = 4 * t + e;
-      if (l < n) sc.off[l] = o;
-      o += v[e];
-    }
-    if (t == 31) sc.total = inc;
-  }
-  __syncthreads();
-  const int C = sc.total;
-  if (C > cap) return -1;
-  const int lane = t & 31;
-  for (int l = t >> 5; l < n; l += nt >> 5) {    // a warp per list, a lane per key
-    const int o = sc.off[l], c = (l + 1 < n ? sc.off[l + 1] : C) - o;
-    for (int e = lane; e < c; e += 32) buf[o + e] = s[(size_t)l * kHeadList + e];
-  }
-  __syncthreads();
-  return C;
-}
-
 // out[0 .. 64) <- the best min(C, 64) of the C distinct keys buf[0 .. C),
 // descending (each placed by counting the larger ones), 0 past C.
 __device__ void rank_place(const hkey* buf, int C, hkey* out) {
@@ -287,60 +233,101 @@ __device__ uint32_t hist_bound(const uint32_t* h, uint32_t need, uint32_t* s_wto
   return s_bin;
 }
 
-__device__ __forceinline__ uint32_t peer_addr(const void* local, uint32_t rank) {
-  uint32_t a;
-  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;"
-               : "=r"(a)
-               : "r"((uint32_t)__cvta_generic_to_shared(local)), "r"(rank));
-  return a;
-}
-__device__ __forceinline__ void st_peer_key(uint32_t a, hkey v) {
-  asm volatile("st.shared::cluster.u64 [%0], %1;" ::"r"(a), "l"(v) : "memory");
-}
-__device__ __forceinline__ void st_peer_u32(uint32_t a, uint32_t v) {
-  asm volatile("st.shared::cluster.u32 [%0], %1;" ::"r"(a), "r"(v) : "memory");
-}
-__device__ __forceinline__ uint32_t cluster_rank() {
-  uint32_t r;
-  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
-  return r;
-}
-// Every thread of every CTA of the cluster: stores before it are visible to
-// loads after it.
-__device__ __forceinline__ void cluster_sync() {
-  asm volatile("barrier.cluster.arrive.release;\n\tbarrier.cluster.wait.acquire;" ::: "memory");
-}
-
-// r of candidate row m for hidden state hb: lane l sums the 16-byte chunks
-// l, l + 32, ... in ascending k with fmaf, then the 5-level butterfly; loads
-// of up to 4 chunks are in flight together.
-__device__ __forceinline__ float verify_row(const HeadParams& p, const float* hb, int m, int lane) {
-  const int8_t* wr = p.W + (int64_t)m * p.ldw;
+// r of up to 4 candidate rows (rows[j], j < n) for hidden state hb, by one
+// warp: per row, lane l sums the 16-byte chunks l, l + 32, ... in ascending k
+// with fmaf, then the 5-level butterfly (the continuous-input kernel's
+// order); the loads of all the rows and of up to 4 chunks are in flight
+// together.
+__device__ __forceinline__ void verify_rows4(const HeadParams& p, const float* hb, const int (&rows)[4],
+                                             int n, int lane, float (&out)[4]) {
   const int nch = (p.K + 511) / 512;
-  float acc = 0.f;
+  float acc[4] = {0.f, 0.f, 0.f, 0.f};
   for (int c0 = 0; c0 < nch; c0 += 4) {
-    uint4 v[4];
+    uint4 v[4][4];
 #pragma unroll
-    for (int t = 0; t < 4; ++t) {
-      const int k = 16 * (lane + 32 * (c0 + t));
-      if (c0 + t < nch && k < p.K) v[t] = ld_weights16(wr + k);
-    }
+    for (int j = 0; j < 4; ++j)
+#pragma unroll
+      for (int t = 0; t < 4; ++t) {
+        const int k = 16 * (lane + 32 * (c0 + t));
+        if (j < n && c0 + t < nch && k < p.K) v[j][t] = ld_weights16(p.W + (int64_t)rows[j] * p.ldw + k);
+      }
 #pragma unroll
     for (int t = 0; t < 4; ++t) {
       const int k = 16 * (lane + 32 * (c0 + t));
       if (c0 + t < nch && k < p.K) {
         float x[16];
         load_x16(hb, k, p.K, x);
-        const uint32_t ww[4] = {v[t].x ^ 0x80808080u, v[t].y ^ 0x80808080u, v[t].z ^ 0x80808080u,
-                                v[t].w ^ 0x80808080u};
 #pragma unroll
-        for (int e = 0; e < 16; ++e) acc = fmaf(byte_to_float(ww[e >> 2], (uint32_t)(e & 3)), x[e], acc);
+        for (int j = 0; j < 4; ++j) {
+          if (j < n) {
+            const uint32_t ww[4] = {v[j][t].x ^ 0x80808080u, v[j][t].y ^ 0x80808080u,
+                                    v[j][t].z ^ 0x80808080u, v[j][t].w ^ 0x80808080u};
+#pragma unroll
+            for (int e = 0; e < 16; ++e)
+              acc[j] = fmaf(byte_to_float(ww[e >> 2], (uint32_t)(e & 3)), x[e], acc[j]);
+          }
+        }
       }
     }
   }
 #pragma unroll
-  for (int d = 16; d >= 1; d >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, d);
-  return __fmul_rn(__ldg(p.scale + m), acc);
+  for (int j = 0; j < 4; ++j) {
+#pragma unroll
+    for (int d = 16; d >= 1; d >>= 1) acc[j] += __shfl_xor_sync(0xffffffffu, acc[j], d);
+    out[j] = j < n ? __fmul_rn(__ldg(p.scale + rows[j]), acc[j]) : 0.f;
+  }
+}
+
+// Step 1 for every hidden state: thread t holds h[4t + 1024 i .. +3], i < NV,
+// in registers (one read of h); the CTA's maximum |h| meets in one barrier
+// and every thread derives s_x; the codes go to shared memory four to a word.
+template <int B, int NV>
+__device__ __forceinline__ void head_codes(const HeadParams& p, int8_t* s_codes, float* s_red, float* s_sx) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+#pragma unroll 1
+  for (int b = 0; b < B; ++b) {
+    const float* hb = p.h + (int64_t)b * p.ldh;
+    float4 hv[NV];
+    float mx = 0.f;
+#pragma unroll
+    for (int i = 0; i < NV; ++i) {
+      const int k = 4 * (int)threadIdx.x + 4 * kHeadThreads * i;
+      hv[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (k + 4 <= p.K) {
+        hv[i] = __ldg(reinterpret_cast<const float4*>(hb + k));   // h 16-byte aligned, ldh % 4 == 0
+      } else if (k < p.K) {
+        hv[i].x = hb[k];
+        if (k + 1 < p.K) hv[i].y = hb[k + 1];
+        if (k + 2 < p.K) hv[i].z = hb[k + 2];
+      }
+      mx = fmaxf(mx, fmaxf(fmaxf(fabsf(hv[i].x), fabsf(hv[i].y)), fmaxf(fabsf(hv[i].z), fabsf(hv[i].w))));
+    }
+#pragma unroll
+    for (int d = 16; d >= 1; d >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, d));
+    if (lane == 0) s_red[warp] = mx;
+    __syncthreads();
+    float a = s_red[0];
+#pragma unroll
+    for (int w = 1; w < kHeadWarps; ++w) a = fmaxf(a, s_red[w]);
+    const float sx = __fdiv_rn(fmaxf(a, 1e-8f), 127.0f);
+    if (threadIdx.x == 0) s_sx[b] = sx;
+#pragma unroll
+    for (int i = 0; i < NV; ++i) {
+      const int k = 4 * (int)threadIdx.x + 4 * kHeadThreads * i;
+      if (k < p.Kpad) {
+        const float e[4] = {hv[i].x, hv[i].y, hv[i].z, hv[i].w};
+        uint32_t packed = 0;
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          int c = 0;
+          if (k + j < p.K) c = (int)fminf(fmaxf(rintf(__fdiv_rn(e[j], sx)), -127.0f), 127.0f);
+          packed |= ((uint32_t)c & 0xffu) << (8 * j);
+        }
+        *reinterpret_cast<uint32_t*>(s_codes + b * p.Kpad + k) = packed;
+      }
+    }
+    __syncthreads();                             // s_red is rewritten by the next hidden state
+  }
 }
 
 template <int B> struct HeadShape { static constexpr int min_ctas = 2; };
@@ -371,54 +358,11 @@ head_kernel(const __grid_constant__ HeadParams p) {
   }
   pdl_wait();
 
-  // 1. activation scale and INT8 codes of each hidden state (zero past K):
-  // thread t holds h[4t + 1024 i .. +3] in registers (one read of h), the
-  // CTA's maximum |h| meets in one barrier, every thread derives s_x
-#pragma unroll 1
-  for (int b = 0; b < B; ++b) {
-    const float* hb = p.h + (int64_t)b * p.ldh;
-    constexpr int kHv = SPIKE_PROJ_HEAD_MAX_K / (4 * kHeadThreads);
-    float4 hv[kHv];
-    float mx = 0.f;
-#pragma unroll
-    for (int i = 0; i < kHv; ++i) {
-      const int k = 4 * (int)threadIdx.x + 4 * kHeadThreads * i;
-      hv[i] = make_float4(0.f, 0.f, 0.f, 0.f);
-      if (k + 4 <= p.K) {
-        hv[i] = __ldg(reinterpret_cast<const float4*>(hb + k));   // h 16-byte aligned, ldh % 4 == 0
-      } else if (k < p.K) {
-        hv[i].x = hb[k];
-        if (k + 1 < p.K) hv[i].y = hb[k + 1];
-        if (k + 2 < p.K) hv[i].z = hb[k + 2];
-      }
-      mx = fmaxf(mx, fmaxf(fmaxf(fabsf(hv[i].x), fabsf(hv[i].y)), fmaxf(fabsf(hv[i].z), fabsf(hv[i].w))));
-    }
-#pragma unroll
-    for (int d = 16; d >= 1; d >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, d));
-    if (lane == 0) s_red[warp] = mx;
-    __syncthreads();
-    float a = s_red[0];
-#pragma unroll
-    for (int w = 1; w < kHeadWarps; ++w) a = fmaxf(a, s_red[w]);
-    const float sx = __fdiv_rn(fmaxf(a, 1e-8f), 127.0f);
-    if (threadIdx.x == 0) s_sx[b] = sx;
-#pragma unroll
-    for (int i = 0; i < kHv; ++i) {
-      const int k = 4 * (int)threadIdx.x + 4 * kHeadThreads * i;
-      if (k < p.Kpad) {
-        const float e[4] = {hv[i].x, hv[i].y, hv[i].z, hv[i].w};
-        uint32_t packed = 0;
-#pragma unroll
-        for (int j = 0; j < 4; ++j) {
-          int c = 0;
-          if (k + j < p.K) c = (int)fminf(fmaxf(rintf(__fdiv_rn(e[j], sx)), -127.0f), 127.0f);
-          packed |= ((uint32_t)c & 0xffu) << (8 * j);
-        }
-        *reinterpret_cast<uint32_t*>(s_codes + b * p.Kpad + k) = packed;
-      }
-    }
-    __syncthreads();                             // s_red is rewritten by the next hidden state
-  }
+  // 1. activation scale and INT8 codes of each hidden state (zero past K);
+  // a compact form for K <= 2048 (the code runs once per CTA, and its size
+  // shows in the start-up)
+  if (p.K <= 2 * 4 * kHeadThreads) head_codes<B, 2>(p, s_codes, s_red, s_sx);
+  else head_codes<B, SPIKE_PROJ_HEAD_MAX_K / (4 * kHeadThreads)>(p, s_codes, s_red, s_sx);
 
   // 2. approximate logits; each warp keeps its best 64 keys per hidden state
   hkey la[B], lb[B], pend[B];
@@ -499,9 +443,7 @@ head_kernel(const __grid_constant__ HeadParams p) {
     s_all[warp * kHeadList + 32 + lane] = lb[b];
     __syncthreads();
     tree_merge(s_all, kHeadWarps, kHeadWarps);
-    const int n8 = (p.nlists + kHeadCluster - 1) / kHeadCluster;
-    const int64_t slot = (int64_t)(b * kHeadCluster + (int)blockIdx.x % kHeadCluster) * n8 +
-                         (int)blockIdx.x / kHeadCluster;
+    const int64_t slot = (int64_t)b * p.nlists + blockIdx.x;
     if (threadIdx.x < kHeadList) {
       const hkey k = s_all[threadIdx.x];
       __stcg(p.lists + slot * kHeadList + threadIdx.x, k);
@@ -518,154 +460,156 @@ head_kernel(const __grid_constant__ HeadParams p) {
   }
 }
 
-// Steps 3-6: one cluster of kHeadCluster CTAs.  Per hidden state, CTA r
-// merges the lists of projection CTAs r, r + 8, ... and pushes the result
-// into CTA 0's s_part[r]; CTA 0 merges those, applies the gate and pushes the
-// final list; warps 0-7 of each CTA recompute one candidate each and push r
-// to CTA 0, which picks the token.  A bulk copy that does not complete
-// within the bounded wait leaves the CTA's share empty and the call reports
-// token -1 (no candidate of an incomplete list is ever read).
+// Steps 3-6, one CTA of kSelThreads threads, per hidden state: the bound T
+// and the leading keys of every list (one round of loads for both), the
+// keys >= T, the best 64 of them by counting, the gate, the candidates
+// recomputed (warp w: candidates w, w + 16, w + 32, w + 48), the token.  When
+// the bound does not narrow the keys to at most kSelThreads (an adversarial
+// spread, e.g. equal logits everywhere), or passes fewer than min(V, 64) (a
+// histogram left dirty by a call that never reached this kernel), every list
+// is merged instead, 15 at a time into a running best 64: slower, and exact
+// either way.
 __global__ void __launch_bounds__(kSelThreads, 1)
 head_select_kernel(const __grid_constant__ HeadParams p) {
   extern __shared__ __align__(16) unsigned char smem[];
-  hkey* s_mine = reinterpret_cast<hkey*>(smem);            // [ceil(nlists / 8)][64]
-  __shared__ hkey s_part[kHeadCluster][kHeadList];
+  hkey* s_lead = reinterpret_cast<hkey*>(smem);            // [nlists][kLead]; 16 lists when merging
+  __shared__ hkey s_cand[kSelThreads];
   __shared__ hkey s_best[kHeadList];
-  __shared__ hkey s_buf[kSelThreads];
-  __shared__ GatherScratch s_gs;
+  __shared__ float s_r[kHeadList];
+  __shared__ int s_long[kSelThreads];
   __shared__ uint32_t s_wtot[kSelWarps];
   __shared__ uint32_t s_bin;
-  __shared__ hkey s_final[kHeadList];
-  __shared__ float s_r[kHeadList];
-  __shared__ uint32_t s_open, s_bad, s_ok;
-  __shared__ float s_gap;
-  __shared__ __align__(8) uint64_t s_bar;
+  __shared__ int s_nc, s_nlong;
 
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const uint32_t rank = cluster_rank();
-  const int csize = kHeadCluster;
-  const int ks = p.k_sel;
-  const int n8 = (p.nlists + csize - 1) / csize;
-  const int mine = p.nlists > (int)rank ? (p.nlists - (int)rank + csize - 1) / csize : 0;
-  if (threadIdx.x == 0) {
-    mbar_init(&s_bar, 1);
-    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-    s_bad = 0;
-  }
-  __syncthreads();
+  const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
+  const int ks = p.k_sel, nl = p.nlists;
   pdl_launch_dependents();
-  pdl_wait();                                    // every CTA list is written
+  pdl_wait();                                    // every CTA list and count is written
   for (int b = 0; b < p.B; ++b) {
-    uint32_t* hc = p.hist + (int64_t)b * kHistWords;
-    if (threadIdx.x == 0 && mine > 0) {
-      // the previous hidden state's reads and writes of s_mine (generic
-      // proxy) come before this copy's writes (async proxy)
-      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-      const uint32_t bytes = (uint32_t)mine * kHeadList * 8;
-      mbar_arrive_expect_tx(&s_bar, bytes);
-      bulk_load(s_mine, p.lists + (int64_t)(b * csize + (int)rank) * n8 * kHeadList, bytes, &s_bar);
+    const hkey* lists = p.lists + (int64_t)b * nl * kHeadList;
+    for (int l = t; l < nl; l += kSelThreads) {  // the leading keys, 32 bytes per list
+      const ulonglong2* src = reinterpret_cast<const ulonglong2*>(lists + (int64_t)l * kHeadList);
+      const ulonglong2 k01 = __ldcg(src), k23 = __ldcg(src + 1);
+      s_lead[l * kLead] = k01.x;
+      s_lead[l * kLead + 1] = k01.y;
+      s_lead[l * kLead + 2] = k23.x;
+      s_lead[l * kLead + 3] = k23.y;
     }
-    // while the lists arrive, the bound T: the histogram bin holding the
-    // 64th best listed key (every CTA finds it; no key of the final 64 lies
-    // below T)
-    const uint32_t tb = hist_bound(hc, kHeadList, s_wtot, s_bin);
+    if (t == 0) {
+      s_nc = 0;
+      s_nlong = 0;
+    }
+    // the bound (its barriers also complete the stores above)
+    const uint32_t tb = hist_bound(p.hist + (int64_t)b * kHistWords, kHeadList, s_wtot, s_bin);
     const hkey T = tb ? (hkey)tb << 32 : 1ull;   // no bound: every key passes
-    if (threadIdx.x == 0 && mine > 0 && !mbar_wait(&s_bar, (uint32_t)(b & 1))) s_bad = 1;
+    for (int l = t; l < nl; l += kSelThreads) {
+      int n = 0;
+#pragma unroll
+      for (int e = 0; e < kLead; ++e) {
+        const hkey k = s_lead[l * kLead + e];
+        if (k >= T) {
+          const int i = atomicAdd(&s_nc, 1);
+          if (i < kSelThreads) s_cand[i] = k;
+          ++n;
+        }
+      }
+      if (n == kLead) {                          // the list may continue past its leading keys
+        const int j = atomicAdd(&s_nlong, 1);
+        if (j < kSelThreads) s_long[j] = l;
+      }
+    }
     __syncthreads();
-    const int have = s_bad ? 0 : mine;
-    // this CTA's best 64 of its keys >= T (all of them, more than
-    // kSelThreads only for adversarial spreads: then the merge tree)
-    const int C = gather_ge(s_mine, have, T, s_buf, kSelThreads, s_gs);
-    if (C >= 0) {
-      rank_place(s_buf, C, s_best);
+    const int nlong = s_nlong;
+    for (int j = warp; j < min(nlong, kSelThreads); j += kSelWarps) {
+      const hkey* L = lists + (int64_t)s_long[j] * kHeadList;
+      for (int e = kLead + lane; e < kHeadList; e += 32) {
+        const hkey k = __ldcg(L + e);
+        if (k >= T) {
+          const int i = atomicAdd(&s_nc, 1);
+          if (i < kSelThreads) s_cand[i] = k;
+        }
+      }
+    }
+    __syncthreads();
+    const int C = s_nc;
+    if (C <= kSelThreads && nlong <= kSelThreads && C >= min(p.V, kHeadList)) {
+      rank_place(s_cand, C, s_best);
     } else {
-      tree_merge(s_mine, have, kSelWarps);
-      if (threadIdx.x < kHeadList) s_best[threadIdx.x] = s_mine[threadIdx.x];
+      hkey* s16 = s_lead;                        // 16 lists: the running best, then 15 more
+      for (int i = t; i < kHeadList; i += kSelThreads) s16[i] = 0ull;
+      for (int base = 0; base < nl; base += 15) {
+        const int cnt = min(15, nl - base);
+        for (int e = t; e < 15 * kHeadList; e += kSelThreads)
+          s16[kHeadList + e] = e / kHeadList < cnt ? __ldcg(lists + (int64_t)base * kHeadList + e) : 0ull;
+        __syncthreads();
+        tree_merge(s16, 16, kSelWarps);
+      }
+      for (int i = t; i < kHeadList; i += kSelThreads) s_best[i] = s16[i];
       __syncthreads();
     }
-    if (threadIdx.x < kHeadList) st_peer_key(peer_addr(&s_part[rank][threadIdx.x], 0u), s_best[threadIdx.x]);
-    if (threadIdx.x == 0 && s_bad) st_peer_u32(peer_addr(&s_bad, 0u), 1u);
-    cluster_sync();                              // the partial results in CTA 0
-    if (rank == 0) {
-      const int C0 = gather_ge(&s_part[0][0], csize, 1ull, s_buf, kSelThreads, s_gs);
-      rank_place(s_buf, C0, s_best);             // C0 <= 8 * 64 = kSelThreads
-      const hkey* fin = s_best;
-      // The 64 best keys >= T are the 64 best keys when at least min(V, 64)
-      // keys pass T, which holds whenever the histogram counted exactly this
-      // call's listed keys; fewer (a histogram left dirty by a call that
-      // never reached this kernel) or a failed copy: token -1 (the histogram
-      // is cleared at the end either way).
-      const bool ok = s_bad == 0 && C0 >= min(p.V, kHeadList);
-      const float g = __fsub_rn(key_z(fin[0]), key_z(fin[1]));
-      const uint32_t open = ok && g < p.tau ? 1u : 0u;
-      if (threadIdx.x < kHeadList) {
-        const hkey k = fin[threadIdx.x];
-        for (int r = 0; r < csize; ++r) st_peer_key(peer_addr(&s_final[threadIdx.x], (uint32_t)r), k);
-      }
-      if (threadIdx.x == 0) {
-        for (int r = 0; r < csize; ++r) st_peer_u32(peer_addr(&s_open, (uint32_t)r), open);
-        s_ok = ok ? 1u : 0u;
-        s_gap = g;
-      }
-    }
-    // (global stores come after the cluster barriers: a barrier's release
-    // would wait for them)
-    cluster_sync();                              // s_final and s_open everywhere
-    if (s_open && warp < kHeadWarps) {
+    const float g = __fsub_rn(key_z(s_best[0]), key_z(s_best[1]));
+    const bool open = g < p.tau;
+    if (open) {
       const float* hb = p.h + (int64_t)b * p.ldh;
-      for (int i = (int)rank + csize * warp; i < ks; i += csize * kHeadWarps) {
-        const float rv = verify_row(p, hb, key_row(s_final[i]), lane);
-        if (lane == 0) st_peer_u32(peer_addr(&s_r[i], 0u), __float_as_uint(rv));
-      }
-    }
-    cluster_sync();                              // every r in CTA 0
-    if (rank == 0) {
-      if (threadIdx.x == 0) {
-        if (!s_open) p.token[b] = s_ok ? key_row(s_final[0]) : -1;
-        if (p.verified) p.verified[b] = (int)s_open;
-        if (p.gap) p.gap[b] = s_gap;
-      }
-      if (p.cand && (int)threadIdx.x < ks) p.cand[(int64_t)b * ks + threadIdx.x] = key_row(s_final[threadIdx.x]);
-    }
-    if (rank == 0 && s_open && warp == 0) {
-      // largest r, equal r: lower row (starting from candidate 0, so the
-      // token is always a candidate)
-      float br = s_r[0];
-      int bm = key_row(s_final[0]);
+      int rows[4];
+      int n = 0;
 #pragma unroll
-      for (int t = 0; t < 2; ++t) {
-        const int i = lane + 32 * t;
-        if (i < ks) {
-          const float rv = s_r[i];
-          const int m = key_row(s_final[i]);
-          if (rv > br || (rv == br && m < bm)) {
-            br = rv;
-            bm = m;
+      for (int j = 0; j < 4; ++j) {
+        const int i = warp + kSelWarps * j;
+        rows[j] = i < ks ? key_row(s_best[i]) : 0;
+        if (i < ks) n = j + 1;
+      }
+      if (n > 0) {
+        float rv[4];
+        verify_rows4(p, hb, rows, n, lane, rv);
+#pragma unroll
+        for (int j = 0; j < 4; ++j)
+          if (j < n && lane == 0) s_r[warp + kSelWarps * j] = rv[j];
+      }
+      __syncthreads();
+    }
+    if (warp == 0) {
+      int token = key_row(s_best[0]);
+      if (open) {
+        // largest r, equal r: lower row (starting from candidate 0, so the
+        // token is always a candidate)
+        float br = s_r[0];
+        int bm = token;
+#pragma unroll
+        for (int q = 0; q < 2; ++q) {
+          const int i = lane + 32 * q;
+          if (i < ks) {
+            const float rv = s_r[i];
+            const int m = key_row(s_best[i]);
+            if (rv > br || (rv == br && m < bm)) {
+              br = rv;
+              bm = m;
+            }
+            if (p.r) p.r[(int64_t)b * ks + i] = rv;
           }
-          if (p.r) p.r[(int64_t)b * ks + i] = rv;
         }
-      }
 #pragma unroll
-      for (int d = 16; d >= 1; d >>= 1) {
-        const float orv = __shfl_xor_sync(0xffffffffu, br, d);
-        const int om = __shfl_xor_sync(0xffffffffu, bm, d);
-        if (orv > br || (orv == br && om < bm)) {
-          br = orv;
-          bm = om;
+        for (int d = 16; d >= 1; d >>= 1) {
+          const float orv = __shfl_xor_sync(0xffffffffu, br, d);
+          const int om = __shfl_xor_sync(0xffffffffu, bm, d);
+          if (orv > br || (orv == br && om < bm)) {
+            br = orv;
+            bm = om;
+          }
         }
+        token = bm;
       }
-      if (lane == 0) p.token[b] = bm;
+      if (lane == 0) {
+        p.token[b] = token;
+        if (p.verified) p.verified[b] = open ? 1 : 0;
+        if (p.gap) p.gap[b] = g;
+      }
     }
-    // Before the next hidden state rewrites s_mine (bulk copy), s_part,
-    // s_best, s_final, s_open and s_r, every reader of them must be done:
-    // one more barrier.
-    if (b + 1 < p.B) cluster_sync();
+    if (p.cand && t < ks) p.cand[(int64_t)b * ks + t] = key_row(s_best[t]);
+    __syncthreads();                             // s_lead, s_cand, s_best, s_r are rewritten next
   }
-  // every CTA has read the histograms: CTA r clears bins 512 r .. 512 r + 511
-  // of each hidden state's for the next call
-  for (int b = 0; b < p.B; ++b)
-    for (int i = threadIdx.x; i < kHistWords / kHeadCluster; i += kSelThreads)
-      p.hist[(int64_t)b * kHistWords + (int)rank * (kHistWords / kHeadCluster) + i] = 0u;
+  // the histograms are read: clear them for the next call
+  for (int i = t; i < p.B * kHistWords; i += kSelThreads) p.hist[i] = 0u;
 }
 
 int g_head_sms = 0;
@@ -699,24 +643,10 @@ cudaError_t launch_head_t(HeadParams p, cudaStream_t s) {
   e = launch_pdl(head_kernel<B>, dim3((unsigned)grid), dim3(kHeadThreads), smem, s, p);
   if (e != cudaSuccess) return e;
 
-  const size_t sel_smem = (size_t)((grid + kHeadCluster - 1) / kHeadCluster) * kHeadList * 8;
+  const size_t sel_smem = (size_t)(grid * kLead > 16 * kHeadList ? grid * kLead : 16 * kHeadList) * 8;
   e = raise_smem(head_select_kernel, sel_smem, g_select_smem);   // one kernel for every B
   if (e != cudaSuccess) return e;
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(kHeadCluster, 1, 1);
-  cfg.blockDim = dim3(kSelThreads, 1, 1);
-  cfg.dynamicSmemBytes = sel_smem;
-  cfg.stream = s;
-  cudaLaunchAttribute attr[2];
-  attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = kHeadCluster;
-  attr[0].val.clusterDim.y = 1;
-  attr[0].val.clusterDim.z = 1;
-  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[1].val.programmaticStreamSerializationAllowed = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = 2;
-  return cudaLaunchKernelEx(&cfg, head_select_kernel, p);
+  return launch_pdl(head_select_kernel, dim3(1), dim3(kSelThreads), sel_smem, s, p);
 }
 
 }  // namespace

@@ -219,3 +219,25 @@ def test_head_errors():
     small = sp.Head(Qd[:5], sd[:5], K=K)
     assert lib.spike_proj_head(small.handle, hd.data_ptr(), 64, 1, 0.5, 6, tok.data_ptr(), None,
                                None, None, None, None, 0, None) == sp.SP_EINVAL   # k_sel > V
+
+
+@pytest.mark.parametrize("V,K", [(3000, 256), (57344, 1536)])
+def test_head_equal_logits(V, K):
+    """A zero hidden state makes every approximate logit 0: the histogram
+    bound passes every listed key, so the selection merges every list (the
+    exact slow path). Candidates are then the lowest rows, the gap is 0 and
+    the recomputed logits are all 0."""
+    if V == 57344:
+        Q, s, Qd, sd = full_head()
+    else:
+        Q, s = small_case(8, V, K)
+        Qd, sd = to_dev(Q), to_dev(s)
+    head = sp.Head(Qd, sd, K=K)
+    h = np.zeros((2, K), np.float32)
+    got = run_head(head, h, 0.5, 64, V)
+    check(got, Q, s, V, K, h, 0.5, 64, f"equal logits V={V}")
+    assert np.array_equal(got["cand"][0], np.arange(64))
+    assert got["token"][0] == 0 and got["gap"][0] == 0.0
+    # and the call after it is fast-path again and right
+    h2 = synth.head_hidden(7, B=2, K=K)
+    check(run_head(head, h2, 0.5, 64, V), Q, s, V, K, h2, 0.5, 64, "after equal logits")
