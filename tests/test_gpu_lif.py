@@ -21,11 +21,14 @@ def lif_gpu(vd, Id, K, beta, theta, bits_d):
     torch.cuda.synchronize()
 
 
-@pytest.mark.parametrize("K,rows", [(1, 1), (31, 3), (32, 2), (33, 5), (1000, 7), (6144, 44),
-                                    (6161, 3)])
-def test_lif_steps_bit_exact(K, rows):
+@pytest.mark.parametrize("K,rows", [(1, 1), (31, 3), (32, 2), (33, 5), (127, 2), (129, 3),
+                                    (1000, 7), (6144, 44), (6161, 3)])
+@pytest.mark.parametrize("vector", [False, True])
+def test_lif_steps_bit_exact(K, rows, vector):
+    """ld = K + 5 takes the scalar form; ld a multiple of 4 (16-byte rows)
+    the vector form."""
     rng = synth.rng_for(820, K, rows)
-    ld = K + 5
+    ld = (K + 3) // 4 * 4 + (4 if K % 4 == 0 else 0) if vector else K + 5
     words = (K + 31) // 32
     v = rng.normal(0.0, 1.0, (rows, ld)).astype(np.float32)
     v[:, K:] = 7.0                                     # row padding: never touched
@@ -41,6 +44,22 @@ def test_lif_steps_bit_exact(K, rows):
         assert np.array_equal(got_v.view(np.uint32), v.view(np.uint32)), f"v differs at step {step}"
         assert np.array_equal(got_bits[:, :words], want_bits), f"bits differ at step {step}"
         assert np.all(got_bits[:, words:] == 0x5A5A5A5A), "wrote past ceil(K/32) words"
+
+
+def test_lif_large_state_vector():
+    """The vector form on a 64-row x 65536-neuron state (the bench's stream
+    shape, scaled down), several steps."""
+    K, rows = 65536, 64
+    rng = synth.rng_for(822)
+    v = rng.normal(0.0, 1.0, (rows, K)).astype(np.float32)
+    I = rng.normal(0.2, 0.8, (rows, K)).astype(np.float32)
+    vd, Id = to_dev(v), to_dev(I)
+    bits_d = torch.zeros((rows, K // 32), dtype=torch.int32, device=DEV)
+    for step in range(3):
+        v, want_bits = oracle.lif(v, I, K, 0.9, 1.0)
+        lif_gpu(vd, Id, K, 0.9, 1.0, bits_d)
+        assert np.array_equal(vd.cpu().numpy().view(np.uint32), v.view(np.uint32)), step
+        assert np.array_equal(bits_d.cpu().numpy().view(np.uint32), want_bits), step
 
 
 def test_lif_special_values():
