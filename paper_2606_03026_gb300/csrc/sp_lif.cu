@@ -13,7 +13,8 @@
 // updates neuron 32 w + l (coalesced 128-byte reads and writes of v and I)
 // and the warp's ballot is spike word w; bits at or past K are 0.  Rows
 // whose elements are 16-byte aligned (v, I 16-byte aligned, ld % 4 == 0) take
-// a vector form: lane l holds neurons 4l .. 4l + 3 of a 128-neuron group (one
+// a vector form when the state is large (at least 2^22 neurons): lane l
+// holds neurons 4l .. 4l + 3 of a 128-neuron group (one
 // 16-byte load of v and of I, two groups in flight per lane), and the group's
 // 4 spike words are assembled from 4 ballots (bit j of ballot c, for lane
 // 8w + j, is neuron 32w + 4j + c).  The state
@@ -165,8 +166,12 @@ cudaError_t launch_lif_params(const LifParams& p, cudaStream_t s) {
     e = cudaDeviceGetAttribute(&g_lif_sms, cudaDevAttrMultiProcessorCount, dev);
     if (e != cudaSuccess) return e;
   }
-  const bool vec = !p.per_row && p.ld % 4 == 0 && ((uintptr_t)p.vin & 15) == 0 &&
-                   ((uintptr_t)p.vout & 15) == 0 && ((uintptr_t)p.I & 15) == 0;
+  // the vector form for large states only: at decode sizes (a few hundred
+  // thousand neurons) its small grid made the following decode launch start
+  // later (producer + decode step 16.2 against 14.7 us with the scalar form)
+  const bool vec = !p.per_row && (int64_t)p.rows * p.K >= ((int64_t)1 << 22) && p.ld % 4 == 0 &&
+                   ((uintptr_t)p.vin & 15) == 0 && ((uintptr_t)p.vout & 15) == 0 &&
+                   ((uintptr_t)p.I & 15) == 0;
   const int64_t total_warps =
       vec ? ((int64_t)p.rows * ((p.K + 127) / 128) + 1) / 2 : (int64_t)p.rows * ((p.K + 31) / 32);
   const int64_t need = (total_warps + kLifThreads / 32 - 1) / (kLifThreads / 32);
