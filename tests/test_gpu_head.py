@@ -96,12 +96,14 @@ def check(got, Q, s, V, K, h, tau, k_sel, what):
             assert got["token"][b] == tb, f"{what}: token differs where the exact logits decide"
 
 
-@pytest.mark.parametrize("V,K", [(5001, 1000), (4096, 1536), (999, 40), (70, 512), (2, 16)])
+@pytest.mark.parametrize("V,K", [(5001, 1000), (4096, 1536), (999, 40), (70, 512), (2, 16),
+                                 (1500, 2048), (1200, 2049), (1000, 8192)])
 @pytest.mark.parametrize("B", [1, 2, 4])
 def test_head_vs_oracle(V, K, B):
     Q, s = small_case(1, V, K)
     head = sp.Head(to_dev(Q), to_dev(s), K=K)
-    h = synth.rng_for(7801, V, K, B).standard_normal((B, K + 4)).astype(np.float32)
+    # row pitch a multiple of 4 floats past K (the API's rule for h)
+    h = synth.rng_for(7801, V, K, B).standard_normal((B, (K + 3) // 4 * 4 + 4)).astype(np.float32)
     for tau in (0.0, 0.5, np.inf):
         for k_sel in sorted({1, min(16, V), min(64, V)}):
             got = run_head(head, h, tau, k_sel, V)
