@@ -360,13 +360,15 @@ constexpr int kClusterLoads = 9;                   // column loads per lane in r
 constexpr int kClusterSlots = 8;                   // and in shared memory
 using ClusterSmem = UnitSmem<kGatherClusterWarps, kGatherClusterMaxCK, kClusterSlots>;
 
-template <int NP>
+// kLif: the fused spike producer (a separate instantiation, so that the plain
+// decode carries none of its code)
+template <int NP, bool kLif>
 __global__ void __launch_bounds__(kGatherClusterThreads, 4)
 gather_cluster_kernel(const __grid_constant__ GatherParamsT<NP> p) {
   __shared__ ClusterSmem sm;
   // [sender chunk][owned group]: kch * ceil(128 / kch) < 128 + kch entries
   __shared__ __align__(16) int4 s_recv[kGatherNT / 4 + kGatherCluster];
-  __shared__ uint32_t s_lif[kGatherClusterMaxCK / 32];   // LIF mode: this chunk's spike words
+  __shared__ uint32_t s_lif[kLif ? kGatherClusterMaxCK / 32 : 1];   // LIF mode: the chunk's spike words
   // every CTA of the cluster arrives here and waits (below) before its first
   // store into a peer's shared memory: the peer is then known to be running
   asm volatile("barrier.cluster.arrive.relaxed;" ::: "memory");
@@ -394,8 +396,7 @@ gather_cluster_kernel(const __grid_constant__ GatherParamsT<NP> p) {
   const int n0 = (cl * P.tpc + ts) * kGatherNT;
   const bool work = n0 < P.N;               // tile slots past the last tile idle
   if (work) {
-    const bool lif = p.lif_I != nullptr;
-    if (lif) {
+    if constexpr (kLif) {
       // fused spike producer: one LIF step of this chunk's neurons (every CTA
       // of the chunk computes the same words from the old state; the CTA of
       // tile slot 0 in cluster 0 writes the new state and the bits)
@@ -421,8 +422,8 @@ gather_cluster_kernel(const __grid_constant__ GatherParamsT<NP> p) {
       __syncthreads();
     }
     unit_partial<kGatherClusterWarps, kGatherClusterMaxCK, kClusterLoads, kClusterSlots>(
-        sm, P, lif ? nullptr : spike_row(p.spikes, p.fmt, j, p.ld_spikes), p.fmt, n0, kc * P.ck,
-        P.ck, lif ? s_lif : nullptr);
+        sm, P, kLif ? nullptr : spike_row(p.spikes, p.fmt, j, p.ld_spikes), p.fmt, n0, kc * P.ck,
+        P.ck, kLif ? s_lif : nullptr);
     asm volatile("barrier.cluster.wait;" ::: "memory");
     const int g = threadIdx.x;              // the 4-channel group of this thread
     if (g < kGatherNT / 4) {
@@ -466,7 +467,7 @@ cudaError_t set_carveout(Kern kernel, std::atomic<uint64_t>& done) {
 }
 
 // Clusters of the cluster form that can be resident at once (per device).
-template <int NP>
+template <int NP, bool kLif>
 int cluster_capacity() {
   static std::atomic<int> cap[64];
   int dev = 0;
@@ -483,7 +484,8 @@ int cluster_capacity() {
   cfg.blockDim = dim3(kGatherClusterThreads, 1, 1);
   cfg.attrs = &attr;
   cfg.numAttrs = 1;
-  if (cudaOccupancyMaxActiveClusters(&n, gather_cluster_kernel<NP>, &cfg) != cudaSuccess || n < 1) {
+  if (cudaOccupancyMaxActiveClusters(&n, gather_cluster_kernel<NP, kLif>, &cfg) != cudaSuccess ||
+      n < 1) {
     (void)cudaGetLastError();
     n = -1;
   }
@@ -518,7 +520,7 @@ bool cluster_form(GatherParamsT<NP>& q, int* grid_x, int* grid_y) {
     total += P.ncl;
     if (P.ncl > widest) widest = P.ncl;
   }
-  if (total > cluster_capacity<NP>()) return false;
+  if (total > (q.lif_I ? cluster_capacity<NP, true>() : cluster_capacity<NP, false>())) return false;
   q.ncl_list = 0;
   if (total <= kGatherMaxClusterList && widest <= 0xff) {
     int c = 0;
@@ -536,10 +538,11 @@ bool cluster_form(GatherParamsT<NP>& q, int* grid_x, int* grid_y) {
 
 template <int NP>
 cudaError_t launch_gather_t(const GatherParamsT<NP>& p, cudaStream_t s) {
-  static std::atomic<uint64_t> carve_t{0}, carve_c{0};
+  static std::atomic<uint64_t> carve_t{0}, carve_c{0}, carve_l{0};
   if (p.units_total <= 0 || p.B <= 0 || p.max_units <= 0) return cudaSuccess;
   // the carveout first: the resident-cluster count depends on it
-  cudaError_t e = set_carveout(gather_cluster_kernel<NP>, carve_c);
+  cudaError_t e = p.lif_I ? set_carveout(gather_cluster_kernel<NP, true>, carve_l)
+                          : set_carveout(gather_cluster_kernel<NP, false>, carve_c);
   if (e != cudaSuccess) return e;
   GatherParamsT<NP> q = p;
   int gx = 0, gy = 0;
@@ -559,7 +562,8 @@ cudaError_t launch_gather_t(const GatherParamsT<NP>& p, cudaStream_t s) {
     attr[1].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 2;
-    return cudaLaunchKernelEx(&cfg, gather_cluster_kernel<NP>, q);
+    return p.lif_I ? cudaLaunchKernelEx(&cfg, gather_cluster_kernel<NP, true>, q)
+                   : cudaLaunchKernelEx(&cfg, gather_cluster_kernel<NP, false>, q);
   }
   e = set_carveout(gather_kernel<NP>, carve_t);
   if (e != cudaSuccess) return e;
