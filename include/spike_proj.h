@@ -20,6 +20,13 @@
  * measured density makes that cheaper.  Every path produces the same INT32
  * accumulators bit for bit, and therefore the same FP32 outputs.
  *
+ * Around the projection the library also has the paper's continuous-input
+ * projection (spike_proj_dense: row-major INT8 weights, FP32 activations),
+ * a spike producer (spike_proj_lif, and spike_proj_group_decode_lif with the
+ * producer inside the decode launch), and the vocabulary head with INT8
+ * activations and FP32 recomputation of the top candidates (spike_proj_head,
+ * Section 5).  Each is documented at its declaration below.
+ *
  * Conventions for every call
  *   - Pointers named d_* or documented as "device" are CUDA device pointers
  *     on the current device; the caller owns them.  A plan BORROWS W and the
