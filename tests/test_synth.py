@@ -68,3 +68,30 @@ def test_seeded_reproducible():
     c = synth.single_projection(1)
     assert np.array_equal(a["Q"], b["Q"]) and np.array_equal(a["x"], b["x"])
     assert not np.array_equal(a["x"], c["x"])
+
+
+def test_head_inputs():
+    """The vocabulary head's stand-in weights: row-major [V, K] INT8 with the
+    Section 2.3 export (every row reaches +-127 at its largest magnitude),
+    logits of about the stated spread, seeded and reproducible."""
+    Q, s = synth.head_weights(V=4096, K=1536)
+    assert Q.shape == (4096, 1536) and Q.dtype == np.int8 and s.shape == (4096,)
+    assert np.all(np.abs(Q.astype(np.int16)).max(axis=1) == 127)
+    Q2, s2 = synth.head_weights(V=4096, K=1536)
+    assert np.array_equal(Q, Q2) and np.array_equal(s, s2)
+    h = synth.head_hidden(0, B=64)
+    z = (Q.astype(np.float64) * s[:, None]) @ h.T.astype(np.float64)
+    assert abs(z.std() - synth.HEAD_LOGIT_STD) < 0.2 * synth.HEAD_LOGIT_STD
+    assert not np.array_equal(synth.head_hidden(0), synth.head_hidden(1))
+
+
+def test_dense_inputs():
+    """Continuous-input stand-ins: row-major weights of the stated shapes with
+    the per-row export, and N(0, 1) hidden states."""
+    for kind, N in synth.DENSE_KINDS.items():
+        W, s = synth.dense_weights(0, kind)
+        assert W.shape == (N, synth.D_MODEL) and W.dtype == np.int8 and s.shape == (N,)
+        assert np.all(np.abs(W.astype(np.int16)).max(axis=1) == 127)
+    x = synth.hidden_state(0, B=4)
+    assert x.shape == (4, synth.D_MODEL) and x.dtype == np.float32
+    assert abs(float(x.std()) - 1.0) < 0.05
