@@ -195,16 +195,14 @@ __device__ void rank_place(const hkey* buf, int C, hkey* out) {
 }
 
 // The lower bound of the leading order bits of the histogram bin that holds
-// the need-th largest key, from a kHistWords-bin histogram in global memory
-// (bin i counts the keys whose leading bits are i): thread t of a
-// kSelThreads-thread CTA reads bins 8t .. 8t + 7, and the suffix sums meet in
-// two barriers.  0 when the histogram holds fewer than need keys.  Every
-// thread calls it.
-__device__ uint32_t hist_bound(const uint32_t* h, uint32_t need, uint32_t* s_wtot, uint32_t& s_bin) {
+// the need-th largest key, from a kHistWords-bin histogram (bin i counts the
+// keys whose leading bits are i): thread t of a kSelThreads-thread CTA holds
+// bins 8t .. 8t + 7 in c (loaded by the caller, so that the loads can be in
+// flight with others), and the suffix sums meet in two barriers.  0 when
+// the histogram holds fewer than need keys.  Every thread calls it.
+__device__ uint32_t hist_bound(const uint32_t (&c)[8], uint32_t need, uint32_t* s_wtot,
+                               uint32_t& s_bin) {
   const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
-  const uint4 q0 = __ldcg(reinterpret_cast<const uint4*>(h) + 2 * t);
-  const uint4 q1 = __ldcg(reinterpret_cast<const uint4*>(h) + 2 * t + 1);
-  const uint32_t c[8] = {q0.x, q0.y, q0.z, q0.w, q1.x, q1.y, q1.z, q1.w};
   uint32_t sum = 0;
 #pragma unroll
   for (int i = 0; i < 8; ++i) sum += c[i];
@@ -487,7 +485,21 @@ head_select_kernel(const __grid_constant__ HeadParams p) {
   pdl_wait();                                    // every CTA list and count is written
   for (int b = 0; b < p.B; ++b) {
     const hkey* lists = p.lists + (int64_t)b * nl * kHeadList;
-    for (int l = t; l < nl; l += kSelThreads) {  // the leading keys, 32 bytes per list
+    // one round of loads: this thread's 8 histogram bins and the leading keys
+    // (32 bytes) of lists t and t + kSelThreads
+    const uint4* hq = reinterpret_cast<const uint4*>(p.hist + (int64_t)b * kHistWords) + 2 * t;
+    const uint4 h0 = __ldcg(hq), h1 = __ldcg(hq + 1);
+    ulonglong2 lead[2][2];
+#pragma unroll
+    for (int q = 0; q < 2; ++q) {
+      const int l = t + q * kSelThreads;
+      if (l < nl) {
+        const ulonglong2* src = reinterpret_cast<const ulonglong2*>(lists + (int64_t)l * kHeadList);
+        lead[q][0] = __ldcg(src);
+        lead[q][1] = __ldcg(src + 1);
+      }
+    }
+    for (int l = t + 2 * kSelThreads; l < nl; l += kSelThreads) {   // more than 1024 lists: never
       const ulonglong2* src = reinterpret_cast<const ulonglong2*>(lists + (int64_t)l * kHeadList);
       const ulonglong2 k01 = __ldcg(src), k23 = __ldcg(src + 1);
       s_lead[l * kLead] = k01.x;
@@ -495,12 +507,23 @@ head_select_kernel(const __grid_constant__ HeadParams p) {
       s_lead[l * kLead + 2] = k23.x;
       s_lead[l * kLead + 3] = k23.y;
     }
+#pragma unroll
+    for (int q = 0; q < 2; ++q) {
+      const int l = t + q * kSelThreads;
+      if (l < nl) {
+        s_lead[l * kLead] = lead[q][0].x;
+        s_lead[l * kLead + 1] = lead[q][0].y;
+        s_lead[l * kLead + 2] = lead[q][1].x;
+        s_lead[l * kLead + 3] = lead[q][1].y;
+      }
+    }
     if (t == 0) {
       s_nc = 0;
       s_nlong = 0;
     }
     // the bound (its barriers also complete the stores above)
-    const uint32_t tb = hist_bound(p.hist + (int64_t)b * kHistWords, kHeadList, s_wtot, s_bin);
+    const uint32_t hc[8] = {h0.x, h0.y, h0.z, h0.w, h1.x, h1.y, h1.z, h1.w};
+    const uint32_t tb = hist_bound(hc, kHeadList, s_wtot, s_bin);
     const hkey T = tb ? (hkey)tb << 32 : 1ull;   // no bound: every key passes
     for (int l = t; l < nl; l += kSelThreads) {
       int n = 0;
