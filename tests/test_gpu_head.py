@@ -243,3 +243,20 @@ def test_head_equal_logits(V, K):
     # and the call after it is fast-path again and right
     h2 = synth.head_hidden(7, B=2, K=K)
     check(run_head(head, h2, 0.5, 64, V), Q, s, V, K, h2, 0.5, 64, "after equal logits")
+
+
+def test_head_codes_at_exact_halves():
+    """Hidden values whose quotient by s_x is exactly an integer plus one half
+    (s_x a power of two): the codes round half to even as IEEE division
+    does, so the approximate logits match the oracle bit for bit."""
+    V, K = 512, 1024
+    Q, s = small_case(9, V, K)
+    rng = synth.rng_for(7809)
+    q = rng.integers(-126, 127, size=(2, K)).astype(np.float64) + 0.5
+    q[:, 0] = 127.0
+    q[1, 0] = -127.0
+    q[:, 1::7] = np.round(q[:, 1::7])                # some exact integers too
+    h = (q * 2.0 ** -5).astype(np.float32)          # s_x = 127 * 2^-5 / 127 = 2^-5 exactly
+    head = sp.Head(to_dev(Q), to_dev(s), K=K)
+    got = run_head(head, h, np.inf, 16, V)
+    check(got, Q, s, V, K, h, np.inf, 16, "exact halves")
