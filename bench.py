@@ -1014,9 +1014,13 @@ def bench_dense(torch, sp, synth, dev, stream, peaks, peak_kind, world, blocks=2
 
 
 def bench_prefill(torch, sp, synth, dev, stream, peaks, peak_kind, world, blocks=22):
-    """512-token prefill over the decoder's blocks: one tensor-core GEMM
-    launch per block, graph-captured.  The spike blocks are 0/1 bytes
-    (torch.bool, SP_SPIKES_BOOL8), which the GEMM reads in place."""
+    """512-token prefill over the decoder's blocks, graph-captured, two ways:
+    grouped (spike_proj_group_prefill: every block's output tiles in ONE
+    persistent tensor-core launch) and per block (one spike_proj_batched
+    SP_GEMM call per block, 22 launches).  The spike blocks are 0/1 bytes
+    (torch.bool, SP_SPIKES_BOOL8), which the GEMM reads in place.  The 22
+    blocks are independent here (synthetic spikes per block), as the decode
+    step's projections are."""
     import oracle
     T, N, K = 512, 1536, 6144
     plans, Xs, outs = [], [], []
@@ -1040,41 +1044,67 @@ def bench_prefill(torch, sp, synth, dev, stream, peaks, peak_kind, world, blocks
     ra, _ = oracle.project(Q0, s0, N, K, X0[rows], "u8")
     assert np.array_equal(outs[0][0].cpu().numpy()[rows], ra), "prefill spot check failed"
 
-    g = torch.cuda.CUDAGraph()
-    with torch.cuda.graph(g, stream=stream):
+    def timed(fn, reps=20):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            fn(torch.cuda.current_stream())
+        with torch.cuda.stream(stream):
+            for _ in range(3):
+                g.replay()
+        stream.synchronize()
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        with torch.cuda.stream(stream):
+            e0.record(stream)
+            for _ in range(reps):
+                g.replay()
+            e1.record(stream)
+        stream.synchronize()
+        return e0.elapsed_time(e1) / reps
+
+    def per_block(st):
         for b in range(blocks):
-            plans[b].batched(Xs[b], "bool8", T, K, outs[b][0], outs[b][1], chosen,
-                             stream=torch.cuda.current_stream())
-    with torch.cuda.stream(stream):
-        for _ in range(3):
-            g.replay()
-    stream.synchronize()
-    reps = 20
-    e0 = torch.cuda.Event(enable_timing=True)
-    e1 = torch.cuda.Event(enable_timing=True)
-    with torch.cuda.stream(stream):
-        e0.record(stream)
-        for _ in range(reps):
-            g.replay()
-        e1.record(stream)
-    stream.synchronize()
-    ms = e0.elapsed_time(e1) / reps
+            plans[b].batched(Xs[b], "bool8", T, K, outs[b][0], outs[b][1], chosen, stream=st)
+
+    group = sp.Group(plans)
+    g_acc = [torch.empty(T, N, dtype=torch.int32, device=dev) for _ in range(blocks)]
+    g_y = [torch.empty(T, N, dtype=torch.float32, device=dev) for _ in range(blocks)]
+
+    def grouped(st):
+        group.prefill(Xs, "bool8", T, K, g_acc, g_y, stream=st)
+
+    ms_chain = timed(per_block)
+    ms = timed(grouped)
+    # the grouped launch gives the per-block results bit for bit
+    same = all(torch.equal(outs[b][0], g_acc[b]) and
+               torch.equal(outs[b][1].view(torch.int32), g_y[b].view(torch.int32))
+               for b in range(blocks))
+    assert same, "grouped prefill differs from the per-block calls"
     ops = 2.0 * T * N * K * blocks
     tops = ops / (ms * 1e-3) / 1e12
+    tops_chain = ops / (ms_chain * 1e-3) / 1e12
     # the contraction runs in e4m3: its peak is the measured bf16 peak times
     # the nominal fp8 / bf16 ratio (2); each weight takes two e4m3 MACs (the
     # 16 h and l planes), so this path's own ceiling is half of that
     peak = 2.0 * float(peaks.get("bf16_tflops", 1900.0))
     dens = float(np.mean([x.float().mean().item() for x in Xs]))
+    group.close()
     for p in plans:
         p.close()
     return {"value": tops * world, "unit": "TOPS", "blocks": blocks, "ms_per_prefill": ms,
             "prefill_tokens_per_s": T / (ms * 1e-3) * world, "chosen_kernel": chosen,
+            "form": "grouped: spike_proj_group_prefill, one gemm_group_kernel launch over "
+                    f"{blocks} x 24 output tiles of 128 x 256, whole K per tile",
+            "per_block": {"ms_per_prefill": ms_chain, "tops": tops_chain,
+                          "frac_of_two_plane_cap": tops_chain / (peak / 2),
+                          "form": f"{blocks} spike_proj_batched SP_GEMM launches (split-K "
+                                  "clusters), one per block"},
             "mean_density": dens, "ops": "2*T*N*K dense-equivalent int8 ops per block",
             "spike_format": "bool8 (0/1 bytes, read in place by the GEMM)",
             "roofline": {"bound": "tensor", "achieved": tops, "peak": peak, "unit": "TFLOP/s",
                          "frac": tops / peak, "frac_of_two_plane_cap": tops / (peak / 2),
-                         "traffic": measured_traffic("gemm_kernel", "sp_gemm.cu"),
+                         "traffic": measured_traffic("gemm_group_kernel", "sp_gemm.cu"),
+                         "kernel": "gemm_group_kernel",
                          "peak_kind": peak_kind + " bf16 burst x 2 (fp8 e4m3 nominal ratio)",
                          "note": "sm_103a has no tcgen05 kind::i8; e4m3 x e4m3 (spikes 0/2^-9, "
                                  "weights as 16h + l planes), fp32 accumulate, exact"}}

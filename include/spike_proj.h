@@ -239,6 +239,35 @@ sp_status spike_proj_group_decode(sp_group_t group, const void *spikes,
                                   sp_fmt fmt, int64_t ld_spikes, int32_t *acc,
                                   float *y, int64_t ld_out, sp_stream_t stream);
 
+/* spike_proj_group_prefill: T spike rows per member through the dense
+ * tensor-core contraction of spike_proj_prefill (SP_GEMM), ACC_j = X_j Q_j^T
+ * and Y_j = ACC_j * s_j per column (Eq. (sparse) for every row, Section 3.2's
+ * 512-token prefill), for EVERY member of the group in ONE persistent launch:
+ * the output tiles of all members (128 rows x 256 channels each) are shared
+ * out over the SMs, and each tile runs over its whole K.  The members are
+ * independent; nothing of member j reaches member i.  Results equal
+ * spike_proj_prefill / spike_proj_batched on each member's plan, bit for bit.
+ *
+ *   X     host array of `count` device pointers; member j's rows at
+ *         X[j] + t*ldx (t < T; words for BITS32, bytes for U8 and BOOL8).
+ *         BOOL8 rows with a 16-byte aligned base and ldx % 16 == 0 are read
+ *         in place; other rows go first through a 0/1 staging pass into the
+ *         member plan's staging copy (one small launch per member).
+ *   T     1 <= T <= every member plan's max_batch (else SP_ERANGE).
+ *   ldx   row stride; ldx >= ceil(K_j/32) words (BITS32) or K_j bytes.
+ *   acc   host array of `count` device pointers, member j's INT32 [T][N_j]
+ *         row-major at acc[j], or NULL for no acc;
+ *   y     likewise FP32 [T][N_j] (acc and y not both NULL).
+ * Every member plan must have been made with SP_PLAN_GEMM (else
+ * SP_EUNSUPPORTED).  The group's error word records a kernel fault
+ * (spike_proj_group_status).  Errors: SP_EINVAL, SP_EALIGN, SP_ERANGE,
+ * SP_EUNSUPPORTED, SP_ENOMEM (the member table, allocated on the host by the
+ * first call), SP_ECUDA. */
+sp_status spike_proj_group_prefill(sp_group_t group, const void *const *X,
+                                   sp_fmt fmt, int32_t T, int64_t ldx,
+                                   int32_t *const *acc, float *const *y,
+                                   sp_stream_t stream);
+
 /* spike_proj_group_decode_host: the same with HOST buffers.  Page-locked
  * buffers (cudaHostAlloc, cudaHostRegister, torch pin_memory) are read and
  * written by the kernel in place, over the CPU-GPU link, with no copy; for

@@ -72,6 +72,14 @@ struct sp_group_s {
   int32_t* d_acc = nullptr;       // [count][maxN]
   float* d_y = nullptr;           // [count][maxN]
   size_t spike_row_bytes = 0;
+  // grouped prefill (every plan made with SP_PLAN_GEMM): the launch's member
+  // table, and per member the caller's 0/1 rows of the last in-place call
+  sp_plan_s* plans[kMaxProblems] = {};
+  GemmGroupArgs* gemm = nullptr;
+  const void* rows_ptr[kMaxProblems] = {};
+  int64_t rows_ld[kMaxProblems] = {};
+  int32_t rows_T[kMaxProblems] = {};
+  CUtensorMap rows_map[kMaxProblems];
 };
 
 namespace {
@@ -137,6 +145,7 @@ void plan_free(sp_plan_s* p) {
 
 void group_free(sp_group_s* g) {
   if (!g) return;
+  delete g->gemm;
   cudaFree(g->ws);
   cudaFree(g->tickets);
   cudaFree(g->err);
@@ -471,7 +480,8 @@ sp_status spike_proj_group_create(sp_group_t* group, const sp_plan_t* plans, int
   std::memset(&g->params, 0, sizeof(g->params));
   int64_t units = 0, ws = 0, tk = 0;
   for (int j = 0; j < count; ++j) {
-    const sp_plan_s* p = plans[j];
+    sp_plan_s* p = plans[j];
+    g->plans[j] = p;
     GatherProblem& P = g->params.prob[j];
     P.W = p->W;
     P.scale = p->scale;
@@ -542,6 +552,68 @@ sp_status spike_proj_group_decode(sp_group_t g, const void* spikes, sp_fmt fmt, 
   P.y = y;
   P.ld_out = ld_out;
   SP_CUDA(launch_gather(P, as_stream(stream)));
+  return SP_OK;
+}
+
+sp_status spike_proj_group_prefill(sp_group_t g, const void* const* X, sp_fmt fmt, int32_t T,
+                                   int64_t ldx, int32_t* const* acc, float* const* y,
+                                   sp_stream_t stream) {
+  if (!g || !X || !fmt_ok(fmt) || T < 1 || (!acc && !y)) return SP_EINVAL;
+  for (int j = 0; j < g->count; ++j) {
+    const sp_plan_s* p = g->plans[j];
+    if (!(p->flags & SP_PLAN_GEMM)) return SP_EUNSUPPORTED;
+    if (T > p->max_batch) return SP_ERANGE;
+    if (!X[j] || (acc && !acc[j]) || (y && !y[j])) return SP_EINVAL;
+    if (ldx < row_elems(fmt, p->K)) return SP_EINVAL;
+    if (fmt == SP_SPIKES_BITS32 && !aligned(X[j], 4)) return SP_EALIGN;
+    if ((acc && !aligned(acc[j], 4)) || (y && !aligned(y[j], 4))) return SP_EALIGN;
+  }
+  if (!g->gemm) {
+    g->gemm = new (std::nothrow) GemmGroupArgs();
+    if (!g->gemm) return SP_ENOMEM;
+  }
+  cudaStream_t s = as_stream(stream);
+  GemmGroupArgs& a = *g->gemm;
+  a.count = g->count;
+  a.err = g->err;
+  int64_t units = 0;
+  // 0/1 byte rows that TMA can address are read in place; any other input
+  // is first written as 0/1 bytes into the member plan's staging copy
+  const bool vec = fmt == SP_SPIKES_BOOL8 && ldx % 16 == 0;
+  for (int j = 0; j < g->count; ++j) {
+    sp_plan_s* p = g->plans[j];
+    GemmMember& M = a.m[j];
+    if (vec && aligned(X[j], 16)) {
+      if (X[j] != g->rows_ptr[j] || ldx != g->rows_ld[j] || T != g->rows_T[j]) {
+        SP_CUDA(gemm_make_rows_map(X[j], ldx, T, p->K, &g->rows_map[j]));
+        g->rows_ptr[j] = X[j];
+        g->rows_ld[j] = ldx;
+        g->rows_T[j] = T;
+      }
+      M.a = g->rows_map[j];
+    } else {
+      SP_CUDA(launch_spikes_to_01(X[j], fmt, ldx, T, p->K, p->Kp, p->Xs, s));
+      M.a = p->maps.a;
+    }
+    M.b = p->maps.b;
+    M.p.scale = p->scale;
+    M.p.acc = acc ? acc[j] : nullptr;
+    M.p.y = y ? y[j] : nullptr;
+    M.p.T = T;
+    M.p.N = p->N;
+    M.p.K = p->K;
+    M.p.err = g->err;
+    M.p.part = nullptr;
+    M.p.part_units = 0;
+    M.tiles_n = ceil_div(p->N, 256);
+    M.nkb = p->Kp / 64;
+    M.unit_begin = (int32_t)units;
+    units += (int64_t)ceil_div(T, 128) * M.tiles_n;
+    if (units > INT32_MAX) return SP_ERANGE;
+    M.unit_end = (int32_t)units;
+  }
+  a.units = (int32_t)units;
+  SP_CUDA(launch_gemm_group(a, s));
   return SP_OK;
 }
 

@@ -486,6 +486,190 @@ gemm_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CU
   }
 }
 
+// ---- grouped persistent launch ------------------------------------------------
+//
+// The output tiles of every member of a group (e.g. the 22 down projections
+// of a 512-token prefill: 22 x 4 x 6 = 528 tiles of 128 x 256) form one list,
+// member after member; CTA b of a grid of min(tiles, SMs) takes tiles b,
+// b + grid, ...  Each tile runs over its whole K, so no partial leaves the
+// SM: the producer / MMA pipeline is the one of gemm_kernel, and the
+// epilogue of tile i (8 warps: TMEM lane quarter w % 4, 16-column half
+// (w - 2) / 4 of every 32-column chunk) overlaps the MMAs of tile i + 1
+// through the double-buffered accumulator.
+
+// Member holding output tile u (members are few, their tile ranges ascending).
+__device__ __forceinline__ int member_of(const GemmGroupArgs& g, int u) {
+  int j = 0;
+  while (j + 1 < g.count && u >= g.m[j].unit_end) ++j;
+  return j;
+}
+
+__global__ void __launch_bounds__(kGemmThreads, 1)
+gemm_group_kernel(const __grid_constant__ GemmGroupArgs g) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  uint8_t* sA = smem;
+  uint8_t* sB = smem + (size_t)STAGES * A_BYTES;
+  uint32_t* s_tr = reinterpret_cast<uint32_t*>(smem + SMEM_RING);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + SMEM_RING + SMEM_TR);
+  uint64_t* full = bars;                 // [STAGES] TMA -> MMA
+  uint64_t* empty = bars + STAGES;       // [STAGES] MMA -> TMA
+  uint64_t* tfull = bars + 2 * STAGES;   // [2] MMA -> epilogue
+  uint64_t* tempty = tfull + 2;          // [2] epilogue -> MMA
+  uint64_t* done = tempty + 2;           // all MMAs retired
+  uint32_t* s_tmem = reinterpret_cast<uint32_t*>(done + 1);
+  volatile int* s_abort = reinterpret_cast<volatile int*>(s_tmem + 1);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&tfull[b], 1);
+      mbar_init(&tempty[b], 8);          // one arrive per epilogue warp
+    }
+    mbar_init(done, 1);
+    *s_abort = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 1) tmem_alloc(s_tmem, TMEM_COLS);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *s_tmem;
+  pdl_launch_dependents();
+  pdl_wait();
+
+  if (warp == 0) {
+    // ------------------------------ TMA producer ------------------------------
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t ph = 0;
+      int issued = 0;
+      int last = -1;
+      for (int u = blockIdx.x; u < g.units && !*s_abort; u += gridDim.x) {
+        const int j = member_of(g, u);
+        const GemmMember& M = g.m[j];
+        if (j != last) {
+          tma_prefetch_desc(&M.a);
+          tma_prefetch_desc(&M.b);
+          last = j;
+        }
+        const int tile = u - M.unit_begin;
+        const int mb = tile / M.tiles_n, nb = tile - mb * M.tiles_n;
+        for (int kb = 0; kb < M.nkb; ++kb) {
+          if (!mbar_wait(&empty[stage], ph ^ 1u)) {
+            *s_abort = 1;
+            atomicExch(g.err, kErrMbarTimeout);
+            break;
+          }
+          mbar_arrive_expect_tx(&full[stage], STAGE_BYTES);
+          tma_load_2d(sA + (size_t)stage * A_BYTES, &M.a, &full[stage], kb * BK, mb * BM);
+          tma_load_2d(sB + (size_t)stage * B_BYTES, &M.b, &full[stage], kb * 2 * BK, nb * BN);
+          ++issued;
+          if (++stage == STAGES) { stage = 0; ph ^= 1u; }
+        }
+      }
+      // drain (bounded): no TMA write is in flight when the CTA exits
+      int s = stage;
+      uint32_t q = ph;
+      for (int i = 0; i < STAGES && i < issued; ++i) {
+        if (--s < 0) { s = STAGES - 1; q ^= 1u; }
+        mbar_wait(&full[s], q);
+      }
+    }
+  } else if (warp == 1) {
+    // ------------------------------ MMA issuer --------------------------------
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t ph = 0;
+      int ab = 0;
+      uint32_t aph = 0;
+      for (int u = blockIdx.x; u < g.units && !*s_abort; u += gridDim.x) {
+        const int nkb = g.m[member_of(g, u)].nkb;
+        if (!mbar_wait(&tempty[ab], aph ^ 1u)) {
+          *s_abort = 1;
+          atomicExch(g.err, kErrMbarTimeout);
+          break;
+        }
+        tc_fence_after();
+        const uint32_t d = tmem_base + (uint32_t)(ab * BN);
+        bool ok = true;
+        for (int kb = 0; kb < nkb; ++kb) {
+          if (!mbar_wait(&full[stage], ph)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint64_t ad = smem_desc(sA + (size_t)stage * A_BYTES, 512, kSwizzle64);
+          const uint64_t bd = smem_desc(sB + (size_t)stage * B_BYTES, 1024, kSwizzle128);
+#pragma unroll
+          for (int k = 0; k < BK / 32; ++k) {
+            mma_e4m3(d, ad + 2u * k, bd + 2u * k, kIdesc, (kb > 0 || k > 0) ? 1u : 0u);
+            mma_e4m3(d, ad + 2u * k, bd + 4u + 2u * k, kIdesc, 1u);
+          }
+          mma_commit(&empty[stage]);
+          if (++stage == STAGES) { stage = 0; ph ^= 1u; }
+        }
+        if (!ok) {
+          *s_abort = 1;
+          atomicExch(g.err, kErrMbarTimeout);
+          break;
+        }
+        mma_commit(&tfull[ab]);
+        if (++ab == 2) { ab = 0; aph ^= 1u; }
+      }
+      mma_commit(done);
+      mbar_wait(done, 0);
+    }
+  } else {
+    // ------------------------------ epilogue ----------------------------------
+    // Warps work alone (no barrier joins them), so a warp that gives up on a
+    // timed-out wait strands no other.
+    const int q = warp & 3;
+    const int half = (warp - 2) >> 2;
+    uint32_t* tr = s_tr + (size_t)(warp - 2) * 32 * TR16_STRIDE;
+    int ab = 0;
+    uint32_t aph = 0;
+    for (int u = blockIdx.x; u < g.units; u += gridDim.x) {
+      const GemmMember& M = g.m[member_of(g, u)];
+      const int tile = u - M.unit_begin;
+      const int mb = tile / M.tiles_n, nb = tile - mb * M.tiles_n;
+      if (!mbar_wait(&tfull[ab], aph)) {
+        *s_abort = 1;
+        if (lane == 0) atomicExch(g.err, kErrMbarTimeout);
+        break;
+      }
+      tc_fence_after();
+      const int row0 = mb * BM + q * 32;
+      const uint32_t trow = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(ab * BN + half * 16);
+#pragma unroll 1
+      for (int c = 0; c < CPT; ++c) {
+        const int col0 = nb * BN + c * 32 + half * 16;
+        uint32_t v[16];
+        tmem_ld16(trow + (uint32_t)(c * 32), v);
+        store_block16(M.p, tr, v, row0, col0, column_scale(M.p, col0 + (lane & 15)));
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&tempty[ab]);
+      if (++ab == 2) { ab = 0; aph ^= 1u; }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem_base, TMEM_COLS);
+  }
+}
+
 // ---- operand preparation ------------------------------------------------------
 
 // e4m3 encoding (1 sign bit, 4 exponent bits with bias 7, 3 mantissa bits) of
@@ -715,6 +899,21 @@ cudaError_t launch_spikes_to_01(const void* spikes, int fmt, int64_t ld, int T, 
                       fmt, ld, T, K, Kp, Xs);
   return launch_pdl(spikes_to_01_kernel<false>, dim3((unsigned)blocks), dim3(threads), 0, s, spikes,
                     fmt, ld, T, K, Kp, Xs);
+}
+
+cudaError_t launch_gemm_group(const GemmGroupArgs& a, cudaStream_t s) {
+  cudaError_t e = init_sms();
+  if (e != cudaSuccess) return e;
+  static bool attr = false;
+  if (!attr) {
+    e = cudaFuncSetAttribute(gemm_group_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)kGemmSmem);
+    if (e != cudaSuccess) return e;
+    attr = true;
+  }
+  if (a.units < 1) return cudaSuccess;
+  const int grid = a.units < g_num_sms ? a.units : g_num_sms;
+  return launch_pdl(gemm_group_kernel, dim3(grid), dim3(kGemmThreads), kGemmSmem, s, a);
 }
 
 int gemm_splits(int T, int N, int Kp, int part_units) {

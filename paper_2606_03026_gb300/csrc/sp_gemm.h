@@ -37,4 +37,27 @@ int gemm_splits(int T, int N, int Kp, int part_units);
 cudaError_t launch_gemm(const CUtensorMap& mapA, const CUtensorMap& mapB, int S, int T, int N,
                         int Kp, const GemmParams& p, cudaStream_t s);
 
+// Grouped form: the output tiles of up to kGemmMaxMembers independent
+// contractions (one per plan of a group, each with its own operands, sizes
+// and outputs) in ONE persistent launch, every tile over its whole K.
+constexpr int kGemmMaxMembers = SPIKE_PROJ_MAX_GROUP;
+struct GemmMember {
+  CUtensorMap a;          // 0/1 spike rows [>= T][Kp] (staging copy or caller's bool8 rows)
+  CUtensorMap b;          // weight planes [N][2 Kp]
+  GemmParams p;           // scale, acc, y, T, N, K of this member (part unused)
+  int32_t tiles_n;        // ceil(N / 256)
+  int32_t nkb;            // Kp / 64 K blocks
+  int32_t unit_begin;     // first output tile of this member in the launch
+  int32_t unit_end;       // one past its last
+};
+// Kernel parameters of one grouped launch, passed by value (__grid_constant__;
+// about 24 KB at 64 members, inside the 32 KB kernel-parameter limit).
+struct GemmGroupArgs {
+  GemmMember m[kGemmMaxMembers];
+  int32_t count;          // members
+  int32_t units;          // output tiles of all members
+  int* err;               // device error word
+};
+cudaError_t launch_gemm_group(const GemmGroupArgs& a, cudaStream_t s);
+
 }  // namespace sp

@@ -49,6 +49,7 @@ _SIGNATURES = {
     "spike_proj_group_decode_lif": ([_P, _P, _P, _P, _I64, ctypes.c_float, ctypes.c_float, _P,
                                      _I64, _P, _P, _I64, _P], ctypes.c_int),
     "spike_proj_group_status": ([_P, _P], ctypes.c_int),
+    "spike_proj_group_prefill": ([_P, _P, ctypes.c_int, _I32, _I64, _P, _P, _P], ctypes.c_int),
     "spike_proj_decode_noalloc": ([_P, _I64, _P, _I32, _I32, _P, ctypes.c_int, _P, _P, _P],
                                   ctypes.c_int),
     "spike_proj_dense": ([_P, _I32, _I32, _P], ctypes.c_int),
@@ -205,6 +206,20 @@ def spike_proj_group_decode_lif(group, v_in, v_out, I, ld, beta, theta, bits=Non
            "spike_proj_group_decode_lif")
 
 
+def _ptr_array(xs):
+    """Host array of device addresses (ctypes), or None."""
+    if xs is None:
+        return None
+    return (ctypes.c_void_p * len(xs))(*[_addr(x) for x in xs])
+
+
+def spike_proj_group_prefill(group, X, fmt, T, ldx, acc=None, y=None, stream=None):
+    """X, acc, y: sequences with one device tensor (or address) per member."""
+    _check(lib().spike_proj_group_prefill(group, _ptr_array(X), _fmt(fmt), T, ldx,
+                                          _ptr_array(acc), _ptr_array(y), _stream(stream)),
+           "spike_proj_group_prefill")
+
+
 def spike_proj_group_status(group, stream=None) -> int:
     return lib().spike_proj_group_status(group, _stream(stream))
 
@@ -332,6 +347,11 @@ class Group:
         [count, >= ceil(maxK/32)]) optionally receives the spike words."""
         spike_proj_group_decode_lif(self.handle, v_in, v_out, I, v_in.stride(0), beta, theta, bits,
                                     0 if bits is None else bits.stride(0), acc, y, ld_out, stream)
+
+    def prefill(self, X, fmt, T, ldx, acc=None, y=None, stream=None):
+        """T rows per member through the tensor-core contraction, all members
+        in one launch: X, acc, y hold one device tensor per member."""
+        spike_proj_group_prefill(self.handle, X, fmt, T, ldx, acc, y, stream)
 
     def status(self, stream=None) -> int:
         return spike_proj_group_status(self.handle, stream)
