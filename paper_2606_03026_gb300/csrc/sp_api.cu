@@ -76,6 +76,8 @@ struct sp_group_s {
   // table, and per member the caller's 0/1 rows of the last in-place call
   sp_plan_s* plans[kMaxProblems] = {};
   GemmGroupArgs* gemm = nullptr;
+  float* gpart = nullptr;         // tail-split partials (groups of SP_PLAN_GEMM plans)
+  uint32_t* gflags = nullptr;     // their flags, zero between launches
   const void* rows_ptr[kMaxProblems] = {};
   int64_t rows_ld[kMaxProblems] = {};
   int32_t rows_T[kMaxProblems] = {};
@@ -146,6 +148,8 @@ void plan_free(sp_plan_s* p) {
 void group_free(sp_group_s* g) {
   if (!g) return;
   delete g->gemm;
+  cudaFree(g->gpart);
+  cudaFree(g->gflags);
   cudaFree(g->ws);
   cudaFree(g->tickets);
   cudaFree(g->err);
@@ -519,6 +523,14 @@ sp_status spike_proj_group_create(sp_group_t* group, const sp_plan_t* plans, int
     group_free(g);
     return st;
   }
+  bool all_gemm = true;
+  for (int j = 0; j < count; ++j) all_gemm = all_gemm && (plans[j]->flags & SP_PLAN_GEMM);
+  if (all_gemm &&
+      ((st = dev_alloc_zero(&g->gpart, (size_t)kGemmGroupSlots * kGemmPartialElems, s)) != SP_OK ||
+       (st = dev_alloc_zero(&g->gflags, (size_t)kGemmGroupSlots * 8, s)) != SP_OK)) {
+    group_free(g);
+    return st;
+  }
   g->params.ws = g->ws;
   g->params.tickets = g->tickets;
   g->params.err = g->err;
@@ -576,7 +588,18 @@ sp_status spike_proj_group_prefill(sp_group_t g, const void* const* X, sp_fmt fm
   GemmGroupArgs& a = *g->gemm;
   a.count = g->count;
   a.err = g->err;
+  a.part = g->gpart;
+  a.flags = g->gflags;
   int64_t units = 0;
+  // CTA pairs (2-SM MMA over 256 rows) when the members' row tiles pair up
+  // with little padding
+  int tm[kMaxProblems], tn[kMaxProblems];
+  for (int j = 0; j < g->count; ++j) {
+    tm[j] = ceil_div(T, 128);
+    tn[j] = ceil_div(g->plans[j]->N, 256);
+  }
+  const int cl = gemm_group_cluster(tm, tn, g->count);
+  a.cl = cl;
   // 0/1 byte rows that TMA can address are read in place; any other input
   // is first written as 0/1 bytes into the member plan's staging copy
   const bool vec = fmt == SP_SPIKES_BOOL8 && ldx % 16 == 0;
@@ -595,7 +618,7 @@ sp_status spike_proj_group_prefill(sp_group_t g, const void* const* X, sp_fmt fm
       SP_CUDA(launch_spikes_to_01(X[j], fmt, ldx, T, p->K, p->Kp, p->Xs, s));
       M.a = p->maps.a;
     }
-    M.b = p->maps.b;
+    M.b = cl == 2 ? p->maps.b128 : p->maps.b;
     M.p.scale = p->scale;
     M.p.acc = acc ? acc[j] : nullptr;
     M.p.y = y ? y[j] : nullptr;
@@ -605,10 +628,10 @@ sp_status spike_proj_group_prefill(sp_group_t g, const void* const* X, sp_fmt fm
     M.p.err = g->err;
     M.p.part = nullptr;
     M.p.part_units = 0;
-    M.tiles_n = ceil_div(p->N, 256);
+    M.tiles_n = tn[j];
     M.nkb = p->Kp / 64;
     M.unit_begin = (int32_t)units;
-    units += (int64_t)ceil_div(T, 128) * M.tiles_n;
+    units += (int64_t)ceil_div(tm[j], cl) * tn[j];
     if (units > INT32_MAX) return SP_ERANGE;
     M.unit_end = (int32_t)units;
   }
@@ -740,6 +763,8 @@ sp_status spike_proj_group_status(sp_group_t g, sp_stream_t stream) {
   SP_CUDA(cudaMemsetAsync(g->err, 0, sizeof(int), s));
   SP_CUDA(cudaMemsetAsync(g->ws, 0, g->ws_elems * sizeof(int32_t), s));
   SP_CUDA(cudaMemsetAsync(g->tickets, 0, g->n_tickets * sizeof(uint32_t), s));
+  if (g->gflags)
+    SP_CUDA(cudaMemsetAsync(g->gflags, 0, (size_t)kGemmGroupSlots * 8 * sizeof(uint32_t), s));
   SP_CUDA(cudaStreamSynchronize(s));
   return SP_EKERNEL;
 }

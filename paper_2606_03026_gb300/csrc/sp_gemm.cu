@@ -490,56 +490,141 @@ gemm_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CU
 //
 // The output tiles of every member of a group (e.g. the 22 down projections
 // of a 512-token prefill: 22 x 4 x 6 = 528 tiles of 128 x 256) form one list,
-// member after member; CTA b of a grid of min(tiles, SMs) takes tiles b,
-// b + grid, ...  Each tile runs over its whole K, so no partial leaves the
-// SM: the producer / MMA pipeline is the one of gemm_kernel, and the
-// epilogue of tile i (8 warps: TMEM lane quarter w % 4, 16-column half
-// (w - 2) / 4 of every 32-column chunk) overlaps the MMAs of tile i + 1
-// through the double-buffered accumulator.
+// member after member.  A unit is CL row tiles of one member with the same 256
+// channels (row tiles CL g + r, r = the CTA's rank in its cluster of CL);
+// cluster c of a persistent grid takes units c, c + clusters, ...  Each tile
+// runs over its whole K, so no partial leaves the SM, and the epilogue of unit
+// i (8 warps: TMEM lane quarter w % 4, 16-column half (w - 2) / 4 of every
+// 32-column chunk) overlaps the MMAs of unit i + 1 through the
+// double-buffered accumulator.
+//
+// CL = 2 runs each unit on a CTA pair with the 2-SM MMA (.cta_group::2,
+// M = 256): each CTA loads its own 128 spike rows and HALF of the 256
+// weight rows of every K block, and one thread of the even CTA issues the
+// MMAs, which read both CTAs' shared memory and write each CTA's own 128
+// accumulator rows.  Per K block an SM then takes in 24 KB instead of 40 KB
+// and its tensor core reads 8 KB instead of 12 KB per MMA, which takes the
+// K loop from shared-memory bound to tensor bound; the ring holds 8 stages
+// instead of 5.  Both CTAs' copies complete on the even CTA's full barrier
+// (which expects the pair's bytes); the even CTA's commits arrive on the
+// empty / accumulator barriers of both CTAs; both CTAs' epilogue warps
+// release an accumulator on the even CTA's barrier.  A row tile past a
+// member's last (T not a multiple of 256) is computed on zero rows (TMA
+// fills past T) and writes nothing.
 
-// Member holding output tile u (members are few, their tile ranges ascending).
+template <int CL>
+struct GroupCfg {
+  static constexpr int kStages = CL == 2 ? 8 : STAGES;
+  static constexpr int kBStage = B_BYTES / CL;      // this CTA's weight rows x 128 B
+  static constexpr uint32_t kStageTx = (uint32_t)CL * (A_BYTES + kBStage);
+  static constexpr size_t kRing = (size_t)kStages * (A_BYTES + kBStage);
+  static constexpr size_t kSmem = 1024 + kRing + SMEM_TR + SMEM_BARS;
+  // kind::f8f6f4 instruction descriptor with M = 128 CL
+  static constexpr uint32_t kIdesc =
+      (1u << 4) | ((uint32_t)(BN >> 3) << 17) | ((uint32_t)((BM * CL) >> 4) << 24);
+};
+static_assert(GroupCfg<1>::kSmem <= 227 * 1024 && GroupCfg<2>::kSmem <= 227 * 1024,
+              "shared memory per CTA");
+static_assert((2 * GroupCfg<2>::kStages + 5) * 8 + 8 <= (int)SMEM_BARS, "barrier area");
+
+// Member holding unit u (members are few, their unit ranges ascending).
 __device__ __forceinline__ int member_of(const GemmGroupArgs& g, int u) {
   int j = 0;
   while (j + 1 < g.count && u >= g.m[j].unit_end) ++j;
   return j;
 }
 
+// One unit of a grouped launch as a CTA of rank `rank` sees it.
+struct GroupUnit {
+  int j;                  // member
+  int mb, nb;             // this CTA's row tile and the channel tile
+  int kb0, kb1;           // K blocks [kb0, kb1)
+  int role;               // 0 whole K, 1 owner of a split unit, 2 helper
+  int slot;               // helper: its partial slot; owner: its first helper's
+};
+
+template <int CL>
+__device__ __forceinline__ GroupUnit group_unit(const GemmGroupArgs& g, int v, int rank) {
+  GroupUnit r;
+  int u = v, s = 0, S = 1;
+  r.role = 0;
+  r.slot = 0;
+  if (v >= g.whole) {
+    S = g.tail_s;
+    const int t = (v - g.whole) / S;
+    s = v - g.whole - t * S;
+    u = g.whole + t;
+    r.role = s == 0 ? 1 : 2;
+    r.slot = t * (S - 1) + (s == 0 ? 0 : s - 1);
+  }
+  r.j = member_of(g, u);
+  const GemmMember& M = g.m[r.j];
+  const int unit = u - M.unit_begin;
+  const int mg = unit / M.tiles_n;
+  r.nb = unit - mg * M.tiles_n;
+  r.mb = mg * CL + rank;
+  r.kb0 = s * M.nkb / S;
+  r.kb1 = (s + 1) * M.nkb / S;
+  return r;
+}
+
+__device__ __forceinline__ uint32_t ld_acquire(const uint32_t* p) {
+  uint32_t v;
+  asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+__device__ __forceinline__ void st_release(uint32_t* p, uint32_t v) {
+  asm volatile("st.release.gpu.global.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+
+template <int CL>
 __global__ void __launch_bounds__(kGemmThreads, 1)
 gemm_group_kernel(const __grid_constant__ GemmGroupArgs g) {
+  using C = GroupCfg<CL>;
+  constexpr int ST = C::kStages;
+  constexpr bool kPair = CL == 2;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
   uint8_t* sA = smem;
-  uint8_t* sB = smem + (size_t)STAGES * A_BYTES;
-  uint32_t* s_tr = reinterpret_cast<uint32_t*>(smem + SMEM_RING);
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + SMEM_RING + SMEM_TR);
-  uint64_t* full = bars;                 // [STAGES] TMA -> MMA
-  uint64_t* empty = bars + STAGES;       // [STAGES] MMA -> TMA
-  uint64_t* tfull = bars + 2 * STAGES;   // [2] MMA -> epilogue
-  uint64_t* tempty = tfull + 2;          // [2] epilogue -> MMA
+  uint8_t* sB = smem + (size_t)ST * A_BYTES;
+  uint32_t* s_tr = reinterpret_cast<uint32_t*>(smem + C::kRing);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::kRing + SMEM_TR);
+  uint64_t* full = bars;                 // [ST] TMA (both CTAs of a pair) -> MMA
+  uint64_t* empty = bars + ST;           // [ST] MMA -> TMA
+  uint64_t* tfull = bars + 2 * ST;       // [2] MMA -> epilogue
+  uint64_t* tempty = tfull + 2;          // [2] epilogue (both CTAs of a pair) -> MMA
   uint64_t* done = tempty + 2;           // all MMAs retired
   uint32_t* s_tmem = reinterpret_cast<uint32_t*>(done + 1);
   volatile int* s_abort = reinterpret_cast<volatile int*>(s_tmem + 1);
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
+  const int rank = kPair ? (int)cluster_ctarank() : 0;
+  const bool leader = rank == 0;
+  const int cluster = (int)blockIdx.x / CL, nclusters = (int)gridDim.x / CL;
 
   if (threadIdx.x == 0) {
-    for (int s = 0; s < STAGES; ++s) {
+    for (int s = 0; s < ST; ++s) {
       mbar_init(&full[s], 1);
       mbar_init(&empty[s], 1);
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&tfull[b], 1);
-      mbar_init(&tempty[b], 8);          // one arrive per epilogue warp
+      mbar_init(&tempty[b], 8 * CL);     // one arrive per epilogue warp of the pair
     }
     mbar_init(done, 1);
     *s_abort = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
-  if (warp == 1) tmem_alloc(s_tmem, TMEM_COLS);
+  if (warp == 1) {
+    if (kPair) tmem_alloc_pair(s_tmem, TMEM_COLS);
+    else tmem_alloc(s_tmem, TMEM_COLS);
+  }
   tc_fence_before();
-  __syncthreads();
+  // both CTAs' barriers exist before either signals the other's
+  if (kPair) cluster_sync();
+  else __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *s_tmem;
   pdl_launch_dependents();
@@ -548,50 +633,61 @@ gemm_group_kernel(const __grid_constant__ GemmGroupArgs g) {
   if (warp == 0) {
     // ------------------------------ TMA producer ------------------------------
     if (lane == 0) {
+      const uint32_t full_cl = kPair ? cluster_addr(full, 0) : 0u;   // even CTA's full[0]
       int stage = 0;
       uint32_t ph = 0;
       int issued = 0;
       int last = -1;
-      for (int u = blockIdx.x; u < g.units && !*s_abort; u += gridDim.x) {
-        const int j = member_of(g, u);
-        const GemmMember& M = g.m[j];
-        if (j != last) {
+      for (int v = cluster; v < g.total && !*s_abort; v += nclusters) {
+        const GroupUnit U = group_unit<CL>(g, v, rank);
+        const GemmMember& M = g.m[U.j];
+        if (U.j != last) {
           tma_prefetch_desc(&M.a);
           tma_prefetch_desc(&M.b);
-          last = j;
+          last = U.j;
         }
-        const int tile = u - M.unit_begin;
-        const int mb = tile / M.tiles_n, nb = tile - mb * M.tiles_n;
-        for (int kb = 0; kb < M.nkb; ++kb) {
+        const int mb = U.mb, nb = U.nb;
+        for (int kb = U.kb0; kb < U.kb1; ++kb) {
           if (!mbar_wait(&empty[stage], ph ^ 1u)) {
             *s_abort = 1;
             atomicExch(g.err, kErrMbarTimeout);
             break;
           }
-          mbar_arrive_expect_tx(&full[stage], STAGE_BYTES);
-          tma_load_2d(sA + (size_t)stage * A_BYTES, &M.a, &full[stage], kb * BK, mb * BM);
-          tma_load_2d(sB + (size_t)stage * B_BYTES, &M.b, &full[stage], kb * 2 * BK, nb * BN);
+          if (leader) mbar_arrive_expect_tx(&full[stage], C::kStageTx);
+          uint8_t* dA = sA + (size_t)stage * A_BYTES;
+          uint8_t* dB = sB + (size_t)stage * C::kBStage;
+          if (kPair) {
+            const uint32_t bar = full_cl + (uint32_t)stage * 8u;
+            tma_load_2d_pair(dA, &M.a, bar, kb * BK, mb * BM);
+            tma_load_2d_pair(dB, &M.b, bar, kb * 2 * BK, nb * BN + rank * (BN / 2));
+          } else {
+            tma_load_2d(dA, &M.a, &full[stage], kb * BK, mb * BM);
+            tma_load_2d(dB, &M.b, &full[stage], kb * 2 * BK, nb * BN);
+          }
           ++issued;
-          if (++stage == STAGES) { stage = 0; ph ^= 1u; }
+          if (++stage == ST) { stage = 0; ph ^= 1u; }
         }
       }
-      // drain (bounded): no TMA write is in flight when the CTA exits
+      // Drain (bounded): the last fills of every slot have landed (the even
+      // CTA's full barriers count both CTAs' copies) and been released by
+      // the MMA, so nothing is in flight towards either CTA when they exit.
       int s = stage;
       uint32_t q = ph;
-      for (int i = 0; i < STAGES && i < issued; ++i) {
-        if (--s < 0) { s = STAGES - 1; q ^= 1u; }
-        mbar_wait(&full[s], q);
+      for (int i = 0; i < ST && i < issued; ++i) {
+        if (--s < 0) { s = ST - 1; q ^= 1u; }
+        if (leader) mbar_wait(&full[s], q);
+        mbar_wait(&empty[s], q);
       }
     }
   } else if (warp == 1) {
     // ------------------------------ MMA issuer --------------------------------
-    if (lane == 0) {
+    if (lane == 0 && leader) {
       int stage = 0;
       uint32_t ph = 0;
       int ab = 0;
       uint32_t aph = 0;
-      for (int u = blockIdx.x; u < g.units && !*s_abort; u += gridDim.x) {
-        const int nkb = g.m[member_of(g, u)].nkb;
+      for (int v = cluster; v < g.total && !*s_abort; v += nclusters) {
+        const GroupUnit U = group_unit<CL>(g, v, rank);
         if (!mbar_wait(&tempty[ab], aph ^ 1u)) {
           *s_abort = 1;
           atomicExch(g.err, kErrMbarTimeout);
@@ -600,31 +696,41 @@ gemm_group_kernel(const __grid_constant__ GemmGroupArgs g) {
         tc_fence_after();
         const uint32_t d = tmem_base + (uint32_t)(ab * BN);
         bool ok = true;
-        for (int kb = 0; kb < nkb; ++kb) {
+        for (int kb = U.kb0; kb < U.kb1; ++kb) {
           if (!mbar_wait(&full[stage], ph)) {
             ok = false;
             break;
           }
           tc_fence_after();
           const uint64_t ad = smem_desc(sA + (size_t)stage * A_BYTES, 512, kSwizzle64);
-          const uint64_t bd = smem_desc(sB + (size_t)stage * B_BYTES, 1024, kSwizzle128);
+          const uint64_t bd = smem_desc(sB + (size_t)stage * C::kBStage, 1024, kSwizzle128);
+          // +2 = the next 32 K elements, +4 = the l plane of the weight rows
 #pragma unroll
           for (int k = 0; k < BK / 32; ++k) {
-            mma_e4m3(d, ad + 2u * k, bd + 2u * k, kIdesc, (kb > 0 || k > 0) ? 1u : 0u);
-            mma_e4m3(d, ad + 2u * k, bd + 4u + 2u * k, kIdesc, 1u);
+            const uint32_t acc = (kb > U.kb0 || k > 0) ? 1u : 0u;
+            if (kPair) {
+              mma_e4m3_pair(d, ad + 2u * k, bd + 2u * k, C::kIdesc, acc);
+              mma_e4m3_pair(d, ad + 2u * k, bd + 4u + 2u * k, C::kIdesc, 1u);
+            } else {
+              mma_e4m3(d, ad + 2u * k, bd + 2u * k, C::kIdesc, acc);
+              mma_e4m3(d, ad + 2u * k, bd + 4u + 2u * k, C::kIdesc, 1u);
+            }
           }
-          mma_commit(&empty[stage]);
-          if (++stage == STAGES) { stage = 0; ph ^= 1u; }
+          if (kPair) mma_commit_pair(&empty[stage], 3);
+          else mma_commit(&empty[stage]);
+          if (++stage == ST) { stage = 0; ph ^= 1u; }
         }
         if (!ok) {
           *s_abort = 1;
           atomicExch(g.err, kErrMbarTimeout);
           break;
         }
-        mma_commit(&tfull[ab]);
+        if (kPair) mma_commit_pair(&tfull[ab], 3);
+        else mma_commit(&tfull[ab]);
         if (++ab == 2) { ab = 0; aph ^= 1u; }
       }
-      mma_commit(done);
+      if (kPair) mma_commit_pair(done, 1);
+      else mma_commit(done);
       mbar_wait(done, 0);
     }
   } else {
@@ -634,39 +740,97 @@ gemm_group_kernel(const __grid_constant__ GemmGroupArgs g) {
     const int q = warp & 3;
     const int half = (warp - 2) >> 2;
     uint32_t* tr = s_tr + (size_t)(warp - 2) * 32 * TR16_STRIDE;
+    const uint32_t tempty_cl = kPair ? cluster_addr(tempty, 0) : 0u;
     int ab = 0;
     uint32_t aph = 0;
-    for (int u = blockIdx.x; u < g.units; u += gridDim.x) {
-      const GemmMember& M = g.m[member_of(g, u)];
-      const int tile = u - M.unit_begin;
-      const int mb = tile / M.tiles_n, nb = tile - mb * M.tiles_n;
+    for (int v = cluster; v < g.total; v += nclusters) {
+      const GroupUnit U = group_unit<CL>(g, v, rank);
+      const GemmMember& M = g.m[U.j];
       if (!mbar_wait(&tfull[ab], aph)) {
         *s_abort = 1;
         if (lane == 0) atomicExch(g.err, kErrMbarTimeout);
         break;
       }
       tc_fence_after();
-      const int row0 = mb * BM + q * 32;
-      const uint32_t trow = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(ab * BN + half * 16);
+      const int row0 = U.mb * BM + q * 32;
+      const bool live = row0 < M.p.T;
+      const uint32_t trow =
+          tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(ab * BN + half * 16);
+      // this warp's 32 x 16 block of chunk c inside a 128 x 256 partial tile
+      const size_t pofs = (size_t)(q * 32 + lane) + (size_t)half * 16 * 128;
+      if (U.role == 2) {
+        // helper: the partial of this CTA's rows to its slot, then this
+        // warp's flag (every lane's stores ordered before it)
+        float* dst = g.part + (size_t)(U.slot * CL + rank) * (BM * BN) + pofs;
+        if (live) {
 #pragma unroll 1
-      for (int c = 0; c < CPT; ++c) {
-        const int col0 = nb * BN + c * 32 + half * 16;
-        uint32_t v[16];
-        tmem_ld16(trow + (uint32_t)(c * 32), v);
-        store_block16(M.p, tr, v, row0, col0, column_scale(M.p, col0 + (lane & 15)));
+          for (int c = 0; c < CPT; ++c) {
+            uint32_t v[16];
+            tmem_ld16(trow + (uint32_t)(c * 32), v);
+#pragma unroll
+            for (int i = 0; i < 16; ++i)
+              __stcg(dst + (size_t)(c * 32 + i) * 128, __uint_as_float(v[i]));
+          }
+        }
+        __threadfence();
+        __syncwarp();
+        if (lane == 0) st_release(g.flags + (size_t)(U.slot * CL + rank) * 8 + (warp - 2), 1u);
+      } else {
+        const int helpers = U.role == 1 ? g.tail_s - 1 : 0;
+        bool ok = true;
+        for (int h = 0; h < helpers && ok; ++h) {
+          // owner: wait (bounded) for the helper's warp that wrote this block
+          const uint32_t* f = g.flags + (size_t)((U.slot + h) * CL + rank) * 8 + (warp - 2);
+          const long long t0 = clock64();
+          while (ld_acquire(f) == 0u) {
+            if (clock64() - t0 > kWaitLimitCycles) {
+              ok = false;
+              break;
+            }
+          }
+        }
+        __syncwarp();
+        if (!ok) {
+          *s_abort = 1;
+          if (lane == 0) atomicExch(g.err, kErrFlagTimeout);
+        } else if (live) {
+#pragma unroll 1
+          for (int c = 0; c < CPT; ++c) {
+            const int col0 = U.nb * BN + c * 32 + half * 16;
+            uint32_t v[16];
+            tmem_ld16(trow + (uint32_t)(c * 32), v);
+            for (int h = 0; h < helpers; ++h) {
+              const float* src = g.part + (size_t)((U.slot + h) * CL + rank) * (BM * BN) + pofs +
+                                 (size_t)c * 32 * 128;
+#pragma unroll
+              for (int i = 0; i < 16; ++i)
+                v[i] = __float_as_uint(__uint_as_float(v[i]) + __ldcg(src + (size_t)i * 128));
+            }
+            store_block16(M.p, tr, v, row0, col0, column_scale(M.p, col0 + (lane & 15)));
+          }
+        }
+        __syncwarp();
+        if (lane == 0)
+          for (int h = 0; h < helpers; ++h)
+            g.flags[(size_t)((U.slot + h) * CL + rank) * 8 + (warp - 2)] = 0u;   // for the next launch
       }
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&tempty[ab]);
+      if (lane == 0) {
+        if (kPair) mbar_arrive_cluster(tempty_cl + (uint32_t)ab * 8u);
+        else mbar_arrive(&tempty[ab]);
+      }
       if (++ab == 2) { ab = 0; aph ^= 1u; }
     }
   }
 
   tc_fence_before();
-  __syncthreads();
+  if (kPair) cluster_sync();             // the pair's MMAs, copies and arrivals are over
+  else __syncthreads();
   if (warp == 1) {
     tc_fence_after();
-    tmem_dealloc(tmem_base, TMEM_COLS);
+    if (kPair) tmem_dealloc_pair(tmem_base, TMEM_COLS);
+    else tmem_dealloc(tmem_base, TMEM_COLS);
   }
 }
 
@@ -865,7 +1029,9 @@ cudaError_t gemm_make_maps(const uint8_t* Xs, int rows_alloc, const uint8_t* Wq,
                     CU_TENSOR_MAP_SWIZZLE_64B))
     return cudaErrorUnknown;
   if (!encode_u8_2d(&out->b, Wq, (uint64_t)2 * Kp, (uint64_t)N, (uint64_t)2 * Kp, 2 * BK, BN,
-                    CU_TENSOR_MAP_SWIZZLE_128B))
+                    CU_TENSOR_MAP_SWIZZLE_128B) ||
+      !encode_u8_2d(&out->b128, Wq, (uint64_t)2 * Kp, (uint64_t)N, (uint64_t)2 * Kp, 2 * BK,
+                    BN / 2, CU_TENSOR_MAP_SWIZZLE_128B))
     return cudaErrorUnknown;
   return cudaSuccess;
 }
@@ -901,19 +1067,110 @@ cudaError_t launch_spikes_to_01(const void* spikes, int fmt, int64_t ld, int T, 
                     fmt, ld, T, K, Kp, Xs);
 }
 
+namespace {
+
+// Largest number of clusters of `cl` CTAs of gemm_group_kernel<cl> that can be
+// resident at once (-1 when the occupancy query fails).
+template <int CL>
+int group_active_clusters() {
+  static int n = 0;
+  if (n == 0) {
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute attr;
+    attr.id = cudaLaunchAttributeClusterDimension;
+    attr.val.clusterDim.x = CL;
+    attr.val.clusterDim.y = 1;
+    attr.val.clusterDim.z = 1;
+    cfg.gridDim = dim3(CL, 1, 1);
+    cfg.blockDim = dim3(kGemmThreads, 1, 1);
+    cfg.dynamicSmemBytes = GroupCfg<CL>::kSmem;
+    cfg.attrs = &attr;
+    cfg.numAttrs = 1;
+    int c = 0;
+    if (cudaOccupancyMaxActiveClusters(&c, gemm_group_kernel<CL>, &cfg) != cudaSuccess || c < 1) {
+      (void)cudaGetLastError();
+      c = -1;
+    }
+    n = c;
+  }
+  return n;
+}
+
+template <int CL>
+cudaError_t launch_group_cl(const GemmGroupArgs& a, cudaStream_t s) {
+  static bool attr_done = false;
+  if (!attr_done) {
+    cudaError_t e = cudaFuncSetAttribute(gemm_group_kernel<CL>,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)GroupCfg<CL>::kSmem);
+    if (e != cudaSuccess) return e;
+    attr_done = true;
+  }
+  int clusters = g_num_sms / CL;
+  if (CL > 1) {
+    const int resident = group_active_clusters<CL>();
+    if (resident < 1) return cudaErrorInvalidConfiguration;
+    if (clusters > resident) clusters = resident;
+  }
+  // Tail split: the r units past the last full round of the grid (all of
+  // them when there are fewer units than clusters) are cut into S K ranges
+  // so that the last round fills the grid.  Sub-units of the last round land
+  // on distinct clusters: the whole units are a multiple of the grid.
+  GemmGroupArgs b = a;
+  b.whole = a.units;
+  b.tail_s = 1;
+  const int r = a.units % clusters;
+  if (a.part && a.flags && r > 0) {
+    int S = clusters / r;
+    if (S > 6) S = 6;
+    int min_nkb = 1 << 30;
+    for (int j = 0; j < a.count; ++j)
+      if (a.m[j].unit_end > a.units - r && a.m[j].nkb < min_nkb) min_nkb = a.m[j].nkb;
+    while (S > 1 && (min_nkb < 4 * S || r * (S - 1) * CL > kGemmGroupSlots)) --S;
+    if (S > 1) {
+      b.whole = a.units - r;
+      b.tail_s = S;
+    }
+  }
+  b.total = b.whole + (a.units - b.whole) * b.tail_s;
+  if (clusters > b.total) clusters = b.total;
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  attr[1].id = cudaLaunchAttributeClusterDimension;
+  attr[1].val.clusterDim.x = CL;
+  attr[1].val.clusterDim.y = 1;
+  attr[1].val.clusterDim.z = 1;
+  cfg.gridDim = dim3(clusters * CL, 1, 1);
+  cfg.blockDim = dim3(kGemmThreads, 1, 1);
+  cfg.dynamicSmemBytes = GroupCfg<CL>::kSmem;
+  cfg.stream = s;
+  cfg.attrs = attr;
+  cfg.numAttrs = CL > 1 ? 2 : 1;
+  return cudaLaunchKernelEx(&cfg, gemm_group_kernel<CL>, b);
+}
+
+}  // namespace
+
+int gemm_group_cluster(const int* tiles_m, const int* tiles_n, int count) {
+  int64_t tiles = 0, pad2 = 0;
+  for (int j = 0; j < count; ++j) {
+    tiles += (int64_t)tiles_m[j] * tiles_n[j];
+    pad2 += (int64_t)(ceil_div(tiles_m[j], 2) * 2 - tiles_m[j]) * tiles_n[j];
+  }
+  return pad2 * 8 <= tiles ? 2 : 1;
+}
+
 cudaError_t launch_gemm_group(const GemmGroupArgs& a, cudaStream_t s) {
   cudaError_t e = init_sms();
   if (e != cudaSuccess) return e;
-  static bool attr = false;
-  if (!attr) {
-    e = cudaFuncSetAttribute(gemm_group_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             (int)kGemmSmem);
-    if (e != cudaSuccess) return e;
-    attr = true;
-  }
   if (a.units < 1) return cudaSuccess;
-  const int grid = a.units < g_num_sms ? a.units : g_num_sms;
-  return launch_pdl(gemm_group_kernel, dim3(grid), dim3(kGemmThreads), kGemmSmem, s, a);
+  switch (a.cl) {
+    case 1: return launch_group_cl<1>(a, s);
+    case 2: return launch_group_cl<2>(a, s);
+    default: return cudaErrorInvalidValue;
+  }
 }
 
 int gemm_splits(int T, int N, int Kp, int part_units) {

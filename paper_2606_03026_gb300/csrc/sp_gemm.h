@@ -12,7 +12,8 @@ namespace sp {
 // bytes of e4m3(16 h) then 64 bytes of e4m3(l), w = 16 h + l).
 struct GemmMaps {
   CUtensorMap a;
-  CUtensorMap b;
+  CUtensorMap b;          // 256-row boxes (one output tile's channels)
+  CUtensorMap b128;       // the same operand in 128-row boxes (half a tile)
 };
 
 int gemm_k_pad(int K);                  // K rounded up to the 64-column K block
@@ -43,7 +44,7 @@ cudaError_t launch_gemm(const CUtensorMap& mapA, const CUtensorMap& mapB, int S,
 constexpr int kGemmMaxMembers = SPIKE_PROJ_MAX_GROUP;
 struct GemmMember {
   CUtensorMap a;          // 0/1 spike rows [>= T][Kp] (staging copy or caller's bool8 rows)
-  CUtensorMap b;          // weight planes [N][2 Kp]
+  CUtensorMap b;          // weight planes [N][2 Kp] in boxes of 256 / CL rows (GemmMaps)
   GemmParams p;           // scale, acc, y, T, N, K of this member (part unused)
   int32_t tiles_n;        // ceil(N / 256)
   int32_t nkb;            // Kp / 64 K blocks
@@ -51,13 +52,36 @@ struct GemmMember {
   int32_t unit_end;       // one past its last
 };
 // Kernel parameters of one grouped launch, passed by value (__grid_constant__;
-// about 24 KB at 64 members, inside the 32 KB kernel-parameter limit).
+// about 24 KB at 64 members, inside the 32 KB kernel-parameter limit).  A
+// unit is CL row tiles of one member with the same 256 channels; with CL = 2
+// a CTA pair computes it with the 2-SM MMA (M = 256), each CTA loading its
+// own 128 spike rows and half of the 256 weight rows.
+//
+// Tail split: when the units do not fill the last round of the persistent
+// grid, each of the last r units is cut into S ranges of its K blocks (S =
+// min(clusters / r, 4)), so the last round runs r S sub-units on as many
+// clusters.  Sub-unit 0 of a split unit owns the output; each other sub-unit
+// writes its fp32 partial (per CTA one 128 x 256 tile) to part and raises a
+// per-warp flag, which the owner's warp waits for (bounded), adds and
+// clears.  The launcher fills whole / tail_s / total.
 struct GemmGroupArgs {
   GemmMember m[kGemmMaxMembers];
   int32_t count;          // members
-  int32_t units;          // output tiles of all members
+  int32_t units;          // units of all members
+  int32_t cl;             // CTAs per unit (1, or 2 for the CTA-pair MMA)
   int* err;               // device error word
+  float* part;            // tail-split partials, kGemmGroupSlots x 128 x 256 fp32 (or null)
+  uint32_t* flags;        // kGemmGroupSlots x 8 words, zero between launches
+  int32_t whole;          // units run over their whole K (the first ones)
+  int32_t tail_s;         // K ranges per tail unit (1: no split)
+  int32_t total;          // whole + (units - whole) * tail_s
 };
+// Partial tiles (128 x 256 fp32, one per CTA of a helper sub-unit) that the
+// tail split may need: at most one per SM.
+constexpr int kGemmGroupSlots = 160;
+// CTAs per unit for a grouped launch whose members have these tile counts:
+// 2 unless pairing row tiles adds more than 1/8 of idle (row-padding) tiles.
+int gemm_group_cluster(const int* tiles_m, const int* tiles_n, int count);
 cudaError_t launch_gemm_group(const GemmGroupArgs& a, cudaStream_t s);
 
 }  // namespace sp

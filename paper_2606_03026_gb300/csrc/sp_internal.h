@@ -32,6 +32,7 @@ enum DeviceError : int {
   kErrBadUnit = 1,        // a unit index decoded outside its problem
   kErrMbarTimeout = 2,    // a bounded mbarrier wait ran out (GEMM)
   kErrTmemAlloc = 3,      // tensor-memory allocation returned an odd address
+  kErrFlagTimeout = 4,    // a bounded wait for another CTA's partial ran out (GEMM)
 };
 
 // One projection as the gather kernel sees it.

@@ -161,6 +161,33 @@ def test_prefill_mixed_decoder_group():
         p.close()
 
 
+@pytest.mark.parametrize("T,shapes", [
+    (256, [(1536, 6144, 1536)] * 3),                  # 2-SM pairs, 18 units split 4 ways
+    (100, [(1536, 2000, 1536), (1536, 2048, 1536)]),  # single CTAs, 12 units split 6 ways
+    (384, [(1024, 3000, 1024)] * 7 + [(1536, 1536, 1536)] * 9),   # a partial last round
+])
+def test_tail_split_shapes(T, shapes):
+    """Groups whose tiles leave the persistent grid's last round partly idle:
+    the tail units run as K ranges on several clusters, the owner adding the
+    helpers' fp32 partials.  Every output against the oracle, twice (the
+    partials' flags are cleared for the next launch)."""
+    members = make_members(shapes, T, seed=len(shapes))
+    group = sp.Group([m[-1] for m in members])
+    ldx = max(m[4] for m in members)
+    xs_dev = []
+    for m in members:
+        r = np.zeros((T, ldx), np.uint8)
+        r[:, : m[4]] = m[2]
+        xs_dev.append(to_dev(r).bool())
+    wants = [oracle.project(Q, s, N, K, x, "u8", ldq=ldq) for (Q, s, x, N, K, ldq, _) in members]
+    for rep in range(2):
+        accs, ys = run_group(group, members, xs_dev, "bool8", T, ldx)
+        for j, (wa, wy) in enumerate(wants):
+            assert_parity(accs[j], ys[j], wa, wy, f"member {j} rep {rep}")
+    assert group.status() == sp.SP_OK
+    group.close()
+
+
 def test_group_prefill_errors():
     members = make_members(RAGGED[:2], 8, seed=9)
     plain = sp.Plan(to_dev(members[0][0]), to_dev(members[0][1]), members[0][3], members[0][4],
