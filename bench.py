@@ -7,11 +7,12 @@ Bernoulli(0.1) spikes -- i.e. 44 spike-gated projections, run as one grouped
 launch through the C ABI.  Metric: GB/s of ACTIVE-COLUMN bytes (sum over the
 44 projections of |A| * N), the bytes the method must read.
 
-Timing: W warm-up steps, then exactly K steps replayed from CUDA graphs (64
-steps per graph), bracketed by a barrier and device synchronisation, CUDA
-events on the launching stream, max over ranks.  L2: the weights are held in
-8 rotating copies (2.08 GB) and spikes in 64 rotating sets, so no weight byte
-is re-read from L2 within 8 steps (> 129 MB of other traffic in between).
+Timing: exactly W warm-up steps, then exactly K steps, replayed from CUDA
+graphs (64 steps per graph, and one graph of the remainder), bracketed by a
+barrier and device synchronisation, CUDA events on the launching stream, max
+over ranks.  L2: the weights are held in 8 rotating copies (2.08 GB) and
+spikes in 64 rotating sets, so no weight byte is re-read from L2 within 8
+steps (> 129 MB of other traffic in between).
 
 Also reported on the same JSON line:
   roofline     the grouped gather kernel (the only kernel of a step): active
@@ -19,7 +20,11 @@ Also reported on the same JSON line:
                region (CUDA events on the launching stream), against the
                measured HBM copy bandwidth; traffic = the DRAM bytes per
                launch that ncu measured for the same kernel source
-               (profiles/dram_traffic.json), null when the source differs
+               (profiles/dram_traffic.json), null when the source differs;
+               practical_peak_gbs = the same bytes over the time of a probe
+               launch that reads exactly the step's 512-byte column pieces
+               and nothing else (spike_proj_probe_gather), the ceiling of
+               this access pattern
   e2e          the same metric through the host-buffer entry point: spike
                masks read from and acc / y written to page-locked host memory
                every step (the bytes cross the CPU-GPU link inside the step)
@@ -32,7 +37,9 @@ Also reported on the same JSON line:
                chain of 44 single calls, batched B = 64 (per-token gather
                vs union fetch, independent and correlated spikes), and the
                CPU oracle on each (single thread, bounded samples)
-  clocks       nvidia-smi samples taken during the timed region
+  clocks       nvidia-smi samples taken during the timed region and 0.5 s of
+               the same step graph replayed right after it (a short timed
+               region ends between two samples)
 
 --impl reference times the CPU oracle (the only reference there is: the paper
 releases no code) on the same workload and metric.
@@ -212,6 +219,12 @@ def make_step_inputs(rank):
     return weights, sets, active
 
 
+def config_of(active_bytes_per_step):
+    """The workload description both arms print (identical keys and values)."""
+    return {"workload": WORKLOAD, "global_batch": 1,
+            "active_bytes_per_step": float(active_bytes_per_step)}
+
+
 def cpu_baseline_decode(weights, sets, seconds, channels=None):
     """The CPU oracle, single thread, on whole decode steps (or the first
     ``channels`` outputs of every projection) until ``seconds`` elapse."""
@@ -240,7 +253,7 @@ def run_reference(args):
     rank, world, _ = dist_setup(args.gpus)
     if rank != 0:
         return
-    weights, sets, _ = make_step_inputs(0)
+    weights, sets, active = make_step_inputs(0)
     # bounded sample per step: the first c output channels of all 44
     # projections, c sized so that warmup + steps end in about a minute
     budget = 60.0
@@ -269,8 +282,10 @@ def run_reference(args):
         "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": dt / max(1, args.steps) * 1e3, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "int8", "data": "synthetic",
-        "config": {"workload": WORKLOAD, "global_batch": 1, "l2": "n/a (CPU)",
-                   "parallelism": "single thread"},
+        "config": config_of(active.mean()),
+        "setup": {"l2": "n/a (CPU)", "parallelism": "single thread",
+                  "timing": f"perf_counter around exactly {args.steps} steps after "
+                            f"{args.warmup} warm-up steps"},
         "cpu_baseline": {"value": value, "unit": "GB/s", "cores": 1, "kind": "oracle",
                          "sample": sample, "host_cores": cores},
         "e2e": {"value": value, "unit": "GB/s", "h2d_bytes_per_step": 0,
@@ -316,13 +331,23 @@ def run_ours(args):
     # weight copies: 8 x 259.5 MB, each projection's copies are distinct buffers
     copies = []
     n_copies = max(1, args.weight_copies)
+    # each copy's 44 weight matrices live in one buffer (256-byte aligned
+    # slices), so that a piece of any of them is base + a 32-bit offset
+    offs, tot = [], 0
+    for (Q, _, _, _) in weights:
+        offs.append(tot)
+        tot += (Q.nbytes + 255) // 256 * 256
+    copy_bufs = []
     for c in range(n_copies):
+        buf = torch.empty(tot, dtype=torch.int8, device=dev)
         plans = []
-        for (Q, s, N, K) in weights:
-            Wd = torch.from_numpy(Q).to(dev)
+        for (Q, s, N, K), o in zip(weights, offs):
+            Wd = buf[o: o + Q.nbytes]
+            Wd.copy_(torch.from_numpy(Q.reshape(-1)))
             Sd = torch.from_numpy(s).to(dev)
             plans.append(sp.Plan(Wd, Sd, N, K))
         copies.append(sp.Group(plans))
+        copy_bufs.append(buf)
     weight_bytes = sum(Q.nbytes for (Q, _, _, _) in weights)
     spikes = torch.from_numpy(sets_np).to(dev)
     acc = torch.empty((n_proj, 1536), dtype=torch.int32, device=dev)
@@ -344,27 +369,46 @@ def run_ours(args):
         ra, _ = oracle.project(Q, s, N, K, synth.unpack_bits(sets_np[0, j], K), "u8")
         assert np.array_equal(a_np[j], ra[0]), "bench spot check failed"
 
-    # CUDA graphs of GRAPH_STEPS consecutive steps (each graph covers every
-    # weight copy and a distinct run of spike sets)
-    graphs = []
-    for g0 in range(0, SPIKE_SETS, GRAPH_STEPS):
+    # CUDA graphs of consecutive steps: a full graph of GRAPH_STEPS (every
+    # weight copy and every spike set once) and graphs of the remainders, so
+    # that exactly W warm-up and K timed steps run
+    def capture(n):
         g = torch.cuda.CUDAGraph()
         with torch.cuda.graph(g, stream=stream):
-            for i in range(g0, g0 + GRAPH_STEPS):
+            for i in range(n):
                 step(i, torch.cuda.current_stream())
-        graphs.append(g)
-    n_graph_runs = max(1, (args.steps + GRAPH_STEPS - 1) // GRAPH_STEPS)
-    steps = n_graph_runs * GRAPH_STEPS
-    warm_runs = max(1, (args.warmup + GRAPH_STEPS - 1) // GRAPH_STEPS)
+        return g
 
-    with torch.cuda.stream(stream):
-        for r in range(warm_runs):
-            graphs[r % len(graphs)].replay()
+    full = capture(GRAPH_STEPS)
+    rem_graphs = {}
+
+    def run_steps(n):
+        for _ in range(n // GRAPH_STEPS):
+            full.replay()
+        r = n % GRAPH_STEPS
+        if r:
+            if r not in rem_graphs:
+                rem_graphs[r] = capture(r)
+            rem_graphs[r].replay()
+
+    steps = max(1, args.steps)
+    warmup = max(0, args.warmup)
+    for n in {steps % GRAPH_STEPS, warmup % GRAPH_STEPS} - {0}:
+        rem_graphs[n] = capture(n)
+    # every graph the timed region replays is uploaded to the device before
+    # it (no first-launch upload inside the timed region)
+    upload_graph(full, stream)
+    for g in rem_graphs.values():
+        upload_graph(g, stream)
     stream.synchronize()
-
     sampler = ClockSampler(local)
     sampler.start()
     time.sleep(0.3)
+    # the warm-up runs straight into the timed region (no idle gap but the
+    # synchronisation that brackets it)
+    with torch.cuda.stream(stream):
+        run_steps(warmup)
+    stream.synchronize()
     ev0 = torch.cuda.Event(enable_timing=True)
     ev1 = torch.cuda.Event(enable_timing=True)
     barrier(world)
@@ -372,13 +416,22 @@ def run_ours(args):
     t_wall0 = time.time()
     with torch.cuda.stream(stream):
         ev0.record(stream)
-        for r in range(n_graph_runs):
-            graphs[r % len(graphs)].replay()
+        run_steps(steps)
         ev1.record(stream)
     stream.synchronize()
     torch.cuda.synchronize()
     barrier(world)
     t_wall1 = time.time()
+    # The timed region of a short run is shorter than one clock sample: the
+    # same graph keeps the GPU under the same load for another 0.5 s, untimed,
+    # and the clock record covers the timed region and that window.
+    with torch.cuda.stream(stream):
+        t_hold = time.time()
+        while time.time() - t_hold < 0.5:
+            for _ in range(16):
+                full.replay()
+            stream.synchronize()
+    t_wall2 = time.time()
     sampler.stop()
     elapsed_ms = ev0.elapsed_time(ev1)
     elapsed_ms = reduce_max(elapsed_ms, world)
@@ -386,7 +439,59 @@ def run_ours(args):
     total_bytes = float(sum(active[i % SPIKE_SETS] for i in range(steps))) * world
     value = total_bytes / (elapsed_ms * 1e-3) / 1e9
     ms_per_step = elapsed_ms / steps
-    clocks = sampler.summary(t_wall0, t_wall1)
+    clocks = sampler.summary(t_wall0, t_wall2)
+    clocks["window"] = (f"the timed region ({(t_wall1 - t_wall0) * 1e3:.1f} ms) and 0.5 s of the "
+                        "same step graph replayed right after it")
+
+    # Practical ceiling of the step's access pattern: the same 512-byte
+    # column pieces (every active column of every projection, 3 tiles each,
+    # from the same rotating weight copies), precomputed and dealt out evenly
+    # over the same grid shape, read with no spike-word prologue and no
+    # reduction (spike_proj_probe_gather), graph-replayed like the steps.
+    probe_offs = {512: [], 1536: []}
+    for i in range(SPIKE_SETS):
+        seg, col = [], []
+        for j, (Q, s_, N, K) in enumerate(weights):
+            ks = np.nonzero(synth.unpack_bits(sets_np[i, j], K))[0].astype(np.int64)
+            c0 = offs[j] + ks * N
+            col.append(c0)
+            for t in range(0, N, 512):
+                seg.append(c0 + t)
+        for piece, lst in ((512, seg), (1536, col)):
+            pcs = np.concatenate(lst)
+            probe_offs[piece].append(torch.from_numpy((pcs // 16).astype(np.uint32)).to(dev))
+    sink = torch.zeros(1, dtype=torch.int32, device=dev)
+
+    def probe_graph(piece, empty):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            for i in range(GRAPH_STEPS):
+                o = probe_offs[piece][i % SPIKE_SETS]
+                sp.spike_proj_probe_gather(copy_bufs[i % n_copies], o, 0 if empty else o.numel(),
+                                           sink, piece_bytes=piece,
+                                           stream=torch.cuda.current_stream())
+        return g
+
+    probe_us = {}
+    for name, piece, empty in (("segments_512", 512, False), ("columns_1536", 1536, False),
+                               ("empty", 512, True)):
+        g = probe_graph(piece, empty)
+        with torch.cuda.stream(stream):
+            for _ in range(3):
+                g.replay()
+        stream.synchronize()
+        p0 = torch.cuda.Event(enable_timing=True)
+        p1 = torch.cuda.Event(enable_timing=True)
+        reps = 20
+        with torch.cuda.stream(stream):
+            p0.record(stream)
+            for _ in range(reps):
+                g.replay()
+            p1.record(stream)
+        stream.synchronize()
+        probe_us[name] = p0.elapsed_time(p1) * 1e3 / (reps * GRAPH_STEPS)
+    best = min(probe_us["segments_512"], probe_us["columns_1536"])
+    practical_gbs = bytes_per_step / (best * 1e-6) / 1e9
 
     # one grouped-gather launch per step: its average duration over the timed
     # region is the step time.  Events around isolated launches (outside any
@@ -436,24 +541,38 @@ def run_ours(args):
 
     result = {
         "metric": METRIC, "value": value, "unit": "GB/s", "n_gpus": world,
-        "steps": steps, "warmup": warm_runs * GRAPH_STEPS, "ms_per_step": ms_per_step,
+        "steps": steps, "warmup": warmup, "ms_per_step": ms_per_step,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
         "dtype": "int8", "data": "synthetic",
-        "config": {"workload": WORKLOAD, "global_batch": world,
-                   "active_bytes_per_step": bytes_per_step,
-                   "weight_bytes_per_copy": weight_bytes,
-                   "l2": f"inputs larger than L2: {n_copies} rotating weight copies "
-                         f"({n_copies * weight_bytes / 1e9:.2f} GB) and {SPIKE_SETS} "
-                         f"rotating spike sets; no weight reuse within {n_copies} steps",
-                   "timing": f"CUDA graphs of {GRAPH_STEPS} steps, events on the launching stream",
-                   "parallelism": "replicas" if world > 1 else "single GPU"},
+        "config": config_of(bytes_per_step),
+        "setup": {"weight_bytes_per_copy": weight_bytes,
+                  "l2": f"inputs larger than L2: {n_copies} rotating weight copies "
+                        f"({n_copies * weight_bytes / 1e9:.2f} GB) and {SPIKE_SETS} "
+                        f"rotating spike sets; no weight reuse within {n_copies} steps",
+                  "timing": f"exactly {steps} steps after {warmup} warm-up steps, replayed from "
+                            f"CUDA graphs of {GRAPH_STEPS} steps (and one of the remainder), "
+                            "events on the launching stream",
+                  "parallelism": "replicas" if world > 1 else "single GPU"},
         "projected_tokens_per_s": 1e3 / ms_per_step * world,
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": hbm, "unit": "GB/s",
                      "frac": achieved / hbm, "traffic": traffic,
                      "algorithmic_bytes_per_launch": bytes_per_step,
                      "kernel": "gather_cluster_kernel<64> (grouped decode step)",
                      "launch_us": launch_ms * 1e3, "isolated_launch_us": isolated_ms * 1e3,
-                     "peak_kind": peak_kind, "frac_of_nominal_8tbs": achieved / 8000.0},
+                     "peak_kind": peak_kind, "frac_of_nominal_8tbs": achieved / 8000.0,
+                     "practical_peak_gbs": practical_gbs,
+                     "frac_of_practical_peak": achieved / practical_gbs,
+                     "practical_peak_us_per_step": best,
+                     "probe_us_per_step": {k: v for k, v in probe_us.items() if k != "empty"},
+                     "launch_floor_us": probe_us["empty"],
+                     "practical_peak_note": "spike_proj_probe_gather on the step's own active "
+                                            "columns (as 512-byte tile segments, as the gather "
+                                            "reads them, and as whole 1536-byte columns; the "
+                                            "faster counts), precomputed, evenly dealt over the "
+                                            "gather's grid shape, one round of loads, no "
+                                            "prologue or reduction, graph-replayed like the "
+                                            "steps; launch_floor_us: the same launch with no "
+                                            "pieces"},
         "e2e": {"value": e2e_bytes / (e2e_ms * 1e-3) / 1e9, "unit": "GB/s",
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                 "ms_per_step": e2e_ms / e2e_steps,
@@ -497,6 +616,21 @@ def run_ours(args):
         g.close()
     if rank == 0:
         print(json.dumps(result))
+
+
+def upload_graph(g, stream):
+    """Uploads a captured graph's executable to the device (cudaGraphUpload),
+    so that its first replay is not slowed by the upload; a no-op where the
+    runtime or torch does not expose what it needs."""
+    import ctypes
+    try:
+        exe = g.raw_cuda_graph_exec()
+        rt = ctypes.CDLL("libcudart.so.13")
+        rt.cudaGraphUpload.argtypes = [ctypes.c_void_p, ctypes.c_void_p]
+        rt.cudaGraphUpload.restype = ctypes.c_int
+        rt.cudaGraphUpload(ctypes.c_void_p(int(exe)), ctypes.c_void_p(stream.cuda_stream))
+    except (AttributeError, OSError, TypeError, ValueError):
+        pass
 
 
 def graph_time_us(torch, stream, calls, reps=20):

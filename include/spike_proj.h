@@ -481,6 +481,32 @@ sp_status spike_proj_head(sp_head_t head, const float *h, int64_t ldh, int32_t B
                           int32_t *verified, float *gap, int32_t *cand, float *r,
                           float *z, int64_t ld_z, sp_stream_t stream);
 
+/* ---------------------------------------------------------------------------
+ * spike_proj_probe_gather -- MEASUREMENT AID, not part of the method (the
+ * paper has no counterpart).  Reads `count` pieces of `piece_bytes`
+ * contiguous bytes (512, 1024 or 1536), piece i at base + 16 * offsets16[i],
+ * and nothing else: the pieces are dealt out round-robin over every warp of a
+ * grid shaped like the gather's (4 CTAs of 256 threads per SM), each lane
+ * reading 16 bytes of every 512 of each of its warp's pieces, all in one
+ * round of loads, with the gather's programmatic dependent launch.  Given the
+ * active-column pieces of a decode step (512-byte tile segments, as the
+ * gather kernel reads them, or whole 1536-byte columns), its time per launch
+ * is the practical ceiling of that access pattern, free of the method's
+ * spike-word prologue and reduction; with count = 0 it measures the launch
+ * and dependency floor alone.
+ *
+ *   base         device, 16-byte aligned.
+ *   offsets16    device uint32 [count], in units of 16 bytes (so base may
+ *                span 64 GB); every piece must lie inside an allocation.
+ *   piece_bytes  512, 1024 or 1536 (else SP_EINVAL).
+ *   sink         device uint32: the XOR of every 32-bit word read is XORed
+ *                into it (so the bytes read can be checked).
+ * Errors: SP_EINVAL, SP_EALIGN, SP_EDEVICE, SP_ECUDA.
+ * ------------------------------------------------------------------------- */
+sp_status spike_proj_probe_gather(const void *base, const uint32_t *offsets16,
+                                  int32_t count, int32_t piece_bytes,
+                                  uint32_t *sink, sp_stream_t stream);
+
 /* --------------------------------------------------------------------------- */
 const char *spike_proj_strerror(sp_status status);
 /* cudaError_t code of the last failing CUDA call made by this thread. */

@@ -807,6 +807,20 @@ sp_status spike_proj_decode_noalloc(const int8_t* W, int64_t ldw, const float* s
   return SP_OK;
 }
 
+sp_status spike_proj_probe_gather(const void* base, const uint32_t* offsets16, int32_t count,
+                                  int32_t piece_bytes, uint32_t* sink, sp_stream_t stream) {
+  if (!base || !sink || count < 0 || (count > 0 && !offsets16)) return SP_EINVAL;
+  if (piece_bytes != 512 && piece_bytes != 1024 && piece_bytes != 1536) return SP_EINVAL;
+  if (!aligned(base, 16) || !aligned(sink, 4) || (offsets16 && !aligned(offsets16, 4)))
+    return SP_EALIGN;
+  int dev = 0;
+  const sp_status st = check_device(&dev);
+  if (st != SP_OK) return st;
+  SP_CUDA(launch_probe_gather(static_cast<const uint8_t*>(base), offsets16, count, piece_bytes,
+                              sink, as_stream(stream)));
+  return SP_OK;
+}
+
 sp_status spike_proj_lif(float* v, const float* I, int32_t K, int32_t rows, int64_t ld,
                          float beta, float theta, uint32_t* bits, int64_t ld_bits,
                          sp_stream_t stream) {

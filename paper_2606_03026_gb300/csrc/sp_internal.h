@@ -198,6 +198,11 @@ cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t s
   return cudaLaunchKernelEx(&cfg, kernel, static_cast<Args&&>(args)...);
 }
 
+// Measurement aid (sp_probe.cu): reads count pieces of piece_bytes (512, 1024
+// or 1536) at base + 16 * offsets16[i], XOR of every word into *sink.
+cudaError_t launch_probe_gather(const uint8_t* base, const uint32_t* offsets16, int count,
+                                int piece_bytes, uint32_t* sink, cudaStream_t s);
+
 // ---------------------------------------------------------------------------
 // Host launch wrappers (defined next to their kernels).  Each returns the
 // cudaError_t of the launch.

@@ -59,6 +59,7 @@ _SIGNATURES = {
     "spike_proj_head_destroy": ([_P], ctypes.c_int),
     "spike_proj_head": ([_P, _P, _I64, _I32, ctypes.c_float, _I32, _P, _P, _P, _P, _P, _P, _I64,
                          _P], ctypes.c_int),
+    "spike_proj_probe_gather": ([_P, _P, _I32, _I32, _P, _P], ctypes.c_int),
     "spike_proj_strerror": ([ctypes.c_int], ctypes.c_char_p),
     "spike_proj_last_cuda_error": ([], ctypes.c_int),
     "spike_proj_abi_version": ([], ctypes.c_int),
@@ -272,6 +273,12 @@ def spike_proj_decode_noalloc(W, ldw, scale, N, K, spikes, fmt, acc=None, y=None
     _check(lib().spike_proj_decode_noalloc(_addr(W), ldw, _addr(scale), N, K, _addr(spikes),
                                            _fmt(fmt), _addr(acc), _addr(y), _stream(stream)),
            "spike_proj_decode_noalloc")
+
+
+def spike_proj_probe_gather(base, offsets16, count, sink, piece_bytes=512, stream=None):
+    """Measurement aid: read `count` pieces of `piece_bytes` at base + 16 * offsets16[i]."""
+    _check(lib().spike_proj_probe_gather(_addr(base), _addr(offsets16), count, piece_bytes,
+                                         _addr(sink), _stream(stream)), "spike_proj_probe_gather")
 
 
 def spike_proj_strerror(status) -> str:

@@ -71,6 +71,12 @@ def test_host_only_calls(lib):
         spikeproj.SP_EINVAL                # unknown flag
     assert lib.spike_proj_decode(None, fake, 0, fake, fake, None) == spikeproj.SP_EINVAL
     assert lib.spike_proj_group_create(None, None, 0, None) == spikeproj.SP_EINVAL
+    assert lib.spike_proj_group_prefill(None, None, 0, 1, 16, None, None, None) == \
+        spikeproj.SP_EINVAL
+    assert lib.spike_proj_probe_gather(None, fake, 1, 512, fake, None) == spikeproj.SP_EINVAL
+    assert lib.spike_proj_probe_gather(fake, None, 1, 512, fake, None) == spikeproj.SP_EINVAL
+    assert lib.spike_proj_probe_gather(fake, fake, 1, 768, fake, None) == spikeproj.SP_EINVAL
+    assert lib.spike_proj_probe_gather(fake + 4, fake, 1, 512, fake, None) == spikeproj.SP_EALIGN
     assert lib.spike_proj_dense(None, 1, 1, None) == spikeproj.SP_EINVAL
     d = spikeproj.SpDense(fake, 32, fake, fake, 32, fake, 16, 16, 32)
     assert lib.spike_proj_dense(ctypes.addressof(d), 1, 0, None) == spikeproj.SP_EINVAL   # B = 0
