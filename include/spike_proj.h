@@ -314,9 +314,9 @@ sp_status spike_proj_group_decode_lif(sp_group_t group, const float *v_in,
 sp_status spike_proj_group_status(sp_group_t group, sp_stream_t stream);
 
 /* ---------------------------------------------------------------------------
- * spike_proj_decode_noalloc -- batch-1 decode (Eq. (sparse)) that allocates
- * no memory at all.  The paper has no counterpart: this is a library
- * convenience, not part of the method.
+ * spike_proj_decode_noalloc -- a batch-1 decode with the same result as
+ * spike_proj_decode, that allocates no memory at all.  The paper has no
+ * counterpart: this is a library convenience, not part of the method.
  *
  * Who needs it: callers that may not allocate device memory on their decode
  * path -- a serving loop where cudaMalloc / cudaFree would synchronise the
@@ -326,22 +326,25 @@ sp_status spike_proj_group_status(sp_group_t group, sp_stream_t stream);
  * arguments directly (no plan) and gives the same bits as
  * spike_proj_decode on a plan of the same W, scale, N and K.
  *
- * Scratch: the split-K workspace, tile tickets and error word live in one
- * fixed array of static device memory inside the library (about 128.5 KiB
- * per device: SPIKE_PROJ_NOALLOC_MAX_N INT32 words plus 128 words), so N is
+ * Scratch: the split-K workspace and tile tickets live in one fixed array of
+ * static device memory inside the library (128 KiB + 256 bytes per device:
+ * SPIKE_PROJ_NOALLOC_MAX_N INT32 words plus one word per 512 outputs), so N is
  * limited to SPIKE_PROJ_NOALLOC_MAX_N; a larger N returns SP_ESCRATCH before
  * anything is enqueued.  No cudaMalloc, cudaFree or other allocating call is
- * made, on the first call or later.
+ * made, on the first call or later.  The kernel it runs cannot fail once
+ * launched (it has no waits and no error path) and returns the scratch to
+ * zero, so nothing has to be cleared between calls.
  *
  * First call per device: it checks the device, looks up the scratch address
- * on the current device, clears the scratch on `stream` and synchronises
- * that stream.  Make the first call on each device before any stream
- * capture begins; later calls on that device only enqueue the kernel.
+ * on the current device, clears the scratch on `stream` (defensively: it is
+ * zero when the library loads) and synchronises that stream.  Make the first
+ * call on each device before any stream capture begins; later calls on that
+ * device only enqueue the kernel.  The address is kept for the life of the
+ * process: after cudaDeviceReset do not call this entry point again.
  *
  * Concurrency: every call on one device shares the one scratch, whatever its
  * W.  Calls whose kernels can overlap on the GPU race on it and give wrong
- * results: issue them on one stream, or order the streams.  The kernel
- * leaves the scratch zeroed for the next call.
+ * results: issue them on one stream, or order the streams.
  *
  *   W, ldw, scale, N, K   as for spike_proj_plan (W, scale borrowed for the
  *                         duration of the call); N <= SPIKE_PROJ_NOALLOC_MAX_N.
@@ -480,6 +483,36 @@ sp_status spike_proj_head(sp_head_t head, const float *h, int64_t ldh, int32_t B
                           float tau, int32_t k_sel, int32_t *token,
                           int32_t *verified, float *gap, int32_t *cand, float *r,
                           float *z, int64_t ld_z, sp_stream_t stream);
+
+/* ---------------------------------------------------------------------------
+ * Test faults -- FOR TESTS OF THE ERROR PATH ONLY (the paper has no
+ * counterpart).  A fault armed on a plan or group applies to the next kernel
+ * launch of that plan or group (any decode, batched, prefill or group call;
+ * the argument checks come first) and is then disarmed:
+ *   SP_FAULT_ABORT  the launch raises the device error word and returns
+ *                   without writing its outputs and without cleaning its
+ *                   workspace (split-K partials and tile tickets stay dirty),
+ *                   as a kernel that failed half way would.
+ *   SP_FAULT_STALL  plans only, and only a tensor-core (SP_GEMM) launch: one
+ *                   TMA copy of the first CTA is never issued, and every wait
+ *                   of that launch is bounded by about 2 ms instead of 1 s, so
+ *                   the MMA's wait for the missing copy runs out: the kernel
+ *                   raises the error word, stops issuing, drains the copies
+ *                   it issued and frees its tensor memory.  Other kernels
+ *                   ignore it (it is still disarmed by their launch).
+ * No fault traps, faults the GPU or spins without bound.  spike_proj_plan_status
+ * / spike_proj_group_status then return SP_EKERNEL, clear the error word and
+ * re-zero the workspace, and the next call is exact again.
+ * Errors: SP_EINVAL (NULL, unknown fault), SP_EUNSUPPORTED (a stall on a
+ * group).
+ * ------------------------------------------------------------------------- */
+typedef enum sp_fault {
+    SP_FAULT_NONE = 0,
+    SP_FAULT_ABORT = 1,
+    SP_FAULT_STALL = 2
+} sp_fault;
+sp_status spike_proj_plan_inject_fault(sp_plan_t plan, int32_t fault);
+sp_status spike_proj_group_inject_fault(sp_group_t group, int32_t fault);
 
 /* ---------------------------------------------------------------------------
  * spike_proj_probe_gather -- MEASUREMENT AID, not part of the method (the

@@ -14,12 +14,13 @@
 using namespace sp;
 
 // Scratch of spike_proj_decode_noalloc, one copy per device in static device
-// memory: the INT32 split-K workspace of one spike row at the largest N, one
-// ticket per 512-channel output tile, and the kernel's error word (the tail is
-// padding).  Zero when the module loads; the gather kernel leaves it zero.
+// memory: the split-K workspace of one spike row at the largest N and one
+// ticket per 512-channel output tile.  Zero when the module loads; every
+// gather launch that completes leaves it zero (the kernel has no error path:
+// no waits, no aborts), so no call has to clear it.
 constexpr int kNoallocMaxN = SPIKE_PROJ_NOALLOC_MAX_N;
 constexpr int kNoallocTickets = kNoallocMaxN / kGatherNT;
-constexpr int kNoallocWords = kNoallocMaxN + 2 * kNoallocTickets;
+constexpr int kNoallocWords = kNoallocMaxN + kNoallocTickets;
 static_assert(kNoallocMaxN % kGatherNT == 0, "whole output tiles");
 static __device__ __align__(256) int32_t g_noalloc_scratch[kNoallocWords];
 
@@ -48,6 +49,7 @@ struct sp_plan_s {
   int32_t rows_T = 0;
   sp_kernel last_kernel = SP_AUTO;
   int32_t last_active = -1;
+  int32_t fault = 0;              // test fault armed for the next launch (sp_fault)
 };
 
 struct sp_head_s {
@@ -78,6 +80,7 @@ struct sp_group_s {
   GemmGroupArgs* gemm = nullptr;
   float* gpart = nullptr;         // tail-split partials (groups of SP_PLAN_GEMM plans)
   uint32_t* gflags = nullptr;     // their flags, zero between launches
+  int32_t fault = 0;              // test fault armed for the next launch (sp_fault)
   const void* rows_ptr[kMaxProblems] = {};
   int64_t rows_ld[kMaxProblems] = {};
   int32_t rows_T[kMaxProblems] = {};
@@ -206,7 +209,9 @@ GatherParams1 single_params(const sp_plan_s* p, const void* spikes, int fmt, int
 
 sp_status run_gather(sp_plan_s* p, const void* spikes, int fmt, int B, int64_t ld, int32_t* acc,
                      float* y, cudaStream_t s) {
-  const GatherParams1 g = single_params(p, spikes, fmt, B, ld, acc, y);
+  GatherParams1 g = single_params(p, spikes, fmt, B, ld, acc, y);
+  g.fault = p->fault;
+  p->fault = 0;
   SP_CUDA(launch_gather(g, s));
   return SP_OK;
 }
@@ -231,6 +236,8 @@ sp_status run_union(sp_plan_s* p, const void* spikes, int fmt, int B, int64_t ld
     u.ws = p->ws;
     u.tickets = p->tickets;
     u.err = p->err;
+    u.fault = p->fault;
+    p->fault = 0;
     SP_CUDA(launch_union(u, s));
   }
   return SP_OK;
@@ -263,6 +270,8 @@ sp_status run_gemm(sp_plan_s* p, const void* spikes, int fmt, int T, int64_t ld,
   g.err = p->err;
   g.part = p->part;
   g.part_units = p->part_units;
+  g.fault = p->fault;
+  p->fault = 0;
   SP_CUDA(launch_gemm(in_place ? p->rows_map : p->maps.a, p->maps.b, S, T, p->N, p->Kp, g, s));
   return SP_OK;
 }
@@ -305,6 +314,8 @@ sp_status run_multi(sp_plan_s* p, const void* spikes, int fmt, int B, int64_t ld
 
 // Per-device address of g_noalloc_scratch, set once by the first call on the
 // device (with that device current).  Later calls read it without a lock.
+// The address belongs to the device's current context: after
+// cudaDeviceReset the entry point must not be called again in this process.
 constexpr int kNoallocDevices = 64;
 std::mutex g_noalloc_mu;
 std::atomic<int32_t*> g_noalloc_ptr[kNoallocDevices];
@@ -323,6 +334,7 @@ sp_status noalloc_scratch(cudaStream_t s, int32_t** out) {
       if (st != SP_OK) return st;
       void* sym = nullptr;
       SP_CUDA(cudaGetSymbolAddress(&sym, g_noalloc_scratch));
+      // defensive: the array is already zero when the module loads
       SP_CUDA(cudaMemsetAsync(sym, 0, sizeof(g_noalloc_scratch), s));
       SP_CUDA(cudaStreamSynchronize(s));
       ptr = static_cast<int32_t*>(sym);
@@ -563,7 +575,11 @@ sp_status spike_proj_group_decode(sp_group_t g, const void* spikes, sp_fmt fmt, 
   P.acc = acc;
   P.y = y;
   P.ld_out = ld_out;
-  SP_CUDA(launch_gather(P, as_stream(stream)));
+  P.fault = g->fault;
+  g->fault = 0;
+  const cudaError_t e = launch_gather(P, as_stream(stream));
+  P.fault = 0;
+  SP_CUDA(e);
   return SP_OK;
 }
 
@@ -628,6 +644,7 @@ sp_status spike_proj_group_prefill(sp_group_t g, const void* const* X, sp_fmt fm
     M.p.err = g->err;
     M.p.part = nullptr;
     M.p.part_units = 0;
+    M.p.fault = g->fault;
     M.tiles_n = tn[j];
     M.nkb = p->Kp / 64;
     M.unit_begin = (int32_t)units;
@@ -636,6 +653,7 @@ sp_status spike_proj_group_prefill(sp_group_t g, const void* const* X, sp_fmt fm
     M.unit_end = (int32_t)units;
   }
   a.units = (int32_t)units;
+  g->fault = 0;
   SP_CUDA(launch_gemm_group(a, s));
   return SP_OK;
 }
@@ -678,7 +696,11 @@ sp_status spike_proj_group_decode_host(sp_group_t g, const void* h_spikes, sp_fm
     P.y = h_y ? g->d_y : nullptr;
     P.ld_out = g->maxN;
   }
-  SP_CUDA(launch_gather(P, s));
+  P.fault = g->fault;
+  g->fault = 0;
+  const cudaError_t el = launch_gather(P, s);
+  P.fault = 0;
+  SP_CUDA(el);
   if (out_mapped) return SP_OK;
   const size_t out_row = (size_t)g->maxN * 4;
   if (h_acc)
@@ -731,6 +753,8 @@ sp_status spike_proj_group_decode_lif(sp_group_t g, const float* v_in, float* v_
   q.lif_ld_bits = ld_bits;
   q.spikes = nullptr;
   q.ld_spikes = 0;
+  q.fault = g->fault;
+  g->fault = 0;
   const cudaError_t e = launch_gather(q, s);
   if (e != cudaErrorNotSupported) {
     SP_CUDA(e);
@@ -802,8 +826,21 @@ sp_status spike_proj_decode_noalloc(const int8_t* W, int64_t ldw, const float* s
   g.ld_out = N;
   g.ws = scratch;
   g.tickets = reinterpret_cast<uint32_t*>(scratch + kNoallocMaxN);
-  g.err = scratch + kNoallocMaxN + kNoallocTickets;
+  g.err = nullptr;                        // the gather kernel never raises one
   SP_CUDA(launch_gather(g, s));
+  return SP_OK;
+}
+
+sp_status spike_proj_plan_inject_fault(sp_plan_t plan, int32_t fault) {
+  if (!plan || fault < SP_FAULT_NONE || fault > SP_FAULT_STALL) return SP_EINVAL;
+  plan->fault = fault;
+  return SP_OK;
+}
+
+sp_status spike_proj_group_inject_fault(sp_group_t group, int32_t fault) {
+  if (!group || fault < SP_FAULT_NONE || fault > SP_FAULT_STALL) return SP_EINVAL;
+  if (fault == SP_FAULT_STALL) return SP_EUNSUPPORTED;
+  group->fault = fault;
   return SP_OK;
 }
 

@@ -305,6 +305,10 @@ gather_kernel(const __grid_constant__ GatherParamsT<NP> p) {
   const int o = threadIdx.x * 4;
   const int n = n0 + o;                     // N % 16 == 0: the 4 channels are all valid or none
   if (kch == 1) {
+    if (p.fault == kFaultAbort) {           // test fault: the output stays unwritten
+      if (threadIdx.x == 0) atomicExch(p.err, kErrInjected);
+      return;
+    }
     if (n < P.N) write4(P, acc_row, y_row, n, unit_sum4(sm, o));
     return;
   }
@@ -326,7 +330,11 @@ gather_kernel(const __grid_constant__ GatherParamsT<NP> p) {
     uint32_t* tk = p.tickets + (int64_t)P.ticket_begin * p.B + (int64_t)t * ntile + nt;
     __threadfence();
     const uint32_t prev = atomicAdd(tk, 1u);
-    const int last = prev == (uint32_t)(kch - 1);
+    int last = prev == (uint32_t)(kch - 1);
+    if (last && p.fault == kFaultAbort) {   // test fault: workspace and ticket left dirty
+      atomicExch(p.err, kErrInjected);
+      last = 0;
+    }
     if (last) {
       atomicExch(tk, 0u);                   // every chunk has arrived: reset
       __threadfence();
@@ -437,6 +445,10 @@ gather_cluster_kernel(const __grid_constant__ GatherParamsT<NP> p) {
   cluster_sync_all();                       // every partial is in its owner's shared memory
   const int g_own = kc * per + threadIdx.x; // this thread's owned group (a contiguous run)
   const int n = n0 + 4 * g_own;
+  if (p.fault == kFaultAbort) {             // test fault: the output stays unwritten
+    if (work && threadIdx.x == 0) atomicExch(p.err, kErrInjected);
+    return;
+  }
   if (work && (int)threadIdx.x < per && g_own < kGatherNT / 4 && n < P.N) {
     int4 s = make_int4(0, 0, 0, 0);
     for (int q = 0; q < kch; ++q) {

@@ -248,6 +248,8 @@ gemm_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CU
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
+  // wait bound: a launch with the test stall fault gives up after ~2 ms
+  const long long lim = a.p.fault == kFaultStall ? kStallWaitCycles : kWaitLimitCycles;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
@@ -285,14 +287,18 @@ gemm_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CU
         int tile, mb, nb, kb0, kb1;
         unit_coords(a, u, tile, mb, nb, kb0, kb1);
         for (int kb = kb0; kb < kb1; ++kb) {
-          if (!mbar_wait(&empty[stage], ph ^ 1u)) {
+          if (!mbar_wait(&empty[stage], ph ^ 1u, lim)) {
             *s_abort = 1;
             atomicExch(a.p.err, kErrMbarTimeout);
             break;
           }
           mbar_arrive_expect_tx(&full[stage], STAGE_BYTES);
-          tma_load_2d(sA + (size_t)stage * A_BYTES, &mapA, &full[stage], kb * BK, mb * BM);
-          tma_load_2d(sB + (size_t)stage * B_BYTES, &mapB, &full[stage], kb * 2 * BK, nb * BN);
+          // test stall fault: CTA 0's first fill is never issued, so its
+          // MMA warp's bounded wait runs out
+          if (!(a.p.fault == kFaultStall && blockIdx.x == 0 && issued == 0)) {
+            tma_load_2d(sA + (size_t)stage * A_BYTES, &mapA, &full[stage], kb * BK, mb * BM);
+            tma_load_2d(sB + (size_t)stage * B_BYTES, &mapB, &full[stage], kb * 2 * BK, nb * BN);
+          }
           ++issued;
           if (++stage == STAGES) { stage = 0; ph ^= 1u; }
         }
@@ -303,7 +309,7 @@ gemm_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CU
       uint32_t q = ph;
       for (int i = 0; i < STAGES && i < issued; ++i) {
         if (--s < 0) { s = STAGES - 1; q ^= 1u; }
-        mbar_wait(&full[s], q);
+        mbar_wait(&full[s], q, lim);
       }
     }
   } else if (warp == 1) {
@@ -316,7 +322,7 @@ gemm_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CU
       for (int u = blockIdx.x; u < a.units && !*s_abort; u += gridDim.x) {
         int tile, mb, nb, kb0, kb1;
         unit_coords(a, u, tile, mb, nb, kb0, kb1);
-        if (!mbar_wait(&tempty[ab], aph ^ 1u)) {
+        if (!mbar_wait(&tempty[ab], aph ^ 1u, lim)) {
           *s_abort = 1;
           atomicExch(a.p.err, kErrMbarTimeout);
           break;
@@ -325,7 +331,7 @@ gemm_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CU
         const uint32_t d = tmem_base + (uint32_t)(ab * BN);
         bool ok = true;
         for (int kb = kb0; kb < kb1; ++kb) {
-          if (!mbar_wait(&full[stage], ph)) {
+          if (!mbar_wait(&full[stage], ph, lim)) {
             ok = false;
             break;
           }
@@ -351,7 +357,7 @@ gemm_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CU
         if (++ab == 2) { ab = 0; aph ^= 1u; }
       }
       mma_commit(done);                      // retire every issued MMA
-      mbar_wait(done, 0);
+      mbar_wait(done, 0, lim);
     }
   } else if (a.splits == 1) {
     if (warp < 6) {                           // the whole-K epilogue uses warps 2-5
@@ -366,7 +372,7 @@ gemm_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CU
       for (int u = blockIdx.x; u < a.units; u += gridDim.x) {
         int tile, mb, nb, kb0, kb1;
         unit_coords(a, u, tile, mb, nb, kb0, kb1);
-        if (!mbar_wait(&tfull[ab], aph)) {
+        if (!mbar_wait(&tfull[ab], aph, lim)) {
           *s_abort = 1;
           if (lane == 0) atomicExch(a.p.err, kErrMbarTimeout);
           break;
@@ -376,6 +382,10 @@ gemm_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CU
         for (int c = 0; c < BN; c += 32) {
           uint32_t v[32];
           tmem_ld32(tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(ab * BN + c), v);
+          if (a.p.fault == kFaultAbort) {    // test fault: the output stays unwritten
+            if (lane == 0) atomicExch(a.p.err, kErrInjected);
+            continue;
+          }
           store_chunk(a.p, tr, v, row0, nb * BN + c, column_scale(a.p, nb * BN + c + lane));
         }
         tc_fence_before();
@@ -387,7 +397,7 @@ gemm_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CU
   } else {
     // ---------------- epilogue (split K): reduce-scatter through L2 -----------
     // One unit per CTA.  Wait for this CTA's accumulator.
-    if (mbar_wait(&tfull[0], 0)) {
+    if (mbar_wait(&tfull[0], 0, lim)) {
       tc_fence_after();
     } else {
       *s_abort = 1;
@@ -459,7 +469,7 @@ gemm_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CU
       for (int j = 0; j < kMaxOwned; ++j) {
         const int c = rank + j * S;
         if (c >= BN / 32) break;
-        if (!mbar_wait(&pfull[j], 0)) {
+        if (!mbar_wait(&pfull[j], 0, lim)) {
           *s_abort = 1;
           if (lane == 0) atomicExch(a.p.err, kErrMbarTimeout);
           break;
@@ -472,6 +482,10 @@ gemm_kernel(const __grid_constant__ CUtensorMap mapA, const __grid_constant__ CU
                              q * 1024 + half * 16 * 32 + lane;
 #pragma unroll
           for (int i = 0; i < 16; ++i) v[i] = __float_as_uint(__uint_as_float(v[i]) + src[i * 32]);
+        }
+        if (a.p.fault == kFaultAbort) {      // test fault: the output stays unwritten
+          if (lane == 0) atomicExch(a.p.err, kErrInjected);
+          continue;
         }
         store_block16(a.p, tr, v, mb * BM + q * 32, nb * BN + c * 32 + half * 16, sc[j]);
       }
@@ -805,6 +819,10 @@ gemm_group_kernel(const __grid_constant__ GemmGroupArgs g) {
 #pragma unroll
               for (int i = 0; i < 16; ++i)
                 v[i] = __float_as_uint(__uint_as_float(v[i]) + __ldcg(src + (size_t)i * 128));
+            }
+            if (M.p.fault == kFaultAbort) {   // test fault: the output stays unwritten
+              if (lane == 0) atomicExch(g.err, kErrInjected);
+              continue;
             }
             store_block16(M.p, tr, v, row0, col0, column_scale(M.p, col0 + (lane & 15)));
           }

@@ -33,7 +33,17 @@ enum DeviceError : int {
   kErrMbarTimeout = 2,    // a bounded mbarrier wait ran out (GEMM)
   kErrTmemAlloc = 3,      // tensor-memory allocation returned an odd address
   kErrFlagTimeout = 4,    // a bounded wait for another CTA's partial ran out (GEMM)
+  kErrInjected = 5,       // a test fault (spike_proj_*_inject_fault) stopped the launch
 };
+
+// Test faults armed for the next launch of a plan or group (sp_fault).
+enum Fault : int {
+  kFaultNone = 0,
+  kFaultAbort = 1,        // the launch raises kErrInjected and leaves its output unwritten
+  kFaultStall = 2,        // GEMM: one TMA copy is never issued; waits bounded by kStallWait
+};
+// Wait bound of a launch with kFaultStall (SM cycles, about 2 ms).
+constexpr long long kStallWaitCycles = 1ll << 22;
 
 // One projection as the gather kernel sees it.
 struct GatherProblem {
@@ -86,6 +96,7 @@ struct GatherParamsT {
   // spike row is made inside the kernel by one LIF step of row j of
   // (lif_vin, lif_I); the new state goes to lif_vout (and the spike words to
   // lif_bits when set), each element by exactly one CTA
+  int32_t fault = 0;      // Fault armed for this launch (kFaultAbort)
   const float* lif_vin = nullptr;
   float* lif_vout = nullptr;
   const float* lif_I = nullptr;
@@ -116,6 +127,7 @@ struct UnionParams {
   int32_t* ws;            // [B][N]
   uint32_t* tickets;      // [ceil(N/kUnionNT)]
   int* err;
+  int32_t fault;          // Fault armed for this launch (kFaultAbort)
 };
 constexpr int kUnionMaxRows = 256;      // rows per union launch
 
@@ -128,6 +140,7 @@ struct GemmParams {
   int* err;
   float* part;            // split-K partials, part_units x (128 x 256) fp32
   int32_t part_units;
+  int32_t fault;          // Fault armed for this launch
 };
 
 // One continuous-input projection as the dense kernel sees it (row-major

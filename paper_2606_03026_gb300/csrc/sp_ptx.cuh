@@ -38,13 +38,15 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
       : "memory");
   return ok != 0;
 }
-// Bounded wait for the phase with the given parity; false on timeout.
-static __device__ __noinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
+// Bounded wait for the phase with the given parity; false on timeout (after
+// `limit` SM cycles).
+static __device__ __noinline__ bool mbar_wait(uint64_t* bar, uint32_t parity,
+                                              long long limit = kWaitLimitCycles) {
   const long long t0 = clock64();
   for (;;) {
     for (int i = 0; i < 16; ++i)
       if (mbar_try_wait(bar, parity)) return true;
-    if (clock64() - t0 > kWaitLimitCycles) return false;
+    if (clock64() - t0 > limit) return false;
   }
 }
 __device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, uint64_t* bar,

@@ -116,7 +116,9 @@ union_kernel(const __grid_constant__ UnionParams p) {
       int o[8];
       unbias16(ev0, od0, n, o);
       unbias16(ev1, od1, n, o + 4);
-      if (ch < p.N) {
+      if (ch < p.N && p.fault == kFaultAbort && kch == 1) {
+        if (lane == 0) atomicExch(p.err, kErrInjected);   // test fault: output unwritten
+      } else if (ch < p.N) {
         if (kch == 1) {
 #pragma unroll
           for (int q = 0; q < 8; ++q) {
@@ -140,7 +142,11 @@ union_kernel(const __grid_constant__ UnionParams p) {
       __syncthreads();
       if (threadIdx.x == 0) {
         const uint32_t prev = atomicAdd(p.tickets + nt, 1u);
-        const int last = prev == (uint32_t)(kch - 1);
+        int last = prev == (uint32_t)(kch - 1);
+        if (last && p.fault == kFaultAbort) {   // test fault: workspace and ticket left dirty
+          atomicExch(p.err, kErrInjected);
+          last = 0;
+        }
         if (last) atomicExch(p.tickets + nt, 0u);
         s_last = last;
       }

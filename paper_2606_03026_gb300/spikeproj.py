@@ -19,6 +19,8 @@ SP_OK, SP_EINVAL, SP_EALIGN, SP_EDEVICE, SP_ECUDA, SP_ENOMEM, SP_ERANGE, \
 SP_SPIKES_BITS32, SP_SPIKES_U8, SP_SPIKES_BOOL8 = 0, 1, 2
 # sp_kernel
 SP_AUTO, SP_GATHER, SP_UNION, SP_GEMM = 0, 1, 2, 3
+# sp_fault (tests of the error path only)
+SP_FAULT_NONE, SP_FAULT_ABORT, SP_FAULT_STALL = 0, 1, 2
 SP_PLAN_GEMM = 0x1
 SPIKE_PROJ_MAX_K = 131072
 SPIKE_PROJ_MAX_GROUP = 64
@@ -60,6 +62,8 @@ _SIGNATURES = {
     "spike_proj_head": ([_P, _P, _I64, _I32, ctypes.c_float, _I32, _P, _P, _P, _P, _P, _P, _I64,
                          _P], ctypes.c_int),
     "spike_proj_probe_gather": ([_P, _P, _I32, _I32, _P, _P], ctypes.c_int),
+    "spike_proj_plan_inject_fault": ([_P, _I32], ctypes.c_int),
+    "spike_proj_group_inject_fault": ([_P, _I32], ctypes.c_int),
     "spike_proj_strerror": ([ctypes.c_int], ctypes.c_char_p),
     "spike_proj_last_cuda_error": ([], ctypes.c_int),
     "spike_proj_abi_version": ([], ctypes.c_int),
@@ -281,6 +285,16 @@ def spike_proj_probe_gather(base, offsets16, count, sink, piece_bytes=512, strea
                                          _addr(sink), _stream(stream)), "spike_proj_probe_gather")
 
 
+def spike_proj_plan_inject_fault(plan, fault):
+    """Tests of the error path only: arm a fault for the plan's next launch."""
+    _check(lib().spike_proj_plan_inject_fault(plan, fault), "spike_proj_plan_inject_fault")
+
+
+def spike_proj_group_inject_fault(group, fault):
+    """Tests of the error path only: arm a fault for the group's next launch."""
+    _check(lib().spike_proj_group_inject_fault(group, fault), "spike_proj_group_inject_fault")
+
+
 def spike_proj_strerror(status) -> str:
     return lib().spike_proj_strerror(status).decode()
 
@@ -319,6 +333,10 @@ class Plan:
 
     def status(self, stream=None) -> int:
         return spike_proj_plan_status(self.handle, stream)
+
+    def inject_fault(self, fault):
+        """Tests of the error path only (SP_FAULT_ABORT / SP_FAULT_STALL)."""
+        spike_proj_plan_inject_fault(self.handle, fault)
 
     def close(self):
         if self.handle:
@@ -362,6 +380,10 @@ class Group:
 
     def status(self, stream=None) -> int:
         return spike_proj_group_status(self.handle, stream)
+
+    def inject_fault(self, fault):
+        """Tests of the error path only (SP_FAULT_ABORT)."""
+        spike_proj_group_inject_fault(self.handle, fault)
 
     def close(self):
         if self.handle:

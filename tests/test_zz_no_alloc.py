@@ -1,5 +1,6 @@
 """The allocation-free decode entry point (fixed static scratch, no plan)
-against the plan-based spike_proj_decode, through the C ABI.
+against the plan-based spike_proj_decode and the CPU oracle, through the C
+ABI.
 
 The file name sorts last so that it also runs after every other test has
 used the library in the same process; it passes alone as well."""
@@ -9,6 +10,7 @@ import numpy as np
 import pytest
 import torch
 
+import oracle
 from gpu_util import DEV, assert_parity, to_dev
 from paper_2606_03026_gb300 import spikeproj as sp
 from paper_2606_03026_gb300 import synth
@@ -45,6 +47,7 @@ def test_noalloc_matches_plan_decode(N, K, ldq, p, fmt):
     W, S = to_dev(Qc), to_dev(s)
     plan = sp.Plan(W, S, N, K, ldw=ldq)
     rows = to_dev(synth.pack_bits(x)) if fmt == "bits" else to_dev(x)
+    ora_acc, ora_y = oracle.project(Qc, s, N, K, x, "u8", ldq=ldq)
     # two calls in a row on different spike rows: the second also shows that
     # the first left the shared scratch clean
     for t in range(2):
@@ -52,8 +55,31 @@ def test_noalloc_matches_plan_decode(N, K, ldq, p, fmt):
         acc, y = noalloc_decode(W, ldq, S, N, K, rows[t], fmt)
         torch.cuda.synchronize()
         assert_parity(acc, y, want_acc.cpu().numpy(), want_y.cpu().numpy(),
-                      f"N={N} K={K} {fmt} call {t}")
+                      f"N={N} K={K} {fmt} call {t} vs spike_proj_decode")
+        assert_parity(acc, y, ora_acc[t], ora_y[t], f"N={N} K={K} {fmt} call {t} vs oracle")
     plan.close()
+
+
+@pytest.mark.gpu
+def test_noalloc_leaves_device_memory_alone():
+    """After a first call, a few hundred more (split-K shapes included) leave
+    the device's free memory exactly as it was: nothing is allocated."""
+    cases = []
+    for (N, K, ldq) in ((1536, 1536, 1536), (2064, 8000, 2080)):
+        Qc, s, x = synth.random_case(400 + K, N, K, T=1, p=0.2, ldq=ldq)
+        cases.append((to_dev(Qc), ldq, to_dev(s), N, K, to_dev(x[0]),
+                      torch.empty(N, dtype=torch.int32, device=DEV),
+                      torch.empty(N, dtype=torch.float32, device=DEV)))
+    for (W, ldq, S, N, K, xr, acc, y) in cases:
+        sp.spike_proj_decode_noalloc(W, ldq, S, N, K, xr, "u8", acc, y)
+    torch.cuda.synchronize()
+    free0, _ = torch.cuda.mem_get_info()
+    for _ in range(200):
+        for (W, ldq, S, N, K, xr, acc, y) in cases:
+            sp.spike_proj_decode_noalloc(W, ldq, S, N, K, xr, "u8", acc, y)
+    torch.cuda.synchronize()
+    free1, _ = torch.cuda.mem_get_info()
+    assert free1 == free0
 
 
 @pytest.mark.gpu
