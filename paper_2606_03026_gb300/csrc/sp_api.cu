@@ -246,6 +246,27 @@ sp_status run_union(sp_plan_s* p, const void* spikes, int fmt, int B, int64_t ld
 sp_status run_gemm(sp_plan_s* p, const void* spikes, int fmt, int T, int64_t ld, int32_t* acc,
                    float* y, cudaStream_t s) {
   if (!(p->flags & SP_PLAN_GEMM)) return SP_EUNSUPPORTED;
+  // a few rows: the transposed small-T form reads the spike rows in place
+  if (const int S = gemm_small_splits(T, p->N, p->Kp)) {
+    GemmSmallArgs g;
+    g.spikes = spikes;
+    g.fmt = fmt;
+    g.ld = ld;
+    g.scale = p->scale;
+    g.acc = acc;
+    g.y = y;
+    g.T = T;
+    g.TN = ceil_div(T, 16) * 16;
+    g.N = p->N;
+    g.K = p->K;
+    g.S = S;
+    g.nkb = p->Kp / 64;
+    g.err = p->err;
+    g.fault = p->fault;
+    p->fault = 0;
+    SP_CUDA(launch_gemm_small(p->maps.p64, g, s));
+    return SP_OK;
+  }
   // 0/1 byte rows that TMA can address are the MMA's spike operand as they
   // stand; any other input is first written as 0/1 bytes into the staging copy
   const bool in_place = fmt == SP_SPIKES_BOOL8 && aligned(spikes, 16) && ld % 16 == 0;
@@ -277,20 +298,31 @@ sp_status run_gemm(sp_plan_s* p, const void* spikes, int fmt, int T, int64_t ld,
 }
 
 // Measured-density dispatch between the per-token gather and the
-// tensor-core GEMM, by a cost model fitted on GB300 (K = 6144, N = 1536,
-// token rates U(0.05, 0.2), B = 1 .. 1024, weights L2-resident, graph-timed):
-//   gather ~ 5 us + active bytes (sum_t |A_t| * N) / 6.7 TB/s
-//   GEMM   ~ max(12.1 us, 11.3 us + 2 B N K ops / 1.4 PFLOP/s)   (SP_PLAN_GEMM plans)
-// (the e4m3 GEMM is flat at 12.1-12.3 us up to B = 128 and takes 25 us at
-// B = 1024).  The crossover lies near 31 k active columns, B ~ 36 at these
-// rates (measured: B = 32 gather 11.3 us / GEMM 12.3 us, B = 48 14.5 / 12.2).
-// The union fetch is never chosen automatically: it was slower than the
-// per-token gather at every batch size measured (its adds are ALU-bound, and
-// the 126 MB L2 serves the per-token re-reads of a 9.4 MB weight matrix).
+// tensor-core GEMM, by a cost model fitted on GB300 (token rates
+// U(0.05, 0.2), weights L2-resident, graph-timed, N x K in {1536 x 6144,
+// 1536 x 1536, 4096 x 1536, 1536 x 16384}, B = 1 .. 256):
+//   gather        ~ 4.2 us + 0.08 us per row after the first
+//                   + active bytes (sum_t |A_t| * N) / 6.7 TB/s
+//   GEMM, T <= 64 ~ 3.4 us + 0.33 us per K block of a CTA's K range
+//                   (ceil(Kp / 64 / S), S = the cluster size) + 0.045 us per row
+//   GEMM, T > 64  ~ max(11.3 us + 2 B N K ops / 1.4 PFLOP/s, 8.5 us + 0.55 us per 1024 of K)
+// (the GEMM only for SP_PLAN_GEMM plans).  Measured at 1536 x 6144: gather
+// 4.2 / 6.7 / 9.0 / 11.6 / 16.5 us at B = 1 / 8 / 16 / 32 / 64, small-T GEMM
+// 7.2 / 7.2 / 7.3 / 8.0 / 9.4 us, the 128-row GEMM 12.1 us at B = 65 .. 128
+// (17.5 us at K = 16384); at 1536 x 1536 the small-T GEMM wins from B = 4
+// (4.5 against 5.4 us).  The union fetch is never chosen automatically: it
+// was slower than the per-token gather at every batch size measured (its
+// adds are ALU-bound, and the 126 MB L2 serves the per-token re-reads of a
+// 9.4 MB weight matrix).
 sp_kernel choose(const sp_plan_s* p, int B, int32_t total) {
   if (!(p->flags & SP_PLAN_GEMM)) return SP_GATHER;
-  const double gather_us = 5.0 + (double)total * p->N / 6.7e6;
-  const double gemm_us = std::max(12.1, 11.3 + 2.0 * B * (double)p->N * p->K / 1.4e9);
+  const double gather_us = 4.2 + 0.08 * (B - 1) + (double)total * p->N / 6.7e6;
+  double gemm_us;
+  const int nkb = p->Kp / 64;
+  if (const int S = gemm_small_splits(B, p->N, p->Kp))
+    gemm_us = 3.4 + 0.33 * ceil_div(nkb, S) + 0.045 * B;
+  else
+    gemm_us = std::max(11.3 + 2.0 * B * (double)p->N * p->K / 1.4e9, 8.5 + 0.55 * p->K / 1024.0);
   return gemm_us < gather_us ? SP_GEMM : SP_GATHER;
 }
 

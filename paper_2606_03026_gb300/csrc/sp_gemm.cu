@@ -78,38 +78,9 @@ static_assert(kGemmSmem <= 227 * 1024, "shared memory per CTA");
 // accumulator units per spike: e4m3 0x01 = 2^-9
 constexpr float kUnitsPerSpike = 512.f;
 
-// Shared-memory matrix descriptors (tcgen05 format) of K-major operands laid
-// out by TMA with a swizzle: rows of 128 bytes (128-byte swizzle, 8-row groups
-// 1024 bytes apart) or of 64 bytes (64-byte swizzle, 8-row groups 512 bytes
-// apart).  Stage buffers are 1024-byte aligned, so the base-offset field is 0.
-// Advancing K by 32 e4m3 elements inside a swizzle row adds 32 bytes to the
-// start address.
-__device__ __forceinline__ uint64_t smem_desc(const void* p, uint32_t group_bytes, uint64_t mode) {
-  const uint64_t addr = smem_u32(p);
-  uint64_t d = (addr >> 4) & 0x3FFFull;    // start address
-  d |= (uint64_t)1 << 16;                  // leading byte offset (unused here)
-  d |= (uint64_t)(group_bytes >> 4) << 32; // stride byte offset
-  d |= (uint64_t)1 << 46;                  // descriptor version for tcgen05
-  d |= mode << 61;                         // swizzle mode
-  return d;
-}
-constexpr uint64_t kSwizzle128 = 2, kSwizzle64 = 4;
 // Instruction descriptor, kind::f8f6f4: D fp32, A and B e4m3 (format 0), both
 // K-major, N = 256, M = 128.
 constexpr uint32_t kIdesc = (1u << 4) | ((uint32_t)(BN >> 3) << 17) | ((uint32_t)(BM >> 4) << 24);
-
-__device__ __forceinline__ uint32_t cluster_ctarank() {
-  uint32_t r;
-  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
-  return r;
-}
-// Arrive + wait on the cluster barrier (release / acquire at cluster scope:
-// memory writes of every thread of the cluster before it are visible to
-// every thread of the cluster after it).  Every thread of every CTA of the
-// cluster executes it.
-__device__ __forceinline__ void cluster_sync() {
-  asm volatile("barrier.cluster.arrive.release;\n\tbarrier.cluster.wait.acquire;" ::: "memory");
-}
 
 // Split-K exchange: one partial chunk (32 columns x 128 rows fp32) is 16 KB;
 // a rank owns at most kMaxOwned of the CPT chunks of a tile (S >= 2), and the
@@ -1049,7 +1020,9 @@ cudaError_t gemm_make_maps(const uint8_t* Xs, int rows_alloc, const uint8_t* Wq,
   if (!encode_u8_2d(&out->b, Wq, (uint64_t)2 * Kp, (uint64_t)N, (uint64_t)2 * Kp, 2 * BK, BN,
                     CU_TENSOR_MAP_SWIZZLE_128B) ||
       !encode_u8_2d(&out->b128, Wq, (uint64_t)2 * Kp, (uint64_t)N, (uint64_t)2 * Kp, 2 * BK,
-                    BN / 2, CU_TENSOR_MAP_SWIZZLE_128B))
+                    BN / 2, CU_TENSOR_MAP_SWIZZLE_128B) ||
+      !encode_u8_2d(&out->p64, Wq, (uint64_t)2 * Kp, (uint64_t)N, (uint64_t)2 * Kp, BK, BN / 2,
+                    CU_TENSOR_MAP_SWIZZLE_64B))
     return cudaErrorUnknown;
   return cudaSuccess;
 }

@@ -14,6 +14,7 @@ struct GemmMaps {
   CUtensorMap a;
   CUtensorMap b;          // 256-row boxes (one output tile's channels)
   CUtensorMap b128;       // the same operand in 128-row boxes (half a tile)
+  CUtensorMap p64;        // one plane of one K block: 128 rows x 64 bytes, 64-byte swizzle
 };
 
 int gemm_k_pad(int K);                  // K rounded up to the 64-column K block
@@ -37,6 +38,35 @@ int gemm_splits(int T, int N, int Kp, int part_units);
 // of X (gemm_make_maps) or the caller's 0/1 rows (gemm_make_rows_map).
 cudaError_t launch_gemm(const CUtensorMap& mapA, const CUtensorMap& mapB, int S, int T, int N,
                         int Kp, const GemmParams& p, cudaStream_t s);
+
+// Small-T form (sp_gemm_small.cu): T <= kGemmSmallMaxT spike rows in any
+// input format, read directly (no staging copy), the product computed
+// transposed (128 output channels per CTA as the MMA's M, the tokens as its
+// N) with K split over a cluster of S in {1, 2, 4, 8} CTAs that reduces
+// through distributed shared memory.  Each CTA holds the 0 / 1 bytes of its K
+// range of all T rows, at most kGemmSmallMaxKB K blocks of 64 columns.
+constexpr int kGemmSmallMaxT = 64;
+constexpr int kGemmSmallMaxS = 8;
+constexpr int kGemmSmallMaxKB = 16;
+struct GemmSmallArgs {
+  const void* spikes;     // row t at spikes + t * ld elements (sp_fmt)
+  int32_t fmt;
+  int64_t ld;
+  const float* scale;
+  int32_t* acc;           // [T][N] or null
+  float* y;               // [T][N] or null
+  int32_t T, TN;          // rows, and the MMA's N (T rounded up to 16)
+  int32_t N, K;
+  int32_t S;              // K ranges = cluster size
+  int32_t nkb;            // Kp / 64
+  int* err;
+  int32_t fault;          // Fault armed for this launch
+};
+// K splits of the small-T form for this shape, 0 when it does not apply
+// (T > kGemmSmallMaxT, or K too long for the per-CTA spike slice).
+int gemm_small_splits(int T, int N, int Kp);
+// mapW: the weight planes, one plane of one K block per box (GemmMaps::p64).
+cudaError_t launch_gemm_small(const CUtensorMap& mapW, const GemmSmallArgs& a, cudaStream_t s);
 
 // Grouped form: the output tiles of up to kGemmMaxMembers independent
 // contractions (one per plan of a group, each with its own operands, sizes

@@ -38,6 +38,18 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
       : "memory");
   return ok != 0;
 }
+// Non-blocking test of the phase with the given parity.
+__device__ __forceinline__ bool mbar_test(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
 // Bounded wait for the phase with the given parity; false on timeout (after
 // `limit` SM cycles).
 static __device__ __noinline__ bool mbar_wait(uint64_t* bar, uint32_t parity,
@@ -46,6 +58,27 @@ static __device__ __noinline__ bool mbar_wait(uint64_t* bar, uint32_t parity,
   for (;;) {
     for (int i = 0; i < 16; ++i)
       if (mbar_try_wait(bar, parity)) return true;
+    if (clock64() - t0 > limit) return false;
+  }
+}
+// The same bounded wait with the thread suspended inside try_wait until the
+// phase completes (or a time hint of about 20 us passes, when the bound is
+// checked again), instead of re-polling: a polling thread issues a
+// shared-memory instruction every few cycles and slows the loads, stores and
+// async copies of every other warp of the SM.
+static __device__ __noinline__ bool mbar_wait_sleep(uint64_t* bar, uint32_t parity,
+                                                    long long limit = kWaitLimitCycles) {
+  const long long t0 = clock64();
+  for (;;) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(smem_u32(bar)), "r"(parity), "r"(20000u)
+        : "memory");
+    if (ok) return true;
     if (clock64() - t0 > limit) return false;
   }
 }
@@ -101,6 +134,36 @@ __device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t cols) {
   asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(cols)
                : "memory");
 }
+// Shared-memory matrix descriptor (tcgen05 format) of a K-major operand laid
+// out with a swizzle: rows of 128 bytes (128-byte swizzle, 8-row groups 1024
+// bytes apart) or of 64 bytes (64-byte swizzle, 8-row groups 512 bytes
+// apart).  Operand buffers are 1024-byte aligned, so the base-offset field is
+// 0.  Advancing K by 32 e4m3 elements inside a swizzle row adds 32 bytes to
+// the start address.
+__device__ __forceinline__ uint64_t smem_desc(const void* p, uint32_t group_bytes, uint64_t mode) {
+  const uint64_t addr = smem_u32(p);
+  uint64_t d = (addr >> 4) & 0x3FFFull;    // start address
+  d |= (uint64_t)1 << 16;                  // leading byte offset (unused here)
+  d |= (uint64_t)(group_bytes >> 4) << 32; // stride byte offset
+  d |= (uint64_t)1 << 46;                  // descriptor version for tcgen05
+  d |= mode << 61;                         // swizzle mode
+  return d;
+}
+constexpr uint64_t kSwizzle128 = 2, kSwizzle64 = 4;
+
+__device__ __forceinline__ uint32_t cluster_ctarank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+// Arrive + wait on the cluster barrier (release / acquire at cluster scope:
+// memory writes of every thread of the cluster before it are visible to
+// every thread of the cluster after it).  Every thread of every CTA of the
+// cluster executes it.
+__device__ __forceinline__ void cluster_sync() {
+  asm volatile("barrier.cluster.arrive.release;\n\tbarrier.cluster.wait.acquire;" ::: "memory");
+}
+
 // D (+)= A B^T for e4m3 A and B in shared memory (descriptors), fp32 D in
 // tensor memory; accumulate = 0 overwrites D.
 __device__ __forceinline__ void mma_e4m3(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc,
@@ -179,6 +242,13 @@ __device__ __forceinline__ void reg_pin(uint32_t (&v)[32]) {
                  "+r"(v[30]), "+r"(v[31])
                :
                : "memory");
+}
+// 4 columns of this warp's 32 TMEM lanes (lane = row, v[i] = column i).
+__device__ __forceinline__ void tmem_ld4(uint32_t taddr, uint32_t (&v)[4]) {
+  asm volatile("tcgen05.ld.sync.aligned.32x32b.x4.b32 {%0, %1, %2, %3}, [%4];"
+               : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3])
+               : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
 // 16 columns of this warp's 32 TMEM lanes (lane = row, v[i] = column i).
 __device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&v)[16]) {

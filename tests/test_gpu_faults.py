@@ -102,6 +102,23 @@ def test_gemm_stall(down):
     check_recovery(plan, call, want_acc, want_y, "gemm stall", fault=sp.SP_FAULT_STALL)
 
 
+def test_small_gemm_stall(down):
+    """A few rows on the tensor cores (the small-T form, K split over a
+    cluster): CTA 0's first weight box is never issued, its MMA thread's
+    bounded wait runs out, and the cluster still completes its barriers."""
+    Qc, s, plan = down
+    _, _, x = synth.random_case(19, 1536, 6144, T=5, p=0.15)
+    want_acc, want_y = oracle.project(Qc, s, 1536, 6144, x, "u8")
+    xd = to_dev(x)
+
+    def call():
+        acc, y = outputs(5, 1536)
+        plan.batched(xd, "u8", 5, 6144, acc, y, "gemm")
+        return acc, y
+
+    check_recovery(plan, call, want_acc, want_y, "small gemm stall", fault=sp.SP_FAULT_STALL)
+
+
 def test_group_abort():
     """A decode step's group (ticket-free cluster form) and the grouped
     prefill (tail split: owners and helpers exchange partials behind flags)."""
