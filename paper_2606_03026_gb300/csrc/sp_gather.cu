@@ -233,17 +233,22 @@ __device__ __forceinline__ int4 unit_sum4(const UnitSmem<W, MAXCK, S>& sm, int o
   return s;
 }
 
-__device__ __forceinline__ void write4(const GatherProblem& P, int32_t* acc_row, float* y_row,
-                                       int n, int4 v) {
+// Scales of channels n .. n + 3 (read only where y is written).
+__device__ __forceinline__ float4 scale4(const GatherProblem& P, int n) {
+  return make_float4(__ldg(P.scale + n), __ldg(P.scale + n + 1), __ldg(P.scale + n + 2),
+                     __ldg(P.scale + n + 3));
+}
+
+// acc and y = s * float(acc) of channels n .. n + 3, sc = their scales.
+__device__ __forceinline__ void write4(int32_t* acc_row, float* y_row, int n, int4 v, float4 sc) {
   // one 16-byte store each where the rows allow it (the output may also be
   // page-locked host memory, where every transaction crosses the link)
   const bool v4 = ((reinterpret_cast<uintptr_t>(acc_row) | reinterpret_cast<uintptr_t>(y_row)) & 15u) == 0;
   if (v4) {
     if (acc_row) *reinterpret_cast<int4*>(acc_row + n) = v;
     if (y_row)
-      *reinterpret_cast<float4*>(y_row + n) =
-          make_float4(scale_out(__ldg(P.scale + n), v.x), scale_out(__ldg(P.scale + n + 1), v.y),
-                      scale_out(__ldg(P.scale + n + 2), v.z), scale_out(__ldg(P.scale + n + 3), v.w));
+      *reinterpret_cast<float4*>(y_row + n) = make_float4(
+          scale_out(sc.x, v.x), scale_out(sc.y, v.y), scale_out(sc.z, v.z), scale_out(sc.w, v.w));
     return;
   }
   if (acc_row) {
@@ -253,10 +258,10 @@ __device__ __forceinline__ void write4(const GatherProblem& P, int32_t* acc_row,
     acc_row[n + 3] = v.w;
   }
   if (y_row) {
-    y_row[n] = scale_out(__ldg(P.scale + n), v.x);
-    y_row[n + 1] = scale_out(__ldg(P.scale + n + 1), v.y);
-    y_row[n + 2] = scale_out(__ldg(P.scale + n + 2), v.z);
-    y_row[n + 3] = scale_out(__ldg(P.scale + n + 3), v.w);
+    y_row[n] = scale_out(sc.x, v.x);
+    y_row[n + 1] = scale_out(sc.y, v.y);
+    y_row[n + 2] = scale_out(sc.z, v.z);
+    y_row[n + 3] = scale_out(sc.w, v.w);
   }
 }
 
@@ -309,7 +314,7 @@ gather_kernel(const __grid_constant__ GatherParamsT<NP> p) {
       if (threadIdx.x == 0) atomicExch(p.err, kErrInjected);
       return;
     }
-    if (n < P.N) write4(P, acc_row, y_row, n, unit_sum4(sm, o));
+    if (n < P.N) write4(acc_row, y_row, n, unit_sum4(sm, o), y_row ? scale4(P, n) : float4{});
     return;
   }
   // Partials go into the workspace as fp32 16-byte vector reductions (one per
@@ -345,9 +350,10 @@ gather_kernel(const __grid_constant__ GatherParamsT<NP> p) {
   if (s_last && n < P.N) {
     const float4 f = __ldcg(reinterpret_cast<const float4*>(ws + n));
     __stcg(reinterpret_cast<float4*>(ws + n), make_float4(0.f, 0.f, 0.f, 0.f));
-    write4(P, acc_row, y_row, n,
+    write4(acc_row, y_row, n,
            make_int4(__float2int_rn(f.x), __float2int_rn(f.y), __float2int_rn(f.z),
-                     __float2int_rn(f.w)));
+                     __float2int_rn(f.w)),
+           y_row ? scale4(P, n) : float4{});
   }
 }
 
@@ -403,6 +409,11 @@ gather_cluster_kernel(const __grid_constant__ GatherParamsT<NP> p) {
   const int kc = rank - ts * kch;
   const int n0 = (cl * P.tpc + ts) * kGatherNT;
   const bool work = n0 < P.N;               // tile slots past the last tile idle
+  // This thread's owned group (a contiguous run of the tile's 4-channel
+  // groups), set after the column loads (nothing extra is live across them).
+  int n = 0;
+  bool owner = false;
+  float4 sc = float4{};
   if (work) {
     if constexpr (kLif) {
       // fused spike producer: one LIF step of this chunk's neurons (every CTA
@@ -432,6 +443,14 @@ gather_cluster_kernel(const __grid_constant__ GatherParamsT<NP> p) {
     unit_partial<kGatherClusterWarps, kGatherClusterMaxCK, kClusterLoads, kClusterSlots>(
         sm, P, kLif ? nullptr : spike_row(p.spikes, p.fmt, j, p.ld_spikes), p.fmt, n0, kc * P.ck,
         P.ck, kLif ? s_lif : nullptr);
+    // the owner's scales, read now: their load overlaps the cluster exchange
+    // instead of following the last barrier
+    {
+      const int g_own = kc * per + (int)threadIdx.x;
+      n = n0 + 4 * g_own;
+      owner = (int)threadIdx.x < per && g_own < kGatherNT / 4 && n < P.N;
+    }
+    if (owner && p.y) sc = scale4(P, n);
     asm volatile("barrier.cluster.wait;" ::: "memory");
     const int g = threadIdx.x;              // the 4-channel group of this thread
     if (g < kGatherNT / 4) {
@@ -443,13 +462,11 @@ gather_cluster_kernel(const __grid_constant__ GatherParamsT<NP> p) {
   }
   if (!work) asm volatile("barrier.cluster.wait;" ::: "memory");
   cluster_sync_all();                       // every partial is in its owner's shared memory
-  const int g_own = kc * per + threadIdx.x; // this thread's owned group (a contiguous run)
-  const int n = n0 + 4 * g_own;
   if (p.fault == kFaultAbort) {             // test fault: the output stays unwritten
     if (work && threadIdx.x == 0) atomicExch(p.err, kErrInjected);
     return;
   }
-  if (work && (int)threadIdx.x < per && g_own < kGatherNT / 4 && n < P.N) {
+  if (owner) {
     int4 s = make_int4(0, 0, 0, 0);
     for (int q = 0; q < kch; ++q) {
       const int4 v = s_recv[q * per + threadIdx.x];
@@ -458,8 +475,8 @@ gather_cluster_kernel(const __grid_constant__ GatherParamsT<NP> p) {
       s.z += v.z;
       s.w += v.w;
     }
-    write4(P, p.acc ? p.acc + (int64_t)j * p.ld_out : nullptr,
-           p.y ? p.y + (int64_t)j * p.ld_out : nullptr, n, s);
+    write4(p.acc ? p.acc + (int64_t)j * p.ld_out : nullptr,
+           p.y ? p.y + (int64_t)j * p.ld_out : nullptr, n, s, sc);
   }
 }
 
