@@ -40,6 +40,8 @@ namespace sp {
 namespace {
 
 static_assert(kGatherNT == 4 * kGatherThreads, "one 4-channel vector per thread in the flush");
+static_assert((kGatherWarps & (kGatherWarps - 1)) == 0 && (kGatherClusterWarps & (kGatherClusterWarps - 1)) == 0,
+              "warp counts are powers of two (rank residues by mask)");
 static_assert(kGatherNT / 4 <= kGatherClusterThreads, "one 4-channel group per thread");
 
 __device__ __forceinline__ void cp_async16(void* smem, const void* gmem) {
@@ -150,14 +152,11 @@ __device__ __forceinline__ void unit_partial(UnitSmem<W, MAXCK, S>& sm, const Ga
   }
   const int total = __shfl_sync(0xffffffffu, incl, 31);
   {
-    uint32_t w = word;
-    int rank = incl - c;
-    while (w) {
-      const int b = __ffs(w) - 1;
-      w &= w - 1u;
-      if (rank % W == warp) sm.cols[warp][rank / W] = k0 + 32 * lane + b;
-      ++rank;
-    }
+    // this lane's bits of rank = warp (mod W): local indices i0, i0 + W, ...
+    const int r0 = incl - c;                // rank of the lane's first set bit
+    const int i0 = (warp - r0) & (W - 1);   // W is a power of two
+    for (int i = i0; i < c; i += W)
+      sm.cols[warp][(r0 + i) / W] = k0 + 32 * lane + (int)__fns(word, 0u, i + 1);
   }
   __syncwarp();
   const int mine = (total - warp + W - 1) / W;       // ranks warp, warp + W, ...
