@@ -357,12 +357,12 @@ gather_kernel(const __grid_constant__ GatherParamsT<NP> p) {
 }
 
 // ---------------------------------------------------------------------------
-// Cluster form: one token per problem, at most kGatherCluster chunks of at
-// most 1024 columns per tile.  256-thread CTAs in clusters of kGatherCluster;
-// a cluster holds tpc tiles x kch chunks of one problem (rank = tile slot *
-// kch + chunk; kch divides kGatherCluster); the grid lists the clusters one
-// by one (or is (clusters of the largest problem x kGatherCluster,
-// problems)).  The 128 4-channel groups of a tile are split into kch
+// Cluster form: one token per problem, at most CL chunks of at most 1024
+// columns per tile.  256-thread CTAs in clusters of CL (6 for a group of
+// projections; 12 or 16 for a single projection, which then spreads over more
+// SMs); a cluster holds tpc tiles x kch chunks of one problem (rank = tile
+// slot * kch + chunk; kch divides CL); the grid lists the clusters one by one
+// (or is (clusters of the largest problem x CL, problems)).  The 128 4-channel groups of a tile are split into kch
 // contiguous runs, run c owned by the CTA of chunk c: every CTA stores its
 // partial of each group into the owner's shared memory (distributed shared memory), one
 // cluster barrier (release / acquire) publishes the stores, and each owner
@@ -375,12 +375,12 @@ using ClusterSmem = UnitSmem<kGatherClusterWarps, kGatherClusterMaxCK, kClusterS
 
 // kLif: the fused spike producer (a separate instantiation, so that the plain
 // decode carries none of its code)
-template <int NP, bool kLif>
+template <int NP, bool kLif, int CL>
 __global__ void __launch_bounds__(kGatherClusterThreads, 4)
 gather_cluster_kernel(const __grid_constant__ GatherParamsT<NP> p) {
   __shared__ ClusterSmem sm;
   // [sender chunk][owned group]: kch * ceil(128 / kch) < 128 + kch entries
-  __shared__ __align__(16) int4 s_recv[kGatherNT / 4 + kGatherCluster];
+  __shared__ __align__(16) int4 s_recv[kGatherNT / 4 + CL];
   __shared__ uint32_t s_lif[kLif ? kGatherClusterMaxCK / 32 : 1];   // LIF mode: the chunk's spike words
   // every CTA of the cluster arrives here and waits (below) before its first
   // store into a peer's shared memory: the peer is then known to be running
@@ -389,8 +389,8 @@ gather_cluster_kernel(const __grid_constant__ GatherParamsT<NP> p) {
   if (blockIdx.y == 0) prefetch_spike_rows(p);   // before the wait: see gather_kernel
   pdl_wait();
 
-  const int c = (int)blockIdx.x / kGatherCluster;
-  const int rank = (int)blockIdx.x - c * kGatherCluster;   // rank in the (6, 1, 1) cluster
+  const int c = (int)blockIdx.x / CL;
+  const int rank = (int)blockIdx.x - c * CL;   // rank in the (CL, 1, 1) cluster
   int j = blockIdx.y, cl = c;
   if (p.ncl_list > 0) {                     // listed clusters: no idle CTAs
     const int e = p.cl_list[c];
@@ -495,7 +495,7 @@ cudaError_t set_carveout(Kern kernel, std::atomic<uint64_t>& done) {
 }
 
 // Clusters of the cluster form that can be resident at once (per device).
-template <int NP, bool kLif>
+template <int NP, bool kLif, int CL>
 int cluster_capacity() {
   static std::atomic<int> cap[64];
   int dev = 0;
@@ -505,14 +505,14 @@ int cluster_capacity() {
   cudaLaunchConfig_t cfg = {};
   cudaLaunchAttribute attr;
   attr.id = cudaLaunchAttributeClusterDimension;
-  attr.val.clusterDim.x = kGatherCluster;
+  attr.val.clusterDim.x = CL;
   attr.val.clusterDim.y = 1;
   attr.val.clusterDim.z = 1;
-  cfg.gridDim = dim3(kGatherCluster, 1, 1);
+  cfg.gridDim = dim3(CL, 1, 1);
   cfg.blockDim = dim3(kGatherClusterThreads, 1, 1);
   cfg.attrs = &attr;
   cfg.numAttrs = 1;
-  if (cudaOccupancyMaxActiveClusters(&n, gather_cluster_kernel<NP, kLif>, &cfg) != cudaSuccess ||
+  if (cudaOccupancyMaxActiveClusters(&n, gather_cluster_kernel<NP, kLif, CL>, &cfg) != cudaSuccess ||
       n < 1) {
     (void)cudaGetLastError();
     n = -1;
@@ -521,60 +521,122 @@ int cluster_capacity() {
   return n;
 }
 
-// Fills the cluster-form fields of q; false when the launch does not fit the
-// cluster form (several tokens, a chunk count above the cluster size, or more
-// clusters than can be resident at once).  Up to kGatherMaxClusterList
-// clusters are listed one by one (a 1-D grid of exactly the clusters with
-// work, all resident together); more take a (clusters x 6, problems) grid in
-// which the problems with fewer clusters leave idle CTAs.
+// Resident-cluster count of the kernel the launch will use (0 on failure).
 template <int NP>
-bool cluster_form(GatherParamsT<NP>& q, int* grid_x, int* grid_y) {
+int capacity_for(bool lif, int CL) {
+  if (lif) return cluster_capacity<NP, true, 6>();
+  switch (CL) {
+    case 16: return cluster_capacity<NP, false, 16>();
+    case 12: return cluster_capacity<NP, false, 12>();
+    default: return cluster_capacity<NP, false, 6>();
+  }
+}
+
+// Fills the cluster-form fields of q and the cluster size *cl_out; false
+// when the launch does not fit the cluster form (several tokens, a chunk
+// count above the cluster size, or more clusters than can be resident at
+// once).  A group of projections takes clusters of 6 and the fewest chunks
+// of at most 1024 columns.  A single projection (which alone would leave
+// most SMs idle) takes the cluster size and chunking with the most working
+// CTAs among clusters of 16, 12 and 6, chunks of 256 to 1024 columns and at
+// most a quarter of the tile slots idle.  Up to kGatherMaxClusterList
+// clusters are listed one by one (a 1-D grid of exactly the clusters with
+// work, all resident together); more take a (clusters x CL, problems) grid
+// in which the problems with fewer clusters leave idle CTAs.
+template <int NP>
+bool cluster_form(GatherParamsT<NP>& q, int* grid_x, int* grid_y, int* cl_out) {
   if (q.B != 1) return false;
+  int CL = 6;
+  if (q.nprob == 1 && !q.lif_I) {
+    GatherProblem& P = q.prob[0];
+    const int ntiles = gather_ntiles(P.N);
+    int best = 0;
+    for (const int cand : {16, 12, 6}) {
+      for (int kch = cand; kch >= 1; --kch) {
+        if (cand % kch != 0) continue;
+        const int ck = ceil_div(ceil_div(P.K, kch), 32) * 32;
+        if (ck > kGatherClusterMaxCK || (ck < 256 && kch > 1)) continue;
+        const int tpc = cand / kch;
+        const int ncl = ceil_div(ntiles, tpc);
+        if (4 * (ncl * tpc - ntiles) > ncl * tpc) continue;   // more than a quarter idle
+        const int working = ntiles * kch;
+        if (working > best) {
+          best = working;
+          CL = cand;
+          P.kch = kch;
+        }
+        break;                              // the most chunks this size allows
+      }
+    }
+    if (best == 0) return false;
+    P.ck = ceil_div(ceil_div(P.K, P.kch), 32) * 32;
+    P.tpc = CL / P.kch;
+    P.ncl = ceil_div(ntiles, P.tpc);
+  } else {
+    for (int j = 0; j < q.nprob; ++j) {
+      GatherProblem& P = q.prob[j];
+      // the fewest chunks (a divisor of the cluster size) of at most 1024 columns
+      int kch = 0;
+      for (int d = 1; d <= CL; ++d)
+        if (CL % d == 0 && ceil_div(P.K, d) <= kGatherClusterMaxCK) {
+          kch = d;
+          break;
+        }
+      if (kch == 0) return false;
+      P.kch = kch;
+      P.ck = ceil_div(ceil_div(P.K, kch), 32) * 32;
+      P.tpc = CL / kch;
+      P.ncl = ceil_div(gather_ntiles(P.N), P.tpc);
+    }
+  }
   int total = 0, widest = 0;
   for (int j = 0; j < q.nprob; ++j) {
-    GatherProblem& P = q.prob[j];
-    // the fewest chunks (a divisor of the cluster size) of at most 1024 columns
-    int kch = 0;
-    for (int d = 1; d <= kGatherCluster; ++d)
-      if (kGatherCluster % d == 0 && ceil_div(P.K, d) <= kGatherClusterMaxCK) {
-        kch = d;
-        break;
-      }
-    if (kch == 0) return false;
-    P.kch = kch;
-    P.ck = ceil_div(ceil_div(P.K, kch), 32) * 32;
-    P.tpc = kGatherCluster / kch;
-    P.ncl = ceil_div(gather_ntiles(P.N), P.tpc);
-    total += P.ncl;
-    if (P.ncl > widest) widest = P.ncl;
+    total += q.prob[j].ncl;
+    if (q.prob[j].ncl > widest) widest = q.prob[j].ncl;
   }
-  if (total > (q.lif_I ? cluster_capacity<NP, true>() : cluster_capacity<NP, false>())) return false;
+  if (total > capacity_for<NP>(q.lif_I != nullptr, CL)) return false;
   q.ncl_list = 0;
   if (total <= kGatherMaxClusterList && widest <= 0xff) {
     int c = 0;
     for (int j = 0; j < q.nprob; ++j)
       for (int cl = 0; cl < q.prob[j].ncl; ++cl) q.cl_list[c++] = (uint16_t)((j << 8) | cl);
     q.ncl_list = total;
-    *grid_x = total * kGatherCluster;
+    *grid_x = total * CL;
     *grid_y = 1;
   } else {
-    *grid_x = widest * kGatherCluster;
+    *grid_x = widest * CL;
     *grid_y = q.nprob;
   }
+  *cl_out = CL;
   return true;
+}
+
+// Sets the one-time attributes of a cluster-form kernel: the largest
+// shared-memory carveout (the resident-cluster count depends on it) and, for
+// clusters above 8 CTAs, the non-portable cluster size.
+template <typename Kern>
+cudaError_t cluster_attrs(Kern kernel, int CL, std::atomic<uint64_t>& done) {
+  cudaError_t e = set_carveout(kernel, done);
+  if (e == cudaSuccess && CL > 8)
+    e = cudaFuncSetAttribute(kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+  return e;
 }
 
 template <int NP>
 cudaError_t launch_gather_t(const GatherParamsT<NP>& p, cudaStream_t s) {
-  static std::atomic<uint64_t> carve_t{0}, carve_c{0}, carve_l{0};
+  static std::atomic<uint64_t> carve_t{0}, carve_c{0}, carve_l{0}, carve_12{0}, carve_16{0};
   if (p.units_total <= 0 || p.B <= 0 || p.max_units <= 0) return cudaSuccess;
-  // the carveout first: the resident-cluster count depends on it
-  cudaError_t e = p.lif_I ? set_carveout(gather_cluster_kernel<NP, true>, carve_l)
-                          : set_carveout(gather_cluster_kernel<NP, false>, carve_c);
+  // the attributes first: the resident-cluster counts depend on the carveout
+  cudaError_t e = p.lif_I ? cluster_attrs(gather_cluster_kernel<NP, true, 6>, 6, carve_l)
+                          : cluster_attrs(gather_cluster_kernel<NP, false, 6>, 6, carve_c);
+  if (e == cudaSuccess && !p.lif_I && p.nprob == 1) {
+    e = cluster_attrs(gather_cluster_kernel<NP, false, 12>, 12, carve_12);
+    if (e == cudaSuccess) e = cluster_attrs(gather_cluster_kernel<NP, false, 16>, 16, carve_16);
+  }
   if (e != cudaSuccess) return e;
   GatherParamsT<NP> q = p;
-  int gx = 0, gy = 0;
-  const bool cluster = cluster_form(q, &gx, &gy);
+  int gx = 0, gy = 0, CL = 6;
+  const bool cluster = cluster_form(q, &gx, &gy, &CL);
   if (p.lif_I && !cluster) return cudaErrorNotSupported;   // the fused producer needs the cluster form
   if (cluster) {
     cudaLaunchConfig_t cfg = {};
@@ -583,15 +645,19 @@ cudaError_t launch_gather_t(const GatherParamsT<NP>& p, cudaStream_t s) {
     cfg.stream = s;
     cudaLaunchAttribute attr[2];
     attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = kGatherCluster;
+    attr[0].val.clusterDim.x = (unsigned)CL;
     attr[0].val.clusterDim.y = 1;
     attr[0].val.clusterDim.z = 1;
     attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     attr[1].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 2;
-    return p.lif_I ? cudaLaunchKernelEx(&cfg, gather_cluster_kernel<NP, true>, q)
-                   : cudaLaunchKernelEx(&cfg, gather_cluster_kernel<NP, false>, q);
+    if (p.lif_I) return cudaLaunchKernelEx(&cfg, gather_cluster_kernel<NP, true, 6>, q);
+    switch (CL) {
+      case 16: return cudaLaunchKernelEx(&cfg, gather_cluster_kernel<NP, false, 16>, q);
+      case 12: return cudaLaunchKernelEx(&cfg, gather_cluster_kernel<NP, false, 12>, q);
+      default: return cudaLaunchKernelEx(&cfg, gather_cluster_kernel<NP, false, 6>, q);
+    }
   }
   e = set_carveout(gather_kernel<NP>, carve_t);
   if (e != cudaSuccess) return e;
