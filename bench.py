@@ -35,7 +35,8 @@ Also reported on the same JSON line:
                6144 -> 1536 down projection at each spike rate (weights
                L2-resident and L2-cold), the decode step as a dependent
                chain of 44 single calls, batched B = 64 (per-token gather
-               vs union fetch, independent and correlated spikes), and the
+               vs union fetch vs the small-T tensor-core GEMM, independent and
+               correlated spikes), and the
                CPU oracle on each (single thread, bounded samples)
   clocks       nvidia-smi samples taken during the timed region and 0.5 s of
                the same step graph replayed right after it (a short timed
@@ -784,6 +785,10 @@ def bench_configs(torch, sp, synth, dev, stream, hbm, copies, spikes, sets_np, a
             row["oracle"] = {"us_per_batch": us, "tokens_per_s": 64e6 / us, "calls": n, "cores": 1}
         b4["correlated" if corr else "independent"] = row
     plan.close()
+    b4["note"] = ("gather: per-token gather (one spike row per token); union: the shared "
+                  "fetch of the union of active columns; gemm: the tensor-core form for "
+                  "T <= 64 rows (weights as the MMA's M operand, K split over a cluster of "
+                  "8; the e4m3 weight planes, 2 bytes per weight, are its bytes_fetched)")
     out["batched_b64_6144x1536"] = b4
 
     # config 5 oracle: one 512-token prefill block, extrapolated to 22 blocks

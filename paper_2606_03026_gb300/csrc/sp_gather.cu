@@ -370,15 +370,19 @@ gather_kernel(const __grid_constant__ GatherParamsT<NP> p) {
 // acc / y.  No workspace, no atomics, and no CTA reads another's shared
 // memory, so none waits for the others after the barrier.
 constexpr int kClusterLoads = 9;                   // column loads per lane in registers (64 registers)
-constexpr int kClusterSlots = 8;                   // and in shared memory
-using ClusterSmem = UnitSmem<kGatherClusterWarps, kGatherClusterMaxCK, kClusterSlots>;
+// and in shared memory: 8 for a group (4 CTAs per SM), 16 for a single
+// projection's clusters of 12 or 16 (fewer CTAs, each with more columns)
+template <int CL> constexpr int cluster_slots() { return CL > 8 ? 16 : 8; }
+template <int CL>
+using ClusterSmem = UnitSmem<kGatherClusterWarps, kGatherClusterMaxCK, cluster_slots<CL>()>;
 
 // kLif: the fused spike producer (a separate instantiation, so that the plain
 // decode carries none of its code)
 template <int NP, bool kLif, int CL>
 __global__ void __launch_bounds__(kGatherClusterThreads, 4)
 gather_cluster_kernel(const __grid_constant__ GatherParamsT<NP> p) {
-  __shared__ ClusterSmem sm;
+  extern __shared__ __align__(16) uint8_t dyn_smem[];   // ClusterSmem<CL>, sized at launch
+  ClusterSmem<CL>& sm = *reinterpret_cast<ClusterSmem<CL>*>(dyn_smem);
   // [sender chunk][owned group]: kch * ceil(128 / kch) < 128 + kch entries
   __shared__ __align__(16) int4 s_recv[kGatherNT / 4 + CL];
   __shared__ uint32_t s_lif[kLif ? kGatherClusterMaxCK / 32 : 1];   // LIF mode: the chunk's spike words
@@ -439,7 +443,7 @@ gather_cluster_kernel(const __grid_constant__ GatherParamsT<NP> p) {
       }
       __syncthreads();
     }
-    unit_partial<kGatherClusterWarps, kGatherClusterMaxCK, kClusterLoads, kClusterSlots>(
+    unit_partial<kGatherClusterWarps, kGatherClusterMaxCK, kClusterLoads, cluster_slots<CL>()>(
         sm, P, kLif ? nullptr : spike_row(p.spikes, p.fmt, j, p.ld_spikes), p.fmt, n0, kc * P.ck,
         P.ck, kLif ? s_lif : nullptr);
     // the owner's scales, read now: their load overlaps the cluster exchange
@@ -510,6 +514,7 @@ int cluster_capacity() {
   attr.val.clusterDim.z = 1;
   cfg.gridDim = dim3(CL, 1, 1);
   cfg.blockDim = dim3(kGatherClusterThreads, 1, 1);
+  cfg.dynamicSmemBytes = sizeof(ClusterSmem<CL>);
   cfg.attrs = &attr;
   cfg.numAttrs = 1;
   if (cudaOccupancyMaxActiveClusters(&n, gather_cluster_kernel<NP, kLif, CL>, &cfg) != cudaSuccess ||
@@ -615,10 +620,12 @@ bool cluster_form(GatherParamsT<NP>& q, int* grid_x, int* grid_y, int* cl_out) {
 // shared-memory carveout (the resident-cluster count depends on it) and, for
 // clusters above 8 CTAs, the non-portable cluster size.
 template <typename Kern>
-cudaError_t cluster_attrs(Kern kernel, int CL, std::atomic<uint64_t>& done) {
+cudaError_t cluster_attrs(Kern kernel, int CL, size_t smem, std::atomic<uint64_t>& done) {
   cudaError_t e = set_carveout(kernel, done);
   if (e == cudaSuccess && CL > 8)
     e = cudaFuncSetAttribute(kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+  if (e == cudaSuccess && smem > 48 * 1024)
+    e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   return e;
 }
 
@@ -627,11 +634,13 @@ cudaError_t launch_gather_t(const GatherParamsT<NP>& p, cudaStream_t s) {
   static std::atomic<uint64_t> carve_t{0}, carve_c{0}, carve_l{0}, carve_12{0}, carve_16{0};
   if (p.units_total <= 0 || p.B <= 0 || p.max_units <= 0) return cudaSuccess;
   // the attributes first: the resident-cluster counts depend on the carveout
-  cudaError_t e = p.lif_I ? cluster_attrs(gather_cluster_kernel<NP, true, 6>, 6, carve_l)
-                          : cluster_attrs(gather_cluster_kernel<NP, false, 6>, 6, carve_c);
+  cudaError_t e = p.lif_I
+                      ? cluster_attrs(gather_cluster_kernel<NP, true, 6>, 6, sizeof(ClusterSmem<6>), carve_l)
+                      : cluster_attrs(gather_cluster_kernel<NP, false, 6>, 6, sizeof(ClusterSmem<6>), carve_c);
   if (e == cudaSuccess && !p.lif_I && p.nprob == 1) {
-    e = cluster_attrs(gather_cluster_kernel<NP, false, 12>, 12, carve_12);
-    if (e == cudaSuccess) e = cluster_attrs(gather_cluster_kernel<NP, false, 16>, 16, carve_16);
+    e = cluster_attrs(gather_cluster_kernel<NP, false, 12>, 12, sizeof(ClusterSmem<12>), carve_12);
+    if (e == cudaSuccess)
+      e = cluster_attrs(gather_cluster_kernel<NP, false, 16>, 16, sizeof(ClusterSmem<16>), carve_16);
   }
   if (e != cudaSuccess) return e;
   GatherParamsT<NP> q = p;
@@ -652,11 +661,20 @@ cudaError_t launch_gather_t(const GatherParamsT<NP>& p, cudaStream_t s) {
     attr[1].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 2;
-    if (p.lif_I) return cudaLaunchKernelEx(&cfg, gather_cluster_kernel<NP, true, 6>, q);
+    if (p.lif_I) {
+      cfg.dynamicSmemBytes = sizeof(ClusterSmem<6>);
+      return cudaLaunchKernelEx(&cfg, gather_cluster_kernel<NP, true, 6>, q);
+    }
     switch (CL) {
-      case 16: return cudaLaunchKernelEx(&cfg, gather_cluster_kernel<NP, false, 16>, q);
-      case 12: return cudaLaunchKernelEx(&cfg, gather_cluster_kernel<NP, false, 12>, q);
-      default: return cudaLaunchKernelEx(&cfg, gather_cluster_kernel<NP, false, 6>, q);
+      case 16:
+        cfg.dynamicSmemBytes = sizeof(ClusterSmem<16>);
+        return cudaLaunchKernelEx(&cfg, gather_cluster_kernel<NP, false, 16>, q);
+      case 12:
+        cfg.dynamicSmemBytes = sizeof(ClusterSmem<12>);
+        return cudaLaunchKernelEx(&cfg, gather_cluster_kernel<NP, false, 12>, q);
+      default:
+        cfg.dynamicSmemBytes = sizeof(ClusterSmem<6>);
+        return cudaLaunchKernelEx(&cfg, gather_cluster_kernel<NP, false, 6>, q);
     }
   }
   e = set_carveout(gather_kernel<NP>, carve_t);
