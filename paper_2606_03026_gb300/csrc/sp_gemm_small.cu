@@ -15,29 +15,28 @@
 // |n| <= 128 K < 2^24, and the epilogue scales by 2^9 and converts to INT32.
 //
 // Decomposition: output tile mt (channels 128 mt ..) x S K ranges, one CTA
-// each; the S CTAs of a tile form a thread-block cluster.  Per CTA (192
+// each; the S CTAs of a tile form a thread-block cluster.  Per CTA (320
 // threads):
 //   warp 0      TMA producer: the two 128 x 64-byte weight boxes (one per
-//               plane) of each 64-column K block into an 8-stage ring.  The planes are
-//               written once, when the plan is made, so the first ring fills
-//               are issued before the dependency wait and overlap the tail of
-//               the previous kernel of the stream.
+//               plane) of each 64-column K block into an 8-stage ring.  The
+//               planes are written once, when the plan is made, so the first
+//               ring fills are issued before the dependency wait and overlap
+//               the tail of the previous kernel of the stream.
 //   warp 1      allocates 64 TMEM columns and issues the MMAs (M = 128,
 //               N = TN, K = 32; two per plane per K block) from one thread.
-//   warps 2-5   after the dependency wait, expand the CTA's K range of all T
+//   warps 2-9   after the dependency wait, expand the CTA's K range of all T
 //               spike rows (any input format) into 0 / 1 bytes in the
 //               64-byte-swizzled K-major layout the MMA reads (the layout a
-//               TMA box with 64-byte swizzle writes), K block by K block,
-//               then read the
-//               accumulator (warp w: TMEM lane quarter w % 4, i.e. 32
-//               channels x TN tokens) and reduce it over the cluster: the
-//               tokens form groups of 4, group g belongs to cluster rank
-//               g % S, every CTA pushes each group's 4 values of its 32
-//               channels into the owner's shared memory (distributed shared
-//               memory), one cluster barrier publishes the pushes, and each
-//               owner adds the S partials of its groups and writes acc / y
-//               (a warp's 32 lanes hold 32 consecutive channels of one token:
-//               128-byte stores).
+//               TMA box with 64-byte swizzle writes), K block by K block.
+//   warps 2-5   then read the accumulator (warp w: TMEM lane quarter w % 4,
+//               i.e. 32 channels x TN tokens) and reduce it over the
+//               cluster: the tokens form groups of 4, group g belongs to
+//               cluster rank g % S, every CTA pushes each group's 4 values of
+//               its 32 channels into the owner's shared memory (distributed
+//               shared memory), one cluster barrier publishes the pushes, and
+//               each owner adds the S partials of its groups and writes acc /
+//               y (a warp's 32 lanes hold 32 consecutive channels of one
+//               token: 128-byte stores).
 // No workspace, no atomics, no flags: the only inter-CTA waits are the two
 // cluster barriers, which every thread of every CTA reaches after bounded
 // work.  Every mbarrier wait is bounded; on timeout the CTA raises the error
