@@ -32,15 +32,17 @@
 //               i.e. 32 channels x TN tokens) and reduce it over the
 //               cluster: the tokens form groups of 4, group g belongs to
 //               cluster rank g % S, every CTA pushes each group's 4 values of
-//               its 32 channels into the owner's shared memory (distributed
-//               shared memory), one cluster barrier publishes the pushes, and
-//               each owner adds the S partials of its groups and writes acc /
-//               y (a warp's 32 lanes hold 32 consecutive channels of one
+//               its 32 channels into the owner's shared memory with st.async
+//               (distributed shared memory), which counts the bytes on the
+//               owner's receive mbarrier; the owner waits on that barrier
+//               alone, adds the S partials of its groups and writes acc / y
+//               (a warp's 32 lanes hold 32 consecutive channels of one
 //               token: 128-byte stores).
-// No workspace, no atomics, no flags: the only inter-CTA waits are the two
-// cluster barriers, which every thread of every CTA reaches after bounded
-// work.  Every mbarrier wait is bounded; on timeout the CTA raises the error
-// word, stops issuing, drains its copies and frees its tensor memory.
+// No workspace, no atomics, no flags: the inter-CTA waits are one cluster
+// barrier (every peer has staged its spike slice, so its receive area is
+// free) and the receive mbarriers.  Every mbarrier wait is bounded; on
+// timeout the CTA raises the error word, stops issuing, drains its copies and
+// frees its tensor memory.
 #include <cuda.h>
 
 #include "sp_gemm.h"
@@ -68,7 +70,7 @@ constexpr size_t kSmRecv = (size_t)kSmRecvSlots * kSmM * 16;
 constexpr size_t kSmBars = 512;
 constexpr size_t kSmSmem = 1024 + kSmRing + kSmX + kSmRecv + kSmBars;
 static_assert(kSmSmem <= 227 * 1024, "shared memory per CTA");
-static_assert((2 * kSmStages + kGemmSmallMaxKB + 2) * 8 + 8 <= (int)kSmBars, "barrier area");
+static_assert((2 * kSmStages + kGemmSmallMaxKB + 3) * 8 + 8 <= (int)kSmBars, "barrier area");
 constexpr float kUnitsPerSpike = 512.f;       // e4m3 0x01 = 2^-9
 
 // Sixteen spikes (bit i = column k0 + i) as sixteen 0 / 1 bytes.
@@ -142,12 +144,13 @@ __device__ __forceinline__ bool mma_block(uint32_t tmem, uint64_t hd, uint64_t l
 }
 
 // Stores 16 bytes into CTA `rank`'s shared memory at the address `local`
-// has in this CTA (distributed shared memory of the cluster).
-__device__ __forceinline__ void st_cluster_v4(uint32_t local, uint32_t rank, uint4 v) {
-  uint32_t addr;
-  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(addr) : "r"(local), "r"(rank));
-  asm volatile("st.shared::cluster.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(v.x),
-               "r"(v.y), "r"(v.z), "r"(v.w)
+// has in this CTA (distributed shared memory of the cluster), counted in
+// bytes on that CTA's mbarrier at the address `bar` has in this CTA.
+__device__ __forceinline__ void st_async_v4(const void* local, const uint64_t* bar, uint32_t rank,
+                                            uint4 v) {
+  asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.v4.u32 [%0], {%1, %2, %3, %4}, [%5];"
+               ::"r"(cluster_addr(local, rank)), "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w),
+               "r"(cluster_addr(bar, rank))
                : "memory");
 }
 
@@ -173,7 +176,8 @@ gemm_small_kernel(const __grid_constant__ CUtensorMap mapW, const __grid_constan
   uint64_t* xready = empty + kSmStages;  // [K block] spike operand staged (one arrival per staging warp)
   uint64_t* tfull = xready + kGemmSmallMaxKB;   // accumulator complete
   uint64_t* done = tfull + 1;            // every MMA retired (MMA thread)
-  uint32_t* s_tmem = reinterpret_cast<uint32_t*>(done + 1);
+  uint64_t* rbar = done + 1;             // the cluster's partials of this rank's groups landed
+  uint32_t* s_tmem = reinterpret_cast<uint32_t*>(rbar + 1);
   volatile int* s_abort = reinterpret_cast<volatile int*>(s_tmem + 1);
 
   const int warp = threadIdx.x >> 5;
@@ -196,8 +200,16 @@ gemm_small_kernel(const __grid_constant__ CUtensorMap mapW, const __grid_constan
     for (int b = 0; b < kGemmSmallMaxKB; ++b) mbar_init(&xready[b], kSmStageWarps);
     mbar_init(tfull, 1);
     mbar_init(done, 1);
+    mbar_init(rbar, 1);
     *s_abort = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    if (S > 1) {
+      // every rank stores its partial of each of this rank's groups (g = rank
+      // mod S) for the 128 channels: S x owned x 128 x 16 bytes
+      const int G = a.TN / 4;
+      const int owned = rank < G ? (G - 1 - rank) / S + 1 : 0;
+      mbar_arrive_expect_tx(rbar, (uint32_t)(S * owned * kSmM * 16));
+    }
     tma_prefetch_desc(&mapW);
   }
   if (warp == 1) tmem_alloc(s_tmem, kSmTmemCols);
@@ -426,16 +438,25 @@ gemm_small_kernel(const __grid_constant__ CUtensorMap mapW, const __grid_constan
 #pragma unroll
         for (int h = 0; h < 4; ++h) {
           const int g = 4 * c + h;
-          st_cluster_v4(smem_u32(&recv[(rank * gpo + g / S) * kSmM + row]), (uint32_t)(g % S),
-                        make_uint4(__float_as_uint(f[4 * h]), __float_as_uint(f[4 * h + 1]),
-                                   __float_as_uint(f[4 * h + 2]), __float_as_uint(f[4 * h + 3])));
+          st_async_v4(&recv[(rank * gpo + g / S) * kSmM + row], rbar, (uint32_t)(g % S),
+                      make_uint4(__float_as_uint(f[4 * h]), __float_as_uint(f[4 * h + 1]),
+                                 __float_as_uint(f[4 * h + 2]), __float_as_uint(f[4 * h + 3])));
         }
       }
     }
-    cluster_sync();                        // every partial is in its owner's shared memory
+  }
+  // every partial of this rank's groups is in its shared memory (no
+  // cluster-wide barrier: a CTA writes as soon as its own groups are in)
+  bool in = true;
+  if (S > 1 && epi) {
+    in = mbar_wait(rbar, 0, lim);
+    if (!in) {
+      *s_abort = 1;
+      atomicExch(a.err, kErrFlagTimeout);
+    }
   }
   // warp-uniform again (the S = 1 path reads TMEM); only the stores check m < N
-  if (epi && __all_sync(0xffffffffu, ok && !*s_abort)) {
+  if (epi && __all_sync(0xffffffffu, ok && in && !*s_abort)) {
     if (a.fault == kFaultAbort) {          // test fault: the output stays unwritten
       if (threadIdx.x == 64) atomicExch(a.err, kErrInjected);
     } else {
