@@ -120,8 +120,9 @@ def test_small_gemm_stall(down):
 
 
 def test_group_abort():
-    """A decode step's group (ticket-free cluster form) and the grouped
-    prefill (tail split: owners and helpers exchange partials behind flags)."""
+    """A decode step's group (ticket-free cluster form) at 3 and 22 blocks
+    (the latter with more CTAs than SMs) and the grouped prefill (tail split:
+    owners and helpers exchange partials behind flags)."""
     weights = synth.decode_step_weights(0, blocks=3)
     plans = [sp.Plan(to_dev(Q), to_dev(s), N, K, max_batch=256, gemm=True)
              for (Q, s, N, K) in weights]
@@ -141,7 +142,27 @@ def test_group_abort():
         group.decode(u8d, "u8", u8.shape[1], acc, y, 1536)
         return acc, y
 
+    # the whole 22-block step
+    wbig = synth.decode_step_weights(1)
+    bplans = [sp.Plan(to_dev(Q), to_dev(s), N, K) for (Q, s, N, K) in wbig]
+    big = sp.Group(bplans)
+    bKs = [w[3] for w in wbig]
+    bxs = synth.decode_step_spikes(8, bKs)
+    bu8 = np.zeros((len(bKs), max(bKs)), np.uint8)
+    for j, x in enumerate(bxs):
+        bu8[j, : x.size] = x
+    bwant = [oracle.project(Q, s, N, K, x, "u8") for (Q, s, N, K), x in zip(wbig, bxs)]
+    want_big_acc = np.concatenate([w[0] for w in bwant])
+    want_big_y = np.concatenate([w[1] for w in bwant])
+    bu8d = to_dev(bu8)
+
+    def big_step():
+        acc, y = outputs(len(bKs), 1536)
+        big.decode(bu8d, "u8", bu8.shape[1], acc, y, 1536)
+        return acc, y
+
     check_recovery(group, step, want_acc, want_y, "group decode")
+    check_recovery(big, big_step, want_big_acc, want_big_y, "group decode, 22 blocks")
 
     T = 256
     X = [synth.prefill_spikes(40 + j, T=T, K=K) for j, K in enumerate(Ks)]
@@ -161,5 +182,6 @@ def test_group_abort():
         group.inject_fault(sp.SP_FAULT_STALL)
     assert e.value.status == sp.SP_EUNSUPPORTED
     group.close()
-    for p in plans:
+    big.close()
+    for p in plans + bplans:
         p.close()

@@ -186,3 +186,39 @@ def test_cluster_layouts(p, ticket):
             assert (acc[j, N:] == 5).all(), "wrote past the member's N"
     assert group.status() == sp.SP_OK
     group.close()
+
+
+def test_large_mixed_group():
+    """24 projections of 8 shapes in one launch (ragged N and K; 1, 3 and 6
+    chunks per tile, so clusters of different layouts run side by side and
+    more CTAs than SMs are resident), spike rates from 0 to 1.  Run twice:
+    the second call must not see the first one's barriers."""
+    shapes = [(1536, 6144), (1552, 1000), (512, 1024), (2064, 3073), (16, 1), (1040, 2049),
+              (3088, 6144), (528, 200)]
+    rates = [0.1, 0.05, 1.0, 0.1, 0.5, 0.0, 0.1, 0.3]
+    cases = [(shapes[i % 8], rates[(i + i // 8) % 8]) for i in range(24)]
+
+    weights, plans, xs = [], [], []
+    for i, ((N, K), p) in enumerate(cases):
+        Qc, s, x = synth.random_case(700 + i, N, K, p=p)
+        weights.append((Qc, s, N, K))
+        plans.append(sp.Plan(to_dev(Qc), to_dev(s), N, K))
+        xs.append(x[0])
+    group = sp.Group(plans)
+    maxK = max(K for (_, K), _ in cases)
+    maxN = max(N for (N, _), _ in cases)
+    bits = np.zeros((len(cases), (maxK + 31) // 32), np.uint32)
+    for j, x in enumerate(xs):
+        b = synth.pack_bits(x)
+        bits[j, : b.size] = b
+    want = [oracle.project(Qc, s, N, K, x, "u8") for (Qc, s, N, K), x in zip(weights, xs)]
+    for rep in range(2):
+        acc = torch.full((len(cases), maxN), 5, dtype=torch.int32, device=DEV)
+        y = torch.full((len(cases), maxN), 5.0, dtype=torch.float32, device=DEV)
+        group.decode(to_dev(bits), "bits", bits.shape[1], acc, y, maxN)
+        torch.cuda.synchronize()
+        for j, (Qc, s, N, K) in enumerate(weights):
+            assert_parity(acc[j, :N], y[j, :N], want[j][0][0], want[j][1][0], f"member {j} rep {rep}")
+            assert (acc[j, N:] == 5).all(), "wrote past the member's N"
+    assert group.status() == sp.SP_OK
+    group.close()
