@@ -83,6 +83,33 @@ def test_noalloc_leaves_device_memory_alone():
 
 
 @pytest.mark.gpu
+def test_noalloc_inside_graph_capture():
+    """After the first call on the device, the entry point only enqueues its
+    kernel, so it can be captured into a CUDA graph; replays give the
+    oracle's results on whatever spike row the captured buffer holds."""
+    N, K, ldq = 1536, 6144, 1536
+    Qc, s, x = synth.random_case(451, N, K, T=3, p=0.15, ldq=ldq)
+    W, S = to_dev(Qc), to_dev(s)
+    rows = to_dev(x)
+    row = rows[0].clone()
+    acc = torch.empty(N, dtype=torch.int32, device=DEV)
+    y = torch.empty(N, dtype=torch.float32, device=DEV)
+    sp.spike_proj_decode_noalloc(W, ldq, S, N, K, row, "u8", acc, y)   # first call: outside capture
+    torch.cuda.synchronize()
+    stream = torch.cuda.Stream()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        sp.spike_proj_decode_noalloc(W, ldq, S, N, K, row, "u8", acc, y,
+                                     stream=torch.cuda.current_stream())
+    want_acc, want_y = oracle.project(Qc, s, N, K, x, "u8", ldq=ldq)
+    for t in (1, 2, 0):
+        row.copy_(rows[t])
+        g.replay()
+        torch.cuda.synchronize()
+        assert_parity(acc, y, want_acc[t], want_y[t], f"graph replay on row {t}")
+
+
+@pytest.mark.gpu
 def test_noalloc_rejects_n_above_the_scratch():
     N, K = sp.SPIKE_PROJ_NOALLOC_MAX_N + 16, 64
     W = torch.zeros((K, N), dtype=torch.int8, device=DEV)
