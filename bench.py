@@ -223,7 +223,9 @@ def make_step_inputs(rank):
 def config_of(active_bytes_per_step):
     """The workload description both arms print (identical keys and values)."""
     return {"workload": WORKLOAD, "global_batch": 1,
-            "active_bytes_per_step": float(active_bytes_per_step)}
+            "active_bytes_per_step": float(active_bytes_per_step),
+            "l2": f"inputs larger than L2: {WEIGHT_COPIES} rotating copies of the weights "
+                  f"and {SPIKE_SETS} rotating spike sets"}
 
 
 def cpu_baseline_decode(weights, sets, seconds, channels=None):
