@@ -331,9 +331,11 @@ sp_status spike_proj_group_status(sp_group_t group, sp_stream_t stream);
  * SPIKE_PROJ_NOALLOC_MAX_N INT32 words plus one word per 512 outputs), so N is
  * limited to SPIKE_PROJ_NOALLOC_MAX_N; a larger N returns SP_ESCRATCH before
  * anything is enqueued.  No cudaMalloc, cudaFree or other allocating call is
- * made, on the first call or later.  The kernel it runs cannot fail once
- * launched (it has no waits and no error path) and returns the scratch to
- * zero, so nothing has to be cleared between calls.
+ * made, on the first call or later.  The kernel it runs returns the scratch
+ * to zero, so nothing has to be cleared between calls.  Its only wait is
+ * bounded (about a second, for the partial sums of the other CTAs of its
+ * thread-block cluster); should that wait ever run out, acc and y are left
+ * unwritten and nothing reports it: this entry point has no status word.
  *
  * First call per device: it checks the device, looks up the scratch address
  * on the current device, clears the scratch on `stream` (defensively: it is

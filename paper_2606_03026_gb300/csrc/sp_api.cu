@@ -858,7 +858,7 @@ sp_status spike_proj_decode_noalloc(const int8_t* W, int64_t ldw, const float* s
   g.ld_out = N;
   g.ws = scratch;
   g.tickets = reinterpret_cast<uint32_t*>(scratch + kNoallocMaxN);
-  g.err = nullptr;                        // the gather kernel never raises one
+  g.err = nullptr;                        // no status word: see the header
   SP_CUDA(launch_gather(g, s));
   return SP_OK;
 }

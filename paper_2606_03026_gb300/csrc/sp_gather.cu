@@ -474,7 +474,7 @@ gather_cluster_kernel(const __grid_constant__ GatherParamsT<NP> p) {
   // the owner's threads wait for the kch partials of their groups (no
   // cluster-wide barrier: a CTA goes on as soon as its own groups are in)
   if ((int)threadIdx.x < per && !mbar_wait(&s_bar, 0)) {
-    atomicExch(p.err, kErrFlagTimeout);
+    if (p.err) atomicExch(p.err, kErrFlagTimeout);   // (the allocation-free call has none)
     return;
   }
   if (p.fault == kFaultAbort) {             // test fault: the output stays unwritten
