@@ -425,51 +425,49 @@ gather_cluster_kernel(const __grid_constant__ GatherParamsT<NP> p) {
   int n = 0;
   bool owner = false;
   float4 sc = float4{};
-  if (work) {
-    if constexpr (kLif) {
-      // fused spike producer: one LIF step of this chunk's neurons (every CTA
-      // of the chunk computes the same words from the old state; the CTA of
-      // tile slot 0 in cluster 0 writes the new state and the bits)
-      const int k0 = kc * P.ck;
-      const float* vr = p.lif_vin + (int64_t)j * p.lif_ld;
-      const float* ir = p.lif_I + (int64_t)j * p.lif_ld;
-      const bool writer = cl == 0 && ts == 0;
-      for (int i = threadIdx.x; i < P.ck; i += kGatherClusterThreads) {   // warp-uniform: ck % 32 == 0
-        const int k = k0 + i;
-        bool fire = false;
-        if (k < P.K) {
-          float u = fmaf(p.lif_beta, vr[k], ir[k]);
-          fire = u >= p.lif_theta;
-          if (fire) u = __fsub_rn(u, p.lif_theta);
-          if (writer) p.lif_vout[(int64_t)j * p.lif_ld + k] = u;
-        }
-        const uint32_t w = __ballot_sync(0xffffffffu, fire);
-        if ((threadIdx.x & 31) == 0) {
-          s_lif[i >> 5] = w;
-          if (writer && p.lif_bits && k < P.K) p.lif_bits[(int64_t)j * p.lif_ld_bits + (k >> 5)] = w;
-        }
+  if constexpr (kLif) {
+    // fused spike producer: one LIF step of this chunk's neurons (every CTA
+    // of the chunk computes the same words from the old state; the CTA of
+    // tile slot 0 in cluster 0 writes the new state and the bits)
+    const int k0 = kc * P.ck;
+    const float* vr = p.lif_vin + (int64_t)j * p.lif_ld;
+    const float* ir = p.lif_I + (int64_t)j * p.lif_ld;
+    const bool writer = cl == 0 && ts == 0;
+    for (int i = threadIdx.x; i < P.ck; i += kGatherClusterThreads) {   // warp-uniform: ck % 32 == 0
+      const int k = k0 + i;
+      bool fire = false;
+      if (k < P.K) {
+        float u = fmaf(p.lif_beta, vr[k], ir[k]);
+        fire = u >= p.lif_theta;
+        if (fire) u = __fsub_rn(u, p.lif_theta);
+        if (writer) p.lif_vout[(int64_t)j * p.lif_ld + k] = u;
       }
-      __syncthreads();
+      const uint32_t w = __ballot_sync(0xffffffffu, fire);
+      if ((threadIdx.x & 31) == 0) {
+        s_lif[i >> 5] = w;
+        if (writer && p.lif_bits && k < P.K) p.lif_bits[(int64_t)j * p.lif_ld_bits + (k >> 5)] = w;
+      }
     }
-    unit_partial<kGatherClusterWarps, kGatherClusterMaxCK, kClusterLoads, cluster_slots<CL>()>(
-        sm, P, kLif ? nullptr : spike_row(p.spikes, p.fmt, j, p.ld_spikes), p.fmt, n0, kc * P.ck,
-        P.ck, kLif ? s_lif : nullptr);
-    // the owner's scales, read now: their load overlaps the cluster exchange
-    // instead of following the last barrier
-    {
-      const int g_own = kc * per + (int)threadIdx.x;
-      n = n0 + 4 * g_own;
-      owner = (int)threadIdx.x < per && g_own < kGatherNT / 4 && n < P.N;
-    }
-    if (owner && p.y) sc = scale4(P, n);
-    asm volatile("barrier.cluster.wait;" ::: "memory");
-    const int g = threadIdx.x;              // the 4-channel group of this thread
-    if (g < kGatherNT / 4) {
-      const int4 v = unit_sum4(sm, 4 * g);
-      const int o = g / per;                // the owning chunk
-      const uint32_t dst = (uint32_t)(ts * kch + o);
-      st_async_v4(cluster_addr(&s_recv[kc * per + (g - o * per)], dst), cluster_addr(&s_bar, dst), v);
-    }
+    __syncthreads();
+  }
+  unit_partial<kGatherClusterWarps, kGatherClusterMaxCK, kClusterLoads, cluster_slots<CL>()>(
+      sm, P, kLif ? nullptr : spike_row(p.spikes, p.fmt, j, p.ld_spikes), p.fmt, n0, kc * P.ck,
+      P.ck, kLif ? s_lif : nullptr);
+  // the owner's scales, read now: their load overlaps the exchange instead
+  // of following the owner's wait
+  {
+    const int g_own = kc * per + (int)threadIdx.x;
+    n = n0 + 4 * g_own;
+    owner = (int)threadIdx.x < per && g_own < kGatherNT / 4 && n < P.N;
+  }
+  if (owner && p.y) sc = scale4(P, n);
+  asm volatile("barrier.cluster.wait;" ::: "memory");
+  const int g = threadIdx.x;              // the 4-channel group of this thread
+  if (g < kGatherNT / 4) {
+    const int4 v = unit_sum4(sm, 4 * g);
+    const int o = g / per;                // the owning chunk
+    const uint32_t dst = (uint32_t)(ts * kch + o);
+    st_async_v4(cluster_addr(&s_recv[kc * per + (g - o * per)], dst), cluster_addr(&s_bar, dst), v);
   }
   // the owner's threads wait for the kch partials of their groups (no
   // cluster-wide barrier: a CTA goes on as soon as its own groups are in)
