@@ -76,6 +76,28 @@ def test_ragged_shapes(N, K, ldq, p):
         assert_parity(acc, y, want_acc[t], want_y[t], f"N={N} K={K} u8 t={t}")
 
 
+# One shape for each cluster layout a single projection can take: (cluster
+# size, chunks per tile) = (6, 1), (6, 2), (6, 6), (12, 3), (12, 6),
+# (12, 12), (16, 1), (16, 2), (16, 4), (16, 8), (16, 16).  In each, every
+# chunk's CTA stores its partial of each 4-channel group into the owning
+# chunk's shared memory and the owner waits for kch x its groups' bytes.
+@pytest.mark.parametrize("N,K", [(2576, 1), (1040, 600), (16, 1536), (2048, 768), (1040, 1536),
+                                 (16, 3072), (6144, 1), (2576, 600), (1040, 1000), (1040, 2049),
+                                 (16, 4100)])
+def test_cluster_layouts_single(N, K):
+    Qc, s, x = synth.random_case(900 + K % 101 + N % 7, N, K, T=2, p=0.3)
+    x[1] = 1                                 # every column active: the largest sums
+    want_acc, want_y = oracle.project(Qc, s, N, K, x, "u8")
+    plan = sp.Plan(to_dev(Qc), to_dev(s), N, K)
+    bits = synth.pack_bits(x)
+    for t in range(2):
+        for fmt, rows in (("bits", bits), ("u8", x)):
+            acc, y = run_decode(plan, to_dev(rows[t]), fmt, N)
+            assert_parity(acc, y, want_acc[t], want_y[t], f"N={N} K={K} row {t} {fmt}")
+    assert plan.status() == sp.SP_OK
+    plan.close()
+
+
 def test_one_hot_every_position():
     """e_k for every k of a ragged K: the output is column k times the scale."""
     N, K = 64, 300
