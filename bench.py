@@ -340,7 +340,7 @@ def run_ours(args):
     for (Q, _, _, _) in weights:
         offs.append(tot)
         tot += (Q.nbytes + 255) // 256 * 256
-    copy_bufs = []
+    copy_bufs, copy_plans = [], []
     for c in range(n_copies):
         buf = torch.empty(tot, dtype=torch.int8, device=dev)
         plans = []
@@ -350,6 +350,7 @@ def run_ours(args):
             Sd = torch.from_numpy(s).to(dev)
             plans.append(sp.Plan(Wd, Sd, N, K))
         copies.append(sp.Group(plans))
+        copy_plans.append(plans)
         copy_bufs.append(buf)
     weight_bytes = sum(Q.nbytes for (Q, _, _, _) in weights)
     spikes = torch.from_numpy(sets_np).to(dev)
@@ -436,6 +437,19 @@ def run_ours(args):
             stream.synchronize()
     t_wall2 = time.time()
     sampler.stop()
+    # the replayed steps kept their results: the last replay of the full
+    # graph ended on its step GRAPH_STEPS - 1, whose 44 outputs must equal
+    # those of 44 separate single-projection launches on the same inputs
+    # (a different cluster layout of the gather)
+    last = GRAPH_STEPS - 1
+    acc1 = torch.empty_like(acc)
+    y1 = torch.empty_like(y)
+    with torch.cuda.stream(stream):
+        for j, pl in enumerate(copy_plans[last % n_copies]):
+            pl.decode(spikes[last % SPIKE_SETS, j], "bits", acc1[j], y1[j], stream=stream)
+    stream.synchronize()
+    assert torch.equal(acc1, acc) and torch.equal(y1.view(torch.int32), y.view(torch.int32)), \
+        "the timed steps' outputs differ from single launches"
     elapsed_ms = ev0.elapsed_time(ev1)
     elapsed_ms = reduce_max(elapsed_ms, world)
     bytes_per_step = float(active.mean())
