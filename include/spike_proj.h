@@ -495,18 +495,23 @@ sp_status spike_proj_head(sp_head_t head, const float *h, int64_t ldh, int32_t B
  *                   without writing its outputs and without cleaning its
  *                   workspace (split-K partials and tile tickets stay dirty),
  *                   as a kernel that failed half way would.
- *   SP_FAULT_STALL  plans only, and only a tensor-core (SP_GEMM) launch: one
- *                   TMA copy of the first CTA is never issued, and every wait
- *                   of that launch is bounded by about 2 ms instead of 1 s, so
+ *   SP_FAULT_STALL  a wait that runs out, in the kernels that wait on other
+ *                   CTAs.  A tensor-core launch of a plan (SP_GEMM): one TMA
+ *                   copy of the first CTA is never issued, and every wait of
+ *                   that launch is bounded by about 2 ms instead of 1 s, so
  *                   the MMA's wait for the missing copy runs out: the kernel
  *                   raises the error word, stops issuing, drains the copies
- *                   it issued and frees its tensor memory.  Other kernels
+ *                   it issued and frees its tensor memory.  A batch-1 decode
+ *                   of a plan or group in thread-block clusters: the first
+ *                   CTA never stores its partial sums into the owners'
+ *                   shared memory, and the owners' waits (bounded by about
+ *                   2 ms) run out: the kernel raises the error word and those
+ *                   owners leave their outputs unwritten.  Other kernels
  *                   ignore it (it is still disarmed by their launch).
  * No fault traps, faults the GPU or spins without bound.  spike_proj_plan_status
  * / spike_proj_group_status then return SP_EKERNEL, clear the error word and
  * re-zero the workspace, and the next call is exact again.
- * Errors: SP_EINVAL (NULL, unknown fault), SP_EUNSUPPORTED (a stall on a
- * group).
+ * Errors: SP_EINVAL (NULL, unknown fault).
  * ------------------------------------------------------------------------- */
 typedef enum sp_fault {
     SP_FAULT_NONE = 0,

@@ -871,7 +871,6 @@ sp_status spike_proj_plan_inject_fault(sp_plan_t plan, int32_t fault) {
 
 sp_status spike_proj_group_inject_fault(sp_group_t group, int32_t fault) {
   if (!group || fault < SP_FAULT_NONE || fault > SP_FAULT_STALL) return SP_EINVAL;
-  if (fault == SP_FAULT_STALL) return SP_EUNSUPPORTED;
   group->fault = fault;
   return SP_OK;
 }

@@ -463,7 +463,10 @@ gather_cluster_kernel(const __grid_constant__ GatherParamsT<NP> p) {
   if (owner && p.y) sc = scale4(P, n);
   asm volatile("barrier.cluster.wait;" ::: "memory");
   const int g = threadIdx.x;              // the 4-channel group of this thread
-  if (g < kGatherNT / 4) {
+  // test stall: the first CTA's partials are never stored, so its tile's
+  // owners wait until their (shortened) bound runs out
+  const bool stall = p.fault == kFaultStall;
+  if (g < kGatherNT / 4 && !(stall && blockIdx.x == 0 && blockIdx.y == 0)) {
     const int4 v = unit_sum4(sm, 4 * g);
     const int o = g / per;                // the owning chunk
     const uint32_t dst = (uint32_t)(ts * kch + o);
@@ -471,7 +474,7 @@ gather_cluster_kernel(const __grid_constant__ GatherParamsT<NP> p) {
   }
   // the owner's threads wait for the kch partials of their groups (no
   // cluster-wide barrier: a CTA goes on as soon as its own groups are in)
-  if ((int)threadIdx.x < per && !mbar_wait(&s_bar, 0)) {
+  if ((int)threadIdx.x < per && !mbar_wait(&s_bar, 0, stall ? kStallWaitCycles : kWaitLimitCycles)) {
     if (p.err) atomicExch(p.err, kErrFlagTimeout);   // (the allocation-free call has none)
     return;
   }

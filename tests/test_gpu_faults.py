@@ -85,6 +85,23 @@ def test_decode_abort(down):
     check_recovery(plan, call, want_acc, want_y, "decode")
 
 
+def test_decode_stall(down):
+    """Batch-1 decode in clusters: the first CTA never stores its partial
+    sums into the owners' shared memory, and the owners' bounded waits for
+    them run out (about 2 ms under the stall fault)."""
+    Qc, s, plan = down
+    _, _, x = synth.random_case(20, 1536, 6144, T=1, p=0.1)
+    want_acc, want_y = oracle.project(Qc, s, 1536, 6144, x, "u8")
+    xd = to_dev(x[0])
+
+    def call():
+        acc, y = outputs(1, 1536)
+        plan.decode(xd, "u8", acc[0], y[0])
+        return acc, y
+
+    check_recovery(plan, call, want_acc, want_y, "decode stall", fault=sp.SP_FAULT_STALL)
+
+
 def test_gemm_stall(down):
     """512-token prefill on the tensor cores (split-K clusters): one TMA copy
     is never issued and the MMA warp's bounded wait runs out; the kernel
@@ -104,8 +121,9 @@ def test_gemm_stall(down):
 
 def test_small_gemm_stall(down):
     """A few rows on the tensor cores (the small-T form, K split over a
-    cluster): CTA 0's first weight box is never issued, its MMA thread's
-    bounded wait runs out, and the cluster still completes its barriers."""
+    cluster): CTA 0's first weight box is never issued and its MMA thread's
+    bounded wait runs out; it stores no partials, so the owners' bounded
+    waits for them run out too."""
     Qc, s, plan = down
     _, _, x = synth.random_case(19, 1536, 6144, T=5, p=0.15)
     want_acc, want_y = oracle.project(Qc, s, 1536, 6144, x, "u8")
@@ -121,8 +139,9 @@ def test_small_gemm_stall(down):
 
 def test_group_abort():
     """A decode step's group (ticket-free cluster form) at 3 and 22 blocks
-    (the latter with more CTAs than SMs) and the grouped prefill (tail split:
-    owners and helpers exchange partials behind flags)."""
+    (the latter with more CTAs than SMs), aborted and stalled, and the
+    grouped prefill (tail split: owners and helpers exchange partials behind
+    flags)."""
     weights = synth.decode_step_weights(0, blocks=3)
     plans = [sp.Plan(to_dev(Q), to_dev(s), N, K, max_batch=256, gemm=True)
              for (Q, s, N, K) in weights]
@@ -163,6 +182,9 @@ def test_group_abort():
 
     check_recovery(group, step, want_acc, want_y, "group decode")
     check_recovery(big, big_step, want_big_acc, want_big_y, "group decode, 22 blocks")
+    check_recovery(group, step, want_acc, want_y, "group decode stall", fault=sp.SP_FAULT_STALL)
+    check_recovery(big, big_step, want_big_acc, want_big_y, "group decode stall, 22 blocks",
+                   fault=sp.SP_FAULT_STALL)
 
     T = 256
     X = [synth.prefill_spikes(40 + j, T=T, K=K) for j, K in enumerate(Ks)]
@@ -178,9 +200,13 @@ def test_group_abort():
         return torch.stack(accs), torch.stack(ys)
 
     check_recovery(group, prefill, wantp_acc, wantp_y, "group prefill")
-    with pytest.raises(sp.SpikeProjError) as e:
-        group.inject_fault(sp.SP_FAULT_STALL)
-    assert e.value.status == sp.SP_EUNSUPPORTED
+    # the grouped prefill does not wait on other CTAs' copies: it ignores a
+    # stall, which its launch still disarms
+    group.inject_fault(sp.SP_FAULT_STALL)
+    acc, y = prefill()
+    torch.cuda.synchronize()
+    assert_parity(acc, y, wantp_acc, wantp_y, "group prefill under an armed stall")
+    assert group.status() == sp.SP_OK
     group.close()
     big.close()
     for p in plans + bplans:
