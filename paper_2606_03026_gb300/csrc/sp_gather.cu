@@ -629,16 +629,25 @@ bool cluster_form(GatherParamsT<NP>& q, int* grid_x, int* grid_y, int* cl_out) {
   return true;
 }
 
-// Sets the one-time attributes of a cluster-form kernel: the largest
-// shared-memory carveout (the resident-cluster count depends on it) and, for
-// clusters above 8 CTAs, the non-portable cluster size.
+// Sets the one-time attributes of a cluster-form kernel, once per device: the
+// largest shared-memory carveout (the resident-cluster count depends on it),
+// for clusters above 8 CTAs the non-portable cluster size, and the dynamic
+// shared memory above 48 KB.  (Each is a driver call of about a microsecond:
+// set on every launch they made a single decode's host time the bound.)
 template <typename Kern>
 cudaError_t cluster_attrs(Kern kernel, int CL, size_t smem, std::atomic<uint64_t>& done) {
-  cudaError_t e = set_carveout(kernel, done);
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  const uint64_t bit = dev < 64 ? (uint64_t)1 << dev : 0;
+  if (bit && (done.load(std::memory_order_relaxed) & bit)) return cudaSuccess;
+  e = cudaFuncSetAttribute(kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
+                           (int)cudaSharedmemCarveoutMaxShared);
   if (e == cudaSuccess && CL > 8)
     e = cudaFuncSetAttribute(kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
   if (e == cudaSuccess && smem > 48 * 1024)
     e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e == cudaSuccess && bit) done.fetch_or(bit, std::memory_order_relaxed);
   return e;
 }
 

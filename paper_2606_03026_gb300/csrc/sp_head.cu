@@ -652,10 +652,17 @@ cudaError_t launch_head_t(HeadParams p, cudaStream_t s) {
   const size_t smem = (size_t)kHeadWarps * kHeadList * 8 + (size_t)B * p.Kpad;
   cudaError_t e = raise_smem(head_kernel<B>, smem, set_proj);
   if (e != cudaSuccess) return e;
-  int per_sm = 0;
-  e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, head_kernel<B>, kHeadThreads, smem);
-  if (e != cudaSuccess) return e;
-  if (per_sm < 1) per_sm = 1;
+  // resident CTAs per SM, queried once per shared-memory size (a driver
+  // call of about a microsecond)
+  static int per_sm = 0;
+  static size_t per_sm_smem = 0;
+  if (per_sm == 0 || per_sm_smem != smem) {
+    int n = 0;
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, head_kernel<B>, kHeadThreads, smem);
+    if (e != cudaSuccess) return e;
+    per_sm = n < 1 ? 1 : n;
+    per_sm_smem = smem;
+  }
   // one wave: every CTA resident at once
   int grid = g_head_sms * per_sm;
   const int need = (p.units + kHeadWarps - 1) / kHeadWarps;
