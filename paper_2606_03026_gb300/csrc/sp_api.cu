@@ -207,8 +207,53 @@ GatherParams1 single_params(const sp_plan_s* p, const void* spikes, int fmt, int
   return g;
 }
 
+// Several rows of one plan as a group of that many one-row problems sharing
+// W: the group launch then runs them in the cluster form (each row's tiles x
+// chunks in clusters, partials exchanged in shared memory) when every
+// cluster can be resident at once, and in the ticket form otherwise.  The
+// workspace and ticket offsets (row t: ws + t N, tickets + t ntiles) are the
+// batched ticket form's, so the plan's workspace serves both.
+GatherParamsG rows_as_group(const sp_plan_s* p, const void* spikes, int fmt, int B, int64_t ld,
+                            int32_t* acc, float* y) {
+  GatherParamsG g;
+  std::memset(&g, 0, sizeof(g));
+  const int units = gather_units(p->N, p->K);
+  for (int t = 0; t < B; ++t) {
+    GatherProblem& P = g.prob[t];
+    P.W = p->W;
+    P.scale = p->scale;
+    P.ldw = (int32_t)p->ldw;
+    P.N = p->N;
+    P.K = p->K;
+    P.unit_begin = t * units;
+    P.ws_begin = t * p->N;
+    P.ticket_begin = t * gather_ntiles(p->N);
+  }
+  g.nprob = B;
+  g.B = 1;
+  g.units_total = B * units;
+  g.max_units = units;
+  g.fmt = fmt;
+  g.spikes = spikes;
+  g.ld_spikes = ld;
+  g.acc = acc;
+  g.y = y;
+  g.ld_out = p->N;
+  g.ws = p->ws;
+  g.tickets = p->tickets;
+  g.err = p->err;
+  return g;
+}
+
 sp_status run_gather(sp_plan_s* p, const void* spikes, int fmt, int B, int64_t ld, int32_t* acc,
                      float* y, cudaStream_t s) {
+  if (B > 1 && B <= kMaxProblems && (int64_t)B * p->N <= INT32_MAX) {
+    GatherParamsG g = rows_as_group(p, spikes, fmt, B, ld, acc, y);
+    g.fault = p->fault;
+    p->fault = 0;
+    SP_CUDA(launch_gather(g, s));
+    return SP_OK;
+  }
   GatherParams1 g = single_params(p, spikes, fmt, B, ld, acc, y);
   g.fault = p->fault;
   p->fault = 0;
@@ -307,8 +352,10 @@ sp_status run_gemm(sp_plan_s* p, const void* spikes, int fmt, int T, int64_t ld,
 //                   (ceil(Kp / 64 / S), S = the cluster size) + 0.045 us per row
 //   GEMM, T > 64  ~ max(11.3 us + 2 B N K ops / 1.4 PFLOP/s, 8.5 us + 0.55 us per 1024 of K)
 // (the GEMM only for SP_PLAN_GEMM plans).  Measured at 1536 x 6144: gather
-// 4.2 / 6.7 / 9.0 / 11.6 / 16.5 us at B = 1 / 8 / 16 / 32 / 64, small-T GEMM
-// 7.2 / 7.2 / 7.3 / 8.0 / 9.4 us, the 128-row GEMM 12.1 us at B = 65 .. 128
+// 4.2 / 6.7 / 9.0 / 11.6 / 16.5 us at B = 1 / 8 / 16 / 32 / 64 in the ticket
+// form, and 6.0 / 7.6 / 9.3 us at B = 8 / 16 / 32 with the rows run as a
+// group (the model's choices are the same for both), small-T GEMM
+// 7.2 / 7.2 / 7.3 / 8.0 / 9.2 us, the 128-row GEMM 12.1 us at B = 65 .. 128
 // (17.5 us at K = 16384); at 1536 x 1536 the small-T GEMM wins from B = 4
 // (4.5 against 5.4 us).  The union fetch is never chosen automatically: it
 // was slower than the per-token gather at every batch size measured (its

@@ -128,6 +128,31 @@ def test_gemm_bool8_rows(T, N, K):
     assert plan.status() == sp.SP_OK
 
 
+@pytest.mark.parametrize("T,N,K", [(2, 1536, 6144), (5, 272, 1000), (17, 1552, 777), (33, 1536, 6144),
+                                   (64, 528, 3073), (65, 1040, 2049), (3, 2064, 8000), (9, 16, 1)])
+def test_gather_rows(T, N, K):
+    """The gather strategy on T rows: up to 64 rows run as a group of
+    one-row problems (the cluster form when every cluster fits at once, else
+    the ticket form with the batched form's workspace offsets; K above 6144
+    is always the ticket form), more than 64 in the batched ticket form.
+    Rows of mixed rates, every format, twice in a row (the second call must
+    find the workspace and tickets clean)."""
+    rng = synth.rng_for(95, T, N, K)
+    Qc, s, _ = synth.random_case(96 + T, N, K, T=1)
+    rates = rng.uniform(0.0, 0.4, size=(T, 1))
+    rates[0] = 1.0
+    X = (rng.random((T, K)) < rates).astype(np.uint8)
+    want_acc, want_y = oracle.project(Qc, s, N, K, X, "u8")
+    plan = sp.Plan(to_dev(Qc), to_dev(s), N, K, max_batch=T)
+    bits = synth.pack_bits(X)
+    for rep in range(2):
+        for fmt, rows, ld in (("bits", bits, bits.shape[1]), ("u8", X, K)):
+            acc, y = run_batched(plan, to_dev(rows), fmt, T, ld, N, "gather")
+            assert_parity(acc, y, want_acc, want_y, f"T={T} N={N} K={K} {fmt} rep {rep}")
+    assert plan.status() == sp.SP_OK
+    plan.close()
+
+
 def test_gemm_extremes():
     """All-ones spikes against -128 / +127 weights: the largest sums the
     tensor-core path must carry exactly (|acc| = 128 * K)."""

@@ -53,21 +53,23 @@ def check_recovery(plan_or_group, call, want_acc, want_y, what, fault=sp.SP_FAUL
     assert plan_or_group.status() == sp.SP_OK
 
 
-@pytest.mark.parametrize("strategy", ["gather", "union", "gemm"])
-def test_batched_abort(down, strategy):
-    """B = 5 rows: the per-token gather's ticket form (12 chunks per tile),
-    the union fetch and the tensor-core GEMM, each stopped half way."""
+@pytest.mark.parametrize("strategy,T", [("gather", 5), ("gather", 64), ("union", 5), ("gemm", 5)])
+def test_batched_abort(down, strategy, T):
+    """The per-token gather at T = 5 rows (the cluster form: rows as a group
+    of one-row problems) and T = 64 (more clusters than can be resident: the
+    ticket form, 12 chunks per tile, workspace and tickets left dirty), the
+    union fetch and the tensor-core GEMM, each stopped half way."""
     Qc, s, plan = down
-    _, _, x = synth.random_case(17, 1536, 6144, T=5, p=0.15)
+    _, _, x = synth.random_case(17, 1536, 6144, T=T, p=0.15)
     want_acc, want_y = oracle.project(Qc, s, 1536, 6144, x, "u8")
     xd = to_dev(x)
 
     def call():
-        acc, y = outputs(5, 1536)
-        plan.batched(xd, "u8", 5, 6144, acc, y, strategy)
+        acc, y = outputs(T, 1536)
+        plan.batched(xd, "u8", T, 6144, acc, y, strategy)
         return acc, y
 
-    check_recovery(plan, call, want_acc, want_y, f"batched {strategy}")
+    check_recovery(plan, call, want_acc, want_y, f"batched {strategy} T={T}")
 
 
 def test_decode_abort(down):
