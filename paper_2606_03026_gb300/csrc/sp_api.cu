@@ -346,7 +346,7 @@ sp_status run_gemm(sp_plan_s* p, const void* spikes, int fmt, int T, int64_t ld,
 // tensor-core GEMM, by a cost model fitted on GB300 (token rates
 // U(0.05, 0.2), weights L2-resident, graph-timed, N x K in {1536 x 6144,
 // 1536 x 1536, 4096 x 1536, 1536 x 16384}, B = 1 .. 256):
-//   gather        ~ 4.2 us + 0.08 us per row after the first
+//   gather        ~ 3.9 us + 0.08 us per row after the first
 //                   + active bytes (sum_t |A_t| * N) / 6.7 TB/s
 //   GEMM, T <= 64 ~ 3.4 us + 0.33 us per K block of a CTA's K range
 //                   (ceil(Kp / 64 / S), S = the cluster size) + 0.045 us per row
@@ -354,16 +354,16 @@ sp_status run_gemm(sp_plan_s* p, const void* spikes, int fmt, int T, int64_t ld,
 // (the GEMM only for SP_PLAN_GEMM plans).  Measured at 1536 x 6144: gather
 // 4.2 / 6.7 / 9.0 / 11.6 / 16.5 us at B = 1 / 8 / 16 / 32 / 64 in the ticket
 // form, and 6.0 / 7.6 / 9.3 us at B = 8 / 16 / 32 with the rows run as a
-// group (the model's choices are the same for both), small-T GEMM
+// group (the fixed term fitted to the latter: 4.2 us before), small-T GEMM
 // 7.2 / 7.2 / 7.3 / 8.0 / 9.2 us, the 128-row GEMM 12.1 us at B = 65 .. 128
-// (17.5 us at K = 16384); at 1536 x 1536 the small-T GEMM wins from B = 4
-// (4.5 against 5.4 us).  The union fetch is never chosen automatically: it
+// (17.5 us at K = 16384); at 1536 x 1536 the gather (rows as a group) wins
+// up to B = 6 (3.6 against 4.5 us at B = 4) and the small-T GEMM from B = 8.  The union fetch is never chosen automatically: it
 // was slower than the per-token gather at every batch size measured (its
 // adds are ALU-bound, and the 126 MB L2 serves the per-token re-reads of a
 // 9.4 MB weight matrix).
 sp_kernel choose(const sp_plan_s* p, int B, int32_t total) {
   if (!(p->flags & SP_PLAN_GEMM)) return SP_GATHER;
-  const double gather_us = 4.2 + 0.08 * (B - 1) + (double)total * p->N / 6.7e6;
+  const double gather_us = 3.9 + 0.08 * (B - 1) + (double)total * p->N / 6.7e6;
   double gemm_us;
   const int nkb = p->Kp / 64;
   if (const int S = gemm_small_splits(B, p->N, p->Kp))

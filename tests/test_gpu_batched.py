@@ -213,8 +213,9 @@ def test_auto_dispatch_by_cost(down):
 
 def test_auto_dispatch_second_shape():
     """A 1536 x 1536 projection (the sequence-mixer shape): the small-T
-    tensor-core form already beats the gather at B = 16, a single row
-    stays on the gather, and every choice is exact against the oracle."""
+    tensor-core form beats the gather at B = 16, one row and four rows stay
+    on the gather (rows run as a group in the cluster form), and every
+    choice is exact against the oracle."""
     c = synth.single_projection(4)
     Qc, s = c["Q"], c["s"]
     plan = sp.Plan(to_dev(Qc), to_dev(s), 1536, 1536, max_batch=64, gemm=True)
@@ -222,7 +223,7 @@ def test_auto_dispatch_second_shape():
     X = (np.random.default_rng(6).random((64, 1536)) < rates).astype(np.uint8)
     want_acc, want_y = oracle.project(Qc, s, 1536, 1536, X, "u8")
     bits = to_dev(synth.pack_bits(X))
-    for B, expect in ((1, "gather"), (16, "gemm"), (64, "gemm")):
+    for B, expect in ((1, "gather"), (4, "gather"), (16, "gemm"), (64, "gemm")):
         acc, y = run_batched(plan, bits, "bits", B, bits.shape[1], 1536, "auto")
         assert plan.last_dispatch()[0] == expect, (B, plan.last_dispatch())
         assert_parity(acc, y, want_acc[:B], want_y[:B], f"1536 x 1536 auto B={B}")
